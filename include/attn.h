@@ -1,0 +1,148 @@
+/*
+ * attn.h -- C ABI of the GB300 (sm_103a) three-stage attention library.
+ *
+ * The library implements the per-layer attention block of the paper's three
+ * static-shape stages (arxiv 2607.15865, Section 4; Table 1):
+ *
+ *   prefill     a prompt of chunk_len tokens attends causally to itself
+ *               (Section 4.2, with_history=False; Listing 1);
+ *   prefill_kv  a chunk of chunk_len new tokens attends to hist_len history
+ *               tokens already in the cache plus itself, causally
+ *               (Section 4.3, with_history=True; Listing 2);
+ *   decode      one new token per sequence attends to the hist_len[b] valid
+ *               tokens of a static-maximum-length cache plus itself
+ *               (Section 4.4; the runtime-filled mask is given as lengths).
+ *
+ * Every stage rotates q and k with RoPE using cos/sin gathered from a table
+ * precomputed per position (Listing 1 "Gather"/"Rope"; Section 4.6.2), writes the
+ * rotated k and the unchanged v of the new tokens into the caller's cache in
+ * place (Listing 2 "Concat"; Section 4.6.3), and computes scaled dot-product
+ * attention with scale 1/sqrt(head_dim) (FAttention, Section 2.2) under the
+ * causal mask (Section 4.6.1).  Grouped-query attention: query head h reads kv
+ * head h / (n_q_heads / n_kv_heads).
+ *
+ * Numerics: the table holds cos/sin of p*theta^(-2j/D) (element j paired with
+ * j + D/2) computed in double and rounded to float; RoPE runs in float and the
+ * rotated q and k are rounded to bf16 (nearest even); scores, softmax and the
+ * value sum accumulate in float; out is rounded to bf16 (nearest even).
+ *
+ * Data types and layouts.  "bf16" below is a pointer to bf16 values given as
+ * their 16-bit patterns (uint16_t), all in device memory, densely packed:
+ *   q    [batch, chunk_len, n_q_heads,  head_dim]
+ *   k, v [batch, chunk_len, n_kv_heads, head_dim]
+ *   k_cache, v_cache [batch, n_kv_heads, max_len, head_dim]
+ *   out  [batch, chunk_len, n_q_heads,  head_dim]
+ * Decode uses chunk_len = 1.  All device pointers must be 16-byte aligned.
+ *
+ * Ownership.  The caller owns every device buffer passed to a call.  The
+ * context owns only its own device memory: the RoPE tables (2 x max_len x
+ * head_dim/2 floats), the decode split-KV partials (batch x n_q_heads x 256 x
+ * (head_dim + 2) floats) and a device error word; all allocated by attn_create
+ * and freed by attn_destroy.  No stage call allocates, frees or synchronises: each one only
+ * enqueues kernels on `stream` and returns.  Calls that use the same context
+ * share its scratch buffers, so they must not run concurrently on different
+ * streams.
+ *
+ * Errors.  Every int-returning call returns ATTN_OK (0) or a negative code and
+ * writes nothing when it rejects its arguments.  Launch failures return
+ * ATTN_ECUDA (attn_last_cuda_error_string() gives the runtime's text).  The
+ * decode lengths live on the device, so a decode whose hist_len[b] is outside
+ * [0, max_len - 1] cannot be rejected on the host: the kernels then skip
+ * sequence b (its cache and out are not written) and set a bit in the context's
+ * device error word, which attn_device_error() reads.  No kernel traps.
+ */
+#ifndef ATTN_GB300_ATTN_H
+#define ATTN_GB300_ATTN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ATTN_OK 0
+#define ATTN_EINVAL (-1)   /* invalid argument or unsupported shape */
+#define ATTN_EARCH (-2)    /* current device is not compute capability 10.3 (sm_103) */
+#define ATTN_ECUDA (-3)    /* a CUDA runtime or launch error */
+#define ATTN_ENOMEM (-4)   /* device memory allocation failed in attn_create */
+#define ATTN_EDEVICE (-5)  /* attn_device_error found the device error word set */
+
+/* Bits of the device error word. */
+#define ATTN_DEVERR_HIST_RANGE 1 /* a decode hist_len[b] was outside [0, max_len - 1] */
+#define ATTN_DEVERR_TIMEOUT 2    /* a pipeline wait inside a kernel exceeded its time limit (about 1 s);
+                                    the affected outputs are not written */
+
+/* Opaque CUDA stream handle; pass a cudaStream_t (0 = legacy default stream). */
+typedef struct CUstream_st* attn_stream_t;
+
+typedef struct attn_cfg {
+    int batch;       /* sequences per call, >= 1 */
+    int n_q_heads;   /* query heads Hq, a multiple of n_kv_heads */
+    int n_kv_heads;  /* key/value heads Hkv; group size Hq/Hkv must be <= 16 */
+    int head_dim;    /* D: 64 or 128 */
+    int max_len;     /* static maximum cache length L (positions 0 .. L-1), 1 .. 1<<20 */
+    double rope_theta; /* RoPE base theta > 0 */
+} attn_cfg;
+
+typedef struct attn_ctx attn_ctx;
+
+/*
+ * Create a context for one shape on the current CUDA device.  Validates cfg,
+ * checks that the device is sm_103, builds the RoPE tables (Section 4.6.2) and
+ * allocates the context's scratch.  *out receives the context on success and
+ * NULL otherwise.  Returns ATTN_OK, ATTN_EINVAL, ATTN_EARCH, ATTN_ENOMEM or
+ * ATTN_ECUDA.  Blocking (it uploads the tables).
+ */
+int attn_create(const attn_cfg* cfg, attn_ctx** out);
+
+/* Free a context and its device memory (blocking).  NULL is ignored. */
+void attn_destroy(attn_ctx* ctx);
+
+/*
+ * Prefill (Section 4.2): positions 0 .. chunk_len-1.  Writes cache slots
+ * [0, chunk_len) of every sequence and out.  1 <= chunk_len <= max_len.
+ */
+int attn_prefill(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v, int chunk_len,
+                 uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream);
+
+/*
+ * Prefill_kv (Section 4.3): the caches hold hist_len valid history tokens in
+ * slots [0, hist_len) of every sequence; the new tokens take positions
+ * hist_len .. hist_len+chunk_len-1 and slots of the same index.  Only those
+ * slots are written.  hist_len >= 0, chunk_len >= 1, hist_len + chunk_len <= max_len.
+ * With hist_len = 0 the result equals attn_prefill (Section 4.2: one template).
+ */
+int attn_prefill_kv(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len,
+                    int chunk_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
+                    attn_stream_t stream);
+
+/*
+ * Decode (Section 4.4): one new token per sequence.  d_hist_len is a device
+ * array [batch] of int32: sequence b has hist_len[b] valid tokens in slots
+ * [0, hist_len[b]); its new token is written to slot hist_len[b] and attends to
+ * slots [0, hist_len[b]].  q [batch,1,Hq,D], k/v [batch,1,Hkv,D], out [batch,1,Hq,D].
+ * Out-of-range lengths: see "Errors" above.
+ */
+int attn_decode(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                const int32_t* d_hist_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
+                attn_stream_t stream);
+
+/*
+ * Synchronise `stream`, read and clear the context's device error word.
+ * *flags (may be NULL) receives the ATTN_DEVERR_* bits.  Returns ATTN_OK when
+ * the word was zero, ATTN_EDEVICE when a bit was set, ATTN_ECUDA on a CUDA error.
+ */
+int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
+
+/* Static text for an ATTN_* code. */
+const char* attn_strerror(int code);
+
+/* Text of the most recent CUDA error seen by this library on the calling thread. */
+const char* attn_last_cuda_error_string(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ATTN_GB300_ATTN_H */

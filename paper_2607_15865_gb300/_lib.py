@@ -1,0 +1,69 @@
+"""ctypes binding of ``libattn_gb300.so`` (include/attn.h): argument marshalling only.
+
+Every stage runs in the library's CUDA kernels; this module never computes any
+part of it and has no fallback: if the library is missing or cannot be loaded it
+raises.  Tensors are torch CUDA tensors (torch provides device memory and
+streams); bf16 tensors may be torch.bfloat16 or int16/uint16 bit patterns.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libattn_gb300.so")
+
+ATTN_OK, ATTN_EINVAL, ATTN_EARCH, ATTN_ECUDA, ATTN_ENOMEM, ATTN_EDEVICE = 0, -1, -2, -3, -4, -5
+DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
+
+EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
+            "attn_device_error", "attn_strerror", "attn_last_cuda_error_string")
+
+
+class AttnCfg(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int), ("n_q_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("max_len", ctypes.c_int), ("rope_theta", ctypes.c_double)]
+
+
+class AttnError(RuntimeError):
+    def __init__(self, code: int, what: str, lib=None):
+        msg = f"{what}: {code}"
+        if lib is not None:
+            msg += f" ({lib.attn_strerror(code).decode()})"
+            if code == ATTN_ECUDA:
+                msg += f": {lib.attn_last_cuda_error_string().decode()}"
+        super().__init__(msg)
+        self.code = code
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load the library (once) and declare its signatures.  Raises if it is absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is missing: build it with paper_2607_15865_gb300.build.build() "
+                          "(or __graft_entry__.build()); there is no fallback path")
+    lib = ctypes.CDLL(path)
+    vp, i32, u16p = ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p
+    lib.attn_create.argtypes = [ctypes.POINTER(AttnCfg), ctypes.POINTER(ctypes.c_void_p)]
+    lib.attn_create.restype = i32
+    lib.attn_destroy.argtypes = [vp]
+    lib.attn_destroy.restype = None
+    lib.attn_prefill.argtypes = [vp, u16p, u16p, u16p, i32, u16p, u16p, u16p, vp]
+    lib.attn_prefill.restype = i32
+    lib.attn_prefill_kv.argtypes = [vp, u16p, u16p, u16p, i32, i32, u16p, u16p, u16p, vp]
+    lib.attn_prefill_kv.restype = i32
+    lib.attn_decode.argtypes = [vp, u16p, u16p, u16p, vp, u16p, u16p, u16p, vp]
+    lib.attn_decode.restype = i32
+    lib.attn_device_error.argtypes = [vp, vp, ctypes.POINTER(ctypes.c_int)]
+    lib.attn_device_error.restype = i32
+    lib.attn_strerror.argtypes = [i32]
+    lib.attn_strerror.restype = ctypes.c_char_p
+    lib.attn_last_cuda_error_string.argtypes = []
+    lib.attn_last_cuda_error_string.restype = ctypes.c_char_p
+    _lib = lib
+    return lib

@@ -1,0 +1,123 @@
+"""Torch-facing wrapper of the C ABI: one context per attention shape.
+
+Argument marshalling only -- every stage runs in the library's CUDA kernels:
+
+  prefill     (Section 4.2)  q [B,S,Hq,D], k/v [B,S,Hkv,D] at positions 0..S-1
+  prefill_kv  (Section 4.3)  the same at positions hist..hist+S-1 over hist cached tokens
+  decode      (Section 4.4)  q [B,1,Hq,D], k/v [B,1,Hkv,D], hist_len [B] int32 on the device
+
+Caches are [B,Hkv,L,D] bf16 tensors owned by the caller and updated in place.
+All calls are asynchronous on the given (default: current) torch CUDA stream.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _lib
+
+_BF16_LIKE = (torch.bfloat16, torch.int16, torch.uint16)
+
+
+def _ptr(t: torch.Tensor, name: str, shape=None) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype not in _BF16_LIKE:
+        raise TypeError(f"{name} must hold bf16 values (torch.bfloat16 or 16-bit integer bit patterns)")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+class Attention:
+    """A context of include/attn.h for one (batch, heads, head_dim, max_len, theta) shape."""
+
+    def __init__(self, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int, max_len: int,
+                 rope_theta: float):
+        self.lib = _lib.load()
+        self.batch, self.n_q_heads, self.n_kv_heads = batch, n_q_heads, n_kv_heads
+        self.head_dim, self.max_len, self.rope_theta = head_dim, max_len, float(rope_theta)
+        cfg = _lib.AttnCfg(batch, n_q_heads, n_kv_heads, head_dim, max_len, float(rope_theta))
+        handle = ctypes.c_void_p()
+        rc = self.lib.attn_create(ctypes.byref(cfg), ctypes.byref(handle))
+        if rc != _lib.ATTN_OK:
+            raise _lib.AttnError(rc, "attn_create", self.lib)
+        self._ctx = handle
+
+    @classmethod
+    def for_shape(cls, shape) -> "Attention":
+        return cls(shape.batch, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.max_len, shape.rope_theta)
+
+    @property
+    def handle(self) -> ctypes.c_void_p:
+        return self._ctx
+
+    def close(self):
+        if getattr(self, "_ctx", None) is not None and self._ctx.value:
+            self.lib.attn_destroy(self._ctx)
+            self._ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, rc: int, what: str):
+        if rc != _lib.ATTN_OK:
+            raise _lib.AttnError(rc, what, self.lib)
+
+    def _cache_shape(self):
+        return (self.batch, self.n_kv_heads, self.max_len, self.head_dim)
+
+    def _new_out(self, q: torch.Tensor, out):
+        return torch.empty_like(q) if out is None else out
+
+    def prefill(self, q, k, v, k_cache, v_cache, out=None, stream=None) -> torch.Tensor:
+        return self.prefill_kv(q, k, v, 0, k_cache, v_cache, out, stream, _stage="attn_prefill")
+
+    def prefill_kv(self, q, k, v, hist_len: int, k_cache, v_cache, out=None, stream=None,
+                   _stage: str = "attn_prefill_kv") -> torch.Tensor:
+        B, S = q.shape[0], q.shape[1]
+        qs = (self.batch, S, self.n_q_heads, self.head_dim)
+        ks = (self.batch, S, self.n_kv_heads, self.head_dim)
+        out = self._new_out(q, out)
+        args = (_ptr(q, "q", qs), _ptr(k, "k", ks), _ptr(v, "v", ks))
+        cache = (_ptr(k_cache, "k_cache", self._cache_shape()), _ptr(v_cache, "v_cache", self._cache_shape()),
+                 _ptr(out, "out", qs))
+        if _stage == "attn_prefill":
+            rc = self.lib.attn_prefill(self._ctx, *args, S, *cache, _stream(stream))
+        else:
+            rc = self.lib.attn_prefill_kv(self._ctx, *args, int(hist_len), S, *cache, _stream(stream))
+        self._check(rc, _stage)
+        return out
+
+    def decode(self, q, k, v, hist_len: torch.Tensor, k_cache, v_cache, out=None, stream=None) -> torch.Tensor:
+        qs = (self.batch, 1, self.n_q_heads, self.head_dim)
+        ks = (self.batch, 1, self.n_kv_heads, self.head_dim)
+        if not (isinstance(hist_len, torch.Tensor) and hist_len.is_cuda and hist_len.dtype == torch.int32
+                and hist_len.is_contiguous() and tuple(hist_len.shape) == (self.batch,)):
+            raise TypeError("hist_len must be a contiguous int32 CUDA tensor of shape [batch]")
+        out = self._new_out(q, out)
+        rc = self.lib.attn_decode(self._ctx, _ptr(q, "q", qs), _ptr(k, "k", ks), _ptr(v, "v", ks),
+                                  hist_len.data_ptr(), _ptr(k_cache, "k_cache", self._cache_shape()),
+                                  _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
+                                  _stream(stream))
+        self._check(rc, "attn_decode")
+        return out
+
+    def device_error(self, stream=None) -> int:
+        """Synchronise, read and clear the device error word; returns its DEVERR_* bits."""
+        flags = ctypes.c_int(0)
+        rc = self.lib.attn_device_error(self._ctx, _stream(stream), ctypes.byref(flags))
+        if rc not in (_lib.ATTN_OK, _lib.ATTN_EDEVICE):
+            raise _lib.AttnError(rc, "attn_device_error", self.lib)
+        return flags.value

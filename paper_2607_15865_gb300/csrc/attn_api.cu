@@ -1,0 +1,265 @@
+// attn_api.cu -- host side of the C ABI declared in include/attn.h.
+//
+// Validates arguments, owns the per-shape context (RoPE tables, decode split-KV
+// partials, device error word), builds the TMA tensor maps for K2, and enqueues
+// the kernels of each stage on the caller's stream:
+//   prefill / prefill_kv : K1 rope_append (new k rotated + k, v appended in place)
+//                          -> K2 flash_fwd (q rotated in-kernel, causal attention)
+//   decode               : K1 rope_append (slot hist_len[b], read on the device)
+//                          -> K3 decode_split -> K4 decode_combine
+// No call allocates, frees or synchronises except attn_create/attn_destroy and
+// attn_device_error.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/attn.h"
+#include "internal.h"
+
+struct attn_ctx {
+    attn_cfg cfg;
+    attn::Shape shape;
+    int device;
+    int num_sms;
+    int nsplit_max;
+    float* d_cos;
+    float* d_sin;
+    float* d_part_o;
+    float* d_part_ml;
+    int* d_err;
+    PFN_cuTensorMapEncodeTiled_v12000 encode;
+};
+
+namespace {
+
+thread_local char g_cuda_msg[256] = "no error";
+
+int cuda_fail(cudaError_t e, const char* where) {
+    std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+    return ATTN_ECUDA;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool cfg_valid(const attn_cfg* c) {
+    if (c == nullptr) return false;
+    if (c->batch < 1 || c->batch > 65535) return false;
+    if (c->n_q_heads < 1 || c->n_kv_heads < 1 || c->n_q_heads % c->n_kv_heads != 0) return false;
+    if (c->n_q_heads / c->n_kv_heads > 16 || c->n_q_heads > 65535) return false;
+    if (c->head_dim != 64 && c->head_dim != 128) return false;
+    if (c->max_len < 1 || c->max_len > (1 << 20)) return false;
+    if (!(c->rope_theta > 0.0) || !std::isfinite(c->rope_theta)) return false;
+    return true;
+}
+
+// Split count of the decode: enough CTAs for ~4 per SM over B*Hkv*passes work
+// items, at most one split per 64 cache slots of the static maximum length.
+int decode_nsplit(const attn_ctx* c) {
+    const int G = c->cfg.n_q_heads / c->cfg.n_kv_heads;
+    const int passes = (G + 7) / 8;
+    const long items = static_cast<long>(c->cfg.batch) * c->cfg.n_kv_heads * passes;
+    long ns = (4L * c->num_sms + items - 1) / items;
+    const long cap = (c->cfg.max_len + 63) / 64;
+    if (ns > cap) ns = cap;
+    if (ns > c->nsplit_max) ns = c->nsplit_max;
+    if (ns < 1) ns = 1;
+    return static_cast<int>(ns);
+}
+
+int encode_map(const attn_ctx* c, CUtensorMap* map, const void* gaddr, cuuint32_t rank, const cuuint64_t* dims,
+               const cuuint64_t* strides, const cuuint32_t* box) {
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUresult r = c->encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(gaddr), dims, strides,
+                                 box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "cuTensorMapEncodeTiled failed (CUresult %d)", static_cast<int>(r));
+        return ATTN_ECUDA;
+    }
+    return ATTN_OK;
+}
+
+// The prefill stages: validate, K1, build the maps over [0, hist+chunk), K2.
+int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist, int chunk,
+                uint16_t* kc, uint16_t* vc, uint16_t* out, cudaStream_t st) {
+    if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || kc == nullptr || vc == nullptr ||
+        out == nullptr)
+        return ATTN_EINVAL;
+    if (chunk < 1 || hist < 0 || static_cast<long>(hist) + chunk > c->cfg.max_len) return ATTN_EINVAL;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(kc) || !aligned16(vc) || !aligned16(out))
+        return ATTN_EINVAL;
+    const attn::Shape& s = c->shape;
+    const cuuint64_t D = static_cast<cuuint64_t>(s.head_dim);
+    attn::FlashMaps maps;
+    {
+        const cuuint64_t dims[4] = {D, static_cast<cuuint64_t>(s.n_q_heads), static_cast<cuuint64_t>(chunk),
+                                    static_cast<cuuint64_t>(s.batch)};
+        const cuuint64_t strides[3] = {D * 2, D * 2 * s.n_q_heads, D * 2 * s.n_q_heads * static_cast<cuuint64_t>(chunk)};
+        const cuuint32_t box[4] = {64, 1, 128, 1};
+        const int rc = encode_map(c, &maps.q, q, 4, dims, strides, box);
+        if (rc != ATTN_OK) return rc;
+    }
+    {
+        const cuuint64_t dims[3] = {D, static_cast<cuuint64_t>(hist + chunk),
+                                    static_cast<cuuint64_t>(s.batch) * s.n_kv_heads};
+        const cuuint64_t strides[2] = {D * 2, D * 2 * static_cast<cuuint64_t>(s.max_len)};
+        const cuuint32_t box[3] = {64, 128, 1};
+        int rc = encode_map(c, &maps.k, kc, 3, dims, strides, box);
+        if (rc == ATTN_OK) rc = encode_map(c, &maps.v, vc, 3, dims, strides, box);
+        if (rc != ATTN_OK) return rc;
+    }
+    cudaError_t e = attn::launch_rope_append(s, k, v, hist, nullptr, chunk, c->d_cos, c->d_sin, kc, vc, c->d_err, st);
+    if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
+    e = attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_err, c->num_sms, st);
+    if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
+    return ATTN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int attn_create(const attn_cfg* cfg, attn_ctx** out) {
+    if (out == nullptr) return ATTN_EINVAL;
+    *out = nullptr;
+    if (!cfg_valid(cfg)) return ATTN_EINVAL;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    cudaDeviceProp prop;
+    e = cudaGetDeviceProperties(&prop, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+    if (prop.major != 10 || prop.minor != 3) return ATTN_EARCH;
+
+    attn_ctx* c = new (std::nothrow) attn_ctx();
+    if (c == nullptr) return ATTN_ENOMEM;
+    c->cfg = *cfg;
+    c->shape = attn::Shape{cfg->batch, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, cfg->max_len};
+    c->device = dev;
+    c->num_sms = prop.multiProcessorCount;
+    c->nsplit_max = 256;
+
+    cudaDriverEntryPointQueryResult qres;
+    void* fn = nullptr;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qres);
+    if (e != cudaSuccess || qres != cudaDriverEntryPointSuccess || fn == nullptr) {
+        delete c;
+        return cuda_fail(e == cudaSuccess ? cudaErrorNotSupported : e, "cuTensorMapEncodeTiled entry point");
+    }
+    c->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    e = attn::configure_flash_fwd();
+    if (e != cudaSuccess) {
+        delete c;
+        return cuda_fail(e, "configure flash_fwd");
+    }
+
+    // RoPE tables (Section 4.6.2): cos/sin of p * theta^(-2j/D), evaluated in double, stored as float.
+    const int half = cfg->head_dim / 2;
+    const size_t ntab = static_cast<size_t>(cfg->max_len) * half;
+    std::vector<float> hc(ntab), hs(ntab);
+    for (int p = 0; p < cfg->max_len; ++p) {
+        for (int j = 0; j < half; ++j) {
+            const double inv_freq = std::pow(cfg->rope_theta, -(2.0 * j) / static_cast<double>(cfg->head_dim));
+            const double ang = static_cast<double>(p) * inv_freq;
+            hc[static_cast<size_t>(p) * half + j] = static_cast<float>(std::cos(ang));
+            hs[static_cast<size_t>(p) * half + j] = static_cast<float>(std::sin(ang));
+        }
+    }
+    const size_t part_rows = static_cast<size_t>(cfg->batch) * cfg->n_q_heads * c->nsplit_max;
+    bool oom = false;
+    oom |= cudaMalloc(&c->d_cos, ntab * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_sin, ntab * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_part_o, part_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_part_ml, part_rows * 2 * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_err, sizeof(int)) != cudaSuccess;
+    if (oom) {
+        cudaGetLastError();
+        attn_destroy(c);
+        return ATTN_ENOMEM;
+    }
+    e = cudaMemcpy(c->d_cos, hc.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->d_sin, hs.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int));
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        attn_destroy(c);
+        return cuda_fail(e, "attn_create upload");
+    }
+    *out = c;
+    return ATTN_OK;
+}
+
+void attn_destroy(attn_ctx* c) {
+    if (c == nullptr) return;
+    cudaDeviceSynchronize();
+    cudaFree(c->d_cos);
+    cudaFree(c->d_sin);
+    cudaFree(c->d_part_o);
+    cudaFree(c->d_part_ml);
+    cudaFree(c->d_err);
+    delete c;
+}
+
+int attn_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int chunk_len,
+                 uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    return run_prefill(c, q, k, v, 0, chunk_len, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int attn_prefill_kv(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len,
+                    int chunk_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    return run_prefill(c, q, k, v, hist_len, chunk_len, k_cache, v_cache, out,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
+                uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
+        k_cache == nullptr || v_cache == nullptr || out == nullptr)
+        return ATTN_EINVAL;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out) || (reinterpret_cast<uintptr_t>(d_hist_len) & 3u))
+        return ATTN_EINVAL;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = attn::launch_rope_append(c->shape, k, v, 0, d_hist_len, 1, c->d_cos, c->d_sin, k_cache, v_cache,
+                                             c->d_err, st);
+    if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
+    e = attn::launch_decode(c->shape, q, d_hist_len, k_cache, v_cache, c->d_cos, c->d_sin, c->d_part_o, c->d_part_ml,
+                            decode_nsplit(c), out, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return ATTN_OK;
+}
+
+int attn_device_error(attn_ctx* c, attn_stream_t stream, int* flags) {
+    if (c == nullptr) return ATTN_EINVAL;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int h = 0;
+    cudaError_t e = cudaMemcpyAsync(&h, c->d_err, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess && h != 0) e = cudaMemsetAsync(c->d_err, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "attn_device_error");
+    if (flags != nullptr) *flags = h;
+    return h ? ATTN_EDEVICE : ATTN_OK;
+}
+
+const char* attn_strerror(int code) {
+    switch (code) {
+        case ATTN_OK: return "success";
+        case ATTN_EINVAL: return "invalid argument or unsupported shape";
+        case ATTN_EARCH: return "the current CUDA device is not sm_103 (GB300)";
+        case ATTN_ECUDA: return "CUDA runtime or launch error";
+        case ATTN_ENOMEM: return "device memory allocation failed";
+        case ATTN_EDEVICE: return "a kernel reported an error in the device error word";
+        default: return "unknown error code";
+    }
+}
+
+const char* attn_last_cuda_error_string(void) { return g_cuda_msg; }
+
+}  // extern "C"

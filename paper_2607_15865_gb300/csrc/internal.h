@@ -1,0 +1,43 @@
+// internal.h -- launchers shared between the translation units of the library.
+// Not part of the public ABI (include/attn.h).
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace attn {
+
+// Error-word bits (mirrors ATTN_DEVERR_* of attn.h).
+constexpr int kDevErrHistRange = 1;
+constexpr int kDevErrTimeout = 2;
+
+struct Shape {
+    int batch, n_q_heads, n_kv_heads, head_dim, max_len;
+};
+
+// K1: RoPE of the new k (table gather, Section 4.6.2) and the in-place append of
+// k and v into cache slots hist+i (Listing 2 "Concat"; Section 4.6.3).
+// hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.
+cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
+                               const int32_t* d_hist, int chunk, const float* cos_tab, const float* sin_tab,
+                               uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st);
+
+// K2: causal flash attention of `chunk` new queries at positions hist.. over cache
+// slots [0, hist+chunk) (prefill: hist=0).  RoPE of q is applied in the kernel.
+struct FlashMaps {
+    CUtensorMap q;  // q [B, S, Hq, D] as 4-D {D, Hq, S, B}; box {64, 1, 128, 1}
+    CUtensorMap k;  // k_cache as 3-D {D, hist+chunk, B*Hkv}; box {64, 128, 1}
+    CUtensorMap v;  // v_cache, same as k
+};
+// Raise the dynamic shared-memory limit of K2 on the current device (once per device).
+cudaError_t configure_flash_fwd();
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
+                             const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st);
+
+// K3 + K4: split-KV decode over slots [0, hist[b]] and the log-sum-exp combine.
+cudaError_t launch_decode(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
+                          const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
+                          float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
+
+}  // namespace attn

@@ -22,12 +22,15 @@ so every tensor of every workload has its own independent stream.
 """
 from __future__ import annotations
 
+import concurrent.futures as cf
+import os
+
 import numpy as np
 
 _GOLDEN = np.uint64(0x9E3779B97F4A7C15)
 _M1 = np.uint64(0xBF58476D1CE4E5B9)
 _M2 = np.uint64(0x94D049BB133111EB)
-_CHUNK = 1 << 22
+_CHUNK = 1 << 20
 
 
 def _mix(z: np.ndarray) -> np.ndarray:
@@ -59,33 +62,75 @@ def splitmix64_stream(key: int, start: int, count: int) -> np.ndarray:
         return _mix(np.uint64(key) + idx * _GOLDEN)
 
 
+def _mix_inplace(z: np.ndarray) -> None:
+    z ^= z >> np.uint64(30)
+    z *= _M1
+    z ^= z >> np.uint64(27)
+    z *= _M2
+    z ^= z >> np.uint64(31)
+
+
+def _normal_pairs(key: int, p0: int, p1: int, out: np.ndarray, n: int) -> None:
+    """Box-Muller pairs p0..p1-1 (stream outputs 2p and 2p+1) into out[2*p0 : min(n, 2*p1)]."""
+    two53 = float(2 ** 53)
+    with np.errstate(over="ignore"):
+        c = np.arange(2 * p0 + 1, 2 * p1 + 1, 2, dtype=np.uint64)  # counter of output 2p
+        z1 = c * _GOLDEN
+        z1 += np.uint64(key)
+        _mix_inplace(z1)
+        c += np.uint64(1)
+        c *= _GOLDEN
+        c += np.uint64(key)
+        _mix_inplace(c)
+    z1 >>= np.uint64(11)
+    c >>= np.uint64(11)
+    r = z1.astype(np.float64)
+    r += 1.0
+    r /= two53                      # u1 in (0, 1]
+    t = c.astype(np.float64)
+    t *= 2.0 * np.pi / two53        # 2*pi*u2 (scaling by 2^-53 is exact)
+    np.log(r, out=r)
+    r *= -2.0
+    np.sqrt(r, out=r)
+    lo, hi = 2 * p0, min(n, 2 * p1)
+    m = p1 - p0
+    if hi - lo == 2 * m:
+        out[lo:hi:2] = r * np.cos(t)
+        out[lo + 1:hi:2] = r * np.sin(t)
+    else:
+        pair = np.empty(2 * m)
+        pair[0::2] = r * np.cos(t)
+        pair[1::2] = r * np.sin(t)
+        out[lo:hi] = pair[: hi - lo]
+
+
 def normal_f64(key: int, n: int) -> np.ndarray:
-    """``n`` standard normal float64 values (Box-Muller on counter-based splitmix64)."""
+    """``n`` standard normal float64 values (Box-Muller on counter-based splitmix64).
+
+    Value 2p is r*cos(2*pi*u2) and value 2p+1 is r*sin(2*pi*u2), where u1 and u2
+    come from stream outputs 2p and 2p+1.  Chunks are independent, so they are
+    evaluated on a few threads (numpy releases the GIL); the result does not
+    depend on the chunking.
+    """
     out = np.empty(n, dtype=np.float64)
     npairs = (n + 1) // 2
-    two53 = float(2 ** 53)
-    for p0 in range(0, npairs, _CHUNK):
-        p1 = min(npairs, p0 + _CHUNK)
-        z = splitmix64_stream(key, 2 * p0, 2 * (p1 - p0)).reshape(-1, 2)
-        u1 = ((z[:, 0] >> np.uint64(11)).astype(np.float64) + 1.0) / two53
-        u2 = (z[:, 1] >> np.uint64(11)).astype(np.float64) / two53
-        r = np.sqrt(-2.0 * np.log(u1))
-        t = 2.0 * np.pi * u2
-        pair = np.empty((p1 - p0, 2), dtype=np.float64)
-        pair[:, 0] = r * np.cos(t)
-        pair[:, 1] = r * np.sin(t)
-        flat = pair.reshape(-1)
-        lo = 2 * p0
-        hi = min(n, 2 * p1)
-        out[lo:hi] = flat[: hi - lo]
+    bounds = [(p0, min(npairs, p0 + _CHUNK)) for p0 in range(0, npairs, _CHUNK)]
+    if len(bounds) <= 1:
+        for p0, p1 in bounds:
+            _normal_pairs(key, p0, p1, out, n)
+        return out
+    workers = max(1, min(8, (os.cpu_count() or 1), len(bounds)))
+    with cf.ThreadPoolExecutor(max_workers=workers) as ex:
+        list(ex.map(lambda b: _normal_pairs(key, b[0], b[1], out, n), bounds))
     return out
 
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """float32 -> bf16 bit pattern (uint16), round to nearest even.  Finite inputs only."""
-    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    u = u + np.uint64(0x7FFF) + ((u >> np.uint64(16)) & np.uint64(1))
-    return (u >> np.uint64(16)).astype(np.uint16)
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    # no uint32 overflow for finite inputs: the largest pattern 0xFF7FFFFF + 0x8000 fits
+    u = u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))
+    return (u >> np.uint32(16)).astype(np.uint16)
 
 
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:

@@ -1,0 +1,59 @@
+"""Helpers shared by the GPU parity tests: device transfer and the parity bar.
+
+The bar (north star of this path): outputs within max-abs 2e-2 and mean-abs 2e-3
+of the oracle; the k cache within 1 bf16 ulp; the v cache bit-exact; every cache
+slot outside the written range bit-unchanged.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from synthetic import gen
+
+MAX_ABS = 2e-2
+MEAN_ABS = 2e-3
+f32 = gen.bf16_bits_to_f32
+
+
+def to_dev(a, device="cuda"):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(device)
+
+
+def to_host(t):
+    return t.detach().cpu().numpy().view(np.uint16)
+
+
+def assert_out_close(got_bits, ref_bits, what):
+    g = f32(got_bits).astype(np.float64)
+    r = f32(ref_bits).astype(np.float64)
+    assert np.isfinite(g).all(), f"{what}: non-finite output"
+    err = np.abs(g - r)
+    mx, mean = float(err.max()), float(err.mean())
+    rel = float(np.linalg.norm(g - r) / max(np.linalg.norm(r), 1e-30))
+    assert mx <= MAX_ABS and mean <= MEAN_ABS, f"{what}: max-abs {mx:.3e} mean-abs {mean:.3e} rel {rel:.3e}"
+    return mx, mean, rel
+
+
+def ulp_diff(a_bits, b_bits):
+    """Distance in bf16 units in the last place between equal-signed bit patterns."""
+    a = a_bits.astype(np.int32)
+    b = b_bits.astype(np.int32)
+    # map sign-magnitude to a monotone integer line
+    a = np.where(a & 0x8000, 0x8000 - (a & 0x7FFF), 0x8000 + a)
+    b = np.where(b & 0x8000, 0x8000 - (b & 0x7FFF), 0x8000 + b)
+    return np.abs(a - b)
+
+
+def assert_cache(got_k, got_v, ref_k, ref_v, before_k, before_v, slots_per_seq, what):
+    """slots_per_seq[b] = (lo, hi): written range of sequence b; all else must be unchanged."""
+    L = got_k.shape[2]
+    for b, (lo, hi) in enumerate(slots_per_seq):
+        keep = np.ones(L, bool)
+        keep[lo:hi] = False
+        assert (got_k[b][:, keep] == before_k[b][:, keep]).all(), f"{what}: k slots outside [{lo},{hi}) changed"
+        assert (got_v[b][:, keep] == before_v[b][:, keep]).all(), f"{what}: v slots outside [{lo},{hi}) changed"
+        if hi > lo:
+            d = ulp_diff(got_k[b][:, lo:hi], ref_k[b][:, lo:hi])
+            assert d.max() <= 1, f"{what}: k cache off by {d.max()} ulp"
+            assert (got_v[b][:, lo:hi] == ref_v[b][:, lo:hi]).all(), f"{what}: v cache differs"

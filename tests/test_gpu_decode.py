@@ -1,0 +1,111 @@
+"""GPU parity of decode (K1 + K3 + K4 through the C ABI) against the CPU oracle.
+
+Covers the decode sweep (batch 1/4/16 x valid lengths 1024/4096/8191 over a
+static maximum of 8192), mixed per-sequence lengths including 0 and max_len-1,
+group sizes 1/7/16 and head_dim 64, the long-context point (32767 valid tokens),
+and out-of-range lengths, which must set the device error word and leave that
+sequence's cache and output untouched.  Slots past hist_len[b] hold NaN.
+"""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from synthetic import workloads as w
+from synthetic.workloads import Shape
+from tests.gpu_util import assert_cache, assert_out_close, to_dev, to_host
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    import torch as t
+    assert t.cuda.is_available(), "GPU tests need a CUDA device"
+    import __graft_entry__
+    __graft_entry__.build()
+    return t
+
+
+def run_decode(torch, shape, q, k, v, hist, kc, vc, out_init=None):
+    from paper_2607_15865_gb300.attention import Attention
+    attn = Attention.for_shape(shape)
+    gk, gv = to_dev(kc), to_dev(vc)
+    hl = torch.from_numpy(np.asarray(hist, np.int32)).cuda()
+    out = to_dev(out_init) if out_init is not None else None
+    out = attn.decode(to_dev(q), to_dev(k), to_dev(v), hl, gk, gv, out=out)
+    torch.cuda.synchronize()
+    flags = attn.device_error()
+    res = to_host(out), to_host(gk), to_host(gv), flags
+    attn.close()
+    return res
+
+
+def check_decode(torch, shape, tag, hist, rows=None):
+    hist = np.asarray(hist, np.int32)
+    q, k, v = w.tokens(shape, tag, 1)
+    kc, vc = w.cache(shape, tag, int(hist.max()), fill="nan")
+    for b in range(shape.batch):  # sequence b has hist[b] valid slots; the rest stays NaN
+        kc[b, :, hist[b]:] = 0x7FC0
+        vc[b, :, hist[b]:] = 0x7FC0
+    out, gk, gv, flags = run_decode(torch, shape, q, k, v, hist, kc, vc)
+    assert flags == 0
+    rk, rv = kc.copy(), vc.copy()
+    O.append(shape, k, v, hist, rk, rv)
+    assert_cache(gk, gv, rk, rv, kc, vc, [(int(h), int(h) + 1) for h in hist], f"{tag} cache")
+    if rows is None:
+        rows = np.array([(b, 0, h) for b in range(shape.batch) for h in range(shape.n_q_heads)], np.int32)
+    ref = O.attend_rows(shape, q, hist, rk, rv, rows)
+    assert_out_close(out[rows[:, 0], rows[:, 1], rows[:, 2]], ref, tag)
+
+
+SWEEP = [(b, h) for b in w.DECODE_BATCHES for h in w.DECODE_HISTS]
+
+
+@pytest.mark.parametrize("batch,hist", SWEEP, ids=[f"b{b}_hist{h}" for b, h in SWEEP])
+def test_decode_sweep(torch, batch, hist):
+    shape = w.decode_shape(batch)
+    rows = None
+    if batch > 4:
+        rng = np.random.default_rng(batch * 7 + hist)
+        pick = [(b, 0, h) for b in (0, batch - 1) for h in range(shape.n_q_heads)]
+        pick += [(int(rng.integers(batch)), 0, int(rng.integers(shape.n_q_heads))) for _ in range(32)]
+        rows = np.array(pick, np.int32)
+    check_decode(torch, shape, f"sweep_b{batch}_{hist}", [hist] * batch, rows)
+
+
+def test_decode_mixed_lengths(torch):
+    shape = Shape("mixed", 5, 32, 8, 128, 8192, 5.0e5)
+    check_decode(torch, shape, "mixed", [0, 1, 127, 4097, 8191])
+
+
+@pytest.mark.parametrize("shape,hist", [
+    (Shape("g7", 2, 28, 4, 128, 1500, 1.0e6), [700, 1499]),
+    (Shape("g1_d64", 3, 4, 4, 64, 900, 1.0e4), [3, 500, 899]),
+    (Shape("g16", 1, 16, 1, 128, 2000, 1.0e4), [1999]),
+    (Shape("g5_d64", 2, 10, 2, 64, 300, 1.0e4), [31, 32]),
+], ids=["group7", "group1_d64", "group16", "group5_d64"])
+def test_decode_group_sizes(torch, shape, hist):
+    check_decode(torch, shape, shape.name, hist)
+
+
+def test_decode_long_context(torch):
+    shape = Shape("long_decode", 1, 40, 8, 128, 32768, 1.0e6)
+    check_decode(torch, shape, "long_decode", [w.LONG_DECODE_HIST])
+
+
+def test_decode_out_of_range_length_sets_error_and_skips(torch):
+    shape = Shape("badlen", 3, 8, 2, 128, 256, 1.0e4)
+    q, k, v = w.tokens(shape, "badlen", 1)
+    kc, vc = w.cache(shape, "badlen", 200, fill="zero")
+    sentinel = np.full(q.shape, 0x4049, np.uint16)  # 3.14 in bf16
+    hist = [100, -1, 256]
+    out, gk, gv, flags = run_decode(torch, shape, q, k, v, hist, kc, vc, out_init=sentinel)
+    assert flags & 1, "an out-of-range hist_len must set ATTN_DEVERR_HIST_RANGE"
+    for b in (1, 2):
+        assert (out[b] == sentinel[b]).all(), "a skipped sequence's output must not be written"
+        assert (gk[b] == kc[b]).all() and (gv[b] == vc[b]).all(), "a skipped sequence's cache must not change"
+    rk, rv = kc.copy(), vc.copy()
+    one = Shape("badlen1", 1, 8, 2, 128, 256, 1.0e4)
+    r0k, r0v = rk[:1].copy(), rv[:1].copy()
+    ref = O.decode(one, q[:1].copy(), k[:1].copy(), v[:1].copy(), np.array([100], np.int32), r0k, r0v)
+    assert_out_close(out[:1], ref, "valid sequence next to invalid ones")

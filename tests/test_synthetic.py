@@ -39,3 +39,15 @@ def test_workload_shapes():
     assert kc.shape == (1, 8, 2048, 128) and (kc[:, :, 1536:] == 0).all() and (kc[:, :, :1536] != 0).any()
     std = gen.bf16_bits_to_f32(q).std()
     assert abs(std - 1 / 8) < 0.01
+
+
+def test_threaded_normal_equals_direct_definition():
+    """The chunked, threaded evaluation equals Box-Muller applied directly to the stream."""
+    key = gen.tensor_key("t", "direct")
+    n = 3 * (1 << 20) + 7
+    z = gen.splitmix64_stream(key, 0, 2 * ((n + 1) // 2)).reshape(-1, 2)
+    u1 = ((z[:, 0] >> np.uint64(11)).astype(np.float64) + 1.0) / 2.0 ** 53
+    u2 = (z[:, 1] >> np.uint64(11)).astype(np.float64) / 2.0 ** 53
+    r = np.sqrt(-2.0 * np.log(u1))
+    ref = np.stack([r * np.cos(2 * np.pi * u2), r * np.sin(2 * np.pi * u2)], 1).reshape(-1)[:n]
+    assert (gen.normal_f64(key, n) == ref).all()
