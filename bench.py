@@ -1,0 +1,417 @@
+"""Throughput of the three-stage attention path (prefill, prefill_kv, decode) on GB300.
+
+One step = one pass of the whole hot path over the long-context workload (batch 1,
+40 query heads, 8 KV heads, head_dim 128, RoPE theta 1e6, static max length
+32768): prefill of 4096 tokens, prefill_kv of a 4096-token chunk over 28672
+history tokens, and one decode step at 32767 valid tokens, all on one KV cache.
+Inputs are seeded synthetic bf16 N(0,1)/sqrt(128) values (synthetic/), resident in
+HBM before the timed region; L2 is flushed (256 MB write) between steps.
+
+value     algorithmic attention FLOP of the step (4*D per unmasked query-key pair
+          per query head, exact causal count) / mean device step time, TFLOP/s.
+e2e       the same metric through the same C-ABI calls with host buffers: every
+          step copies its q/k/v from pinned host memory and its outputs back.
+roofline  the dominant kernel (flash_fwd) against the measured bf16 tensor peak.
+stages    per-stage times; prefill stages in TFLOP/s, decode in HBM GB/s.
+cpu_baseline  the CPU oracle on a bounded row sample of the same step.
+
+--impl reference times the CPU oracle (the reference arm of this path) instead.
+Multi-GPU (torchrun): every rank runs its own replica of the workload (weak
+scaling, no collective on the data path); value is the whole-job aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synthetic import gen  # noqa: E402
+from synthetic import workloads as w  # noqa: E402
+
+METRIC = "prefill/prefill_kv attn TFLOP/s; decode KV GB/s; % of GB300 roofline"
+WORKLOAD = ("long-context three-stage step: B1 Hq40 Hkv8 D128 theta1e6 L32768; prefill 4096 + "
+            "prefill_kv 4096 over 28672 + decode at 32767")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ----------------------------------------------------------------------------- work accounting
+
+
+def prefill_pairs(hist: int, chunk: int) -> int:
+    """Unmasked (query, key) pairs of one head: row i sees hist + i + 1 keys."""
+    return chunk * hist + chunk * (chunk + 1) // 2
+
+
+def attn_flops(shape, pairs_per_head: int) -> float:
+    return 4.0 * shape.head_dim * shape.n_q_heads * shape.batch * pairs_per_head
+
+
+def decode_bytes(shape, hist: int) -> float:
+    """Algorithmic HBM bytes of one decode step per sequence: the K/V history read once,
+    q and the new k/v read, the new k/v written to the cache, out written (bf16)."""
+    d, hq, hkv = shape.head_dim, shape.n_q_heads, shape.n_kv_heads
+    return shape.batch * (hist * hkv * d * 2 * 2 + hq * d * 2 * 2 + hkv * d * 2 * 4)
+
+
+S = w.LONG
+STAGES = {
+    "prefill": dict(hist=0, chunk=w.LONG_PREFILL),
+    "prefill_kv": dict(hist=w.LONG_PKV_HIST, chunk=w.LONG_PKV_CHUNK),
+    "decode": dict(hist=w.LONG_DECODE_HIST, chunk=1),
+}
+FLOPS = {k: attn_flops(S, prefill_pairs(v["hist"], v["chunk"])) for k, v in STAGES.items()}
+STEP_FLOPS = sum(FLOPS.values())
+DECODE_BYTES = decode_bytes(S, w.LONG_DECODE_HIST)
+
+
+# ----------------------------------------------------------------------------- helpers
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+def make_inputs():
+    """Seeded host inputs of the step (bf16 bit patterns)."""
+    data = {}
+    for name, st in STAGES.items():
+        data[name] = w.tokens(S, f"bench_{name}", st["chunk"])
+    kc, vc = w.cache(S, "bench_history", w.LONG_PKV_HIST, fill="zero")
+    return data, kc, vc
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(self.dev)], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def flash_traffic_from_profile():
+    """DRAM bytes per flash_fwd launch from the committed ncu summary, if it was taken
+    on the current kernel source (its sha256 is recorded there); else None."""
+    path = os.path.join(ROOT, "profiles", "flash_fwd_long_prefill_kv.md")
+    src = os.path.join(ROOT, "paper_2607_15865_gb300", "csrc", "flash_fwd.cu")
+    if not os.path.exists(path):
+        return None
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    kv = {}
+    for line in open(path):
+        if line.startswith("- ") and ":" in line:
+            k, v = line[2:].split(":", 1)
+            kv[k.strip()] = v.strip().strip("`")
+    if kv.get("kernel_source_sha256_16") != sha:
+        return None
+    try:
+        return float(kv["dram_bytes_per_launch_full_size"])
+    except (KeyError, ValueError):
+        return None
+
+
+# ----------------------------------------------------------------------------- oracle sample
+
+
+def oracle_sample(data, kc0, vc0, rows_pkv: int, rows_prefill: int, seed: int = 7):
+    """Runs the oracle over a bounded row sample of one step (append every stage's new
+    tokens in order, then the sampled rows of each stage).  Returns (rows, outputs,
+    algorithmic FLOP of the sampled rows, seconds)."""
+    from oracle import oracle as O
+    rng = np.random.default_rng(seed)
+    kc, vc = kc0.copy(), vc0.copy()
+    picks = {"prefill": rows_prefill, "prefill_kv": rows_pkv, "decode": S.n_q_heads}
+    rows, outs, flops = {}, {}, 0.0
+    t0 = time.perf_counter()
+    for name, st in STAGES.items():
+        q, k, v = data[name]
+        O.append(S, k, v, st["hist"], kc, vc)
+        n = picks[name]
+        if name == "decode":
+            r = np.array([(0, 0, h) for h in range(S.n_q_heads)], np.int32)
+        else:
+            r = np.stack([np.zeros(n, np.int64), rng.integers(0, st["chunk"], n),
+                          rng.integers(0, S.n_q_heads, n)], 1).astype(np.int32)
+        outs[name] = O.attend_rows(S, q, st["hist"], kc, vc, r)
+        rows[name] = r
+        flops += float(sum(4.0 * S.head_dim * (st["hist"] + int(i) + 1) for i in r[:, 1]))
+    return rows, outs, flops, time.perf_counter() - t0
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return 0
+    data, kc, vc = make_inputs()
+    oracle_sample(data, kc, vc, 2, 2)  # build + warm the oracle library
+    times, flops = [], []
+    for _ in range(args.warmup):
+        oracle_sample(data, kc, vc, args.ref_rows, max(1, args.ref_rows // 4))
+    for i in range(args.steps):
+        _, _, f, t = oracle_sample(data, kc, vc, args.ref_rows, max(1, args.ref_rows // 4), seed=100 + i)
+        times.append(t)
+        flops.append(f)
+    value = sum(flops) / sum(times) / 1e12
+    sample = (f"per step {args.ref_rows} prefill_kv rows + {max(1, args.ref_rows // 4)} prefill rows + "
+              f"{S.n_q_heads} decode rows of the workload, all new tokens appended")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- our arm
+
+
+def run_ours(args):
+    import torch
+
+    rank, local_rank, world = dist_env()
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend=backend)
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.attention import Attention
+
+    data, kc_h, vc_h = make_inputs()
+    d = {name: tuple(torch.from_numpy(a.view(np.int16)).to(dev) for a in arrs) for name, arrs in data.items()}
+    kc = torch.from_numpy(kc_h.view(np.int16)).to(dev)
+    vc = torch.from_numpy(vc_h.view(np.int16)).to(dev)
+    hist_dec = torch.full((S.batch,), STAGES["decode"]["hist"], dtype=torch.int32, device=dev)
+    outs = {name: torch.empty_like(d[name][0]) for name in STAGES}
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    attn = Attention.for_shape(S)
+    stream = torch.cuda.current_stream()
+
+    def step(src=None):
+        qkv = d if src is None else src
+        attn.prefill(*qkv["prefill"], kc, vc, out=outs["prefill"], stream=stream)
+        attn.prefill_kv(*qkv["prefill_kv"], STAGES["prefill_kv"]["hist"], kc, vc, out=outs["prefill_kv"],
+                        stream=stream)
+        attn.decode(*qkv["decode"], hist_dec, kc, vc, out=outs["decode"], stream=stream)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    if attn.device_error() != 0:
+        raise RuntimeError("device error word set during warm-up")
+
+    # ------------------------------------------------------------ timed region (device-resident inputs)
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    attn.timing_read()
+    attn.timing_enable(8 * K)
+    sampler = ClockSampler(local_rank)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)  # let the sampler start before the GPU gets busy
+    for i in range(K):
+        flush.zero_()
+        ev[i][0].record(stream)
+        attn.prefill(*d["prefill"], kc, vc, out=outs["prefill"], stream=stream)
+        ev[i][1].record(stream)
+        attn.prefill_kv(*d["prefill_kv"], STAGES["prefill_kv"]["hist"], kc, vc, out=outs["prefill_kv"], stream=stream)
+        ev[i][2].record(stream)
+        attn.decode(*d["decode"], hist_dec, kc, vc, out=outs["decode"], stream=stream)
+        ev[i][3].record(stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    kern = attn.timing_read()
+    attn.timing_enable(0)
+    step_ms = [ev[i][0].elapsed_time(ev[i][3]) for i in range(K)]
+    stage_ms = {name: sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(K)) / K
+                for j, name in enumerate(STAGES)}
+    ms = sum(step_ms) / K
+    if dist is not None:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    if attn.device_error() != 0:
+        raise RuntimeError("device error word set during the timed region")
+
+    # ------------------------------------------------------------ end to end (host buffers)
+    host = {name: tuple(torch.from_numpy(a.view(np.int16)).pin_memory() for a in arrs) for name, arrs in data.items()}
+    host_out = {name: torch.empty(tuple(outs[name].shape), dtype=torch.int16).pin_memory() for name in STAGES}
+    h2d = sum(t.numel() * 2 for arrs in host.values() for t in arrs)
+    d2h = sum(t.numel() * 2 for t in host_out.values())
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    torch.cuda.synchronize()
+    for i in range(K):
+        flush.zero_()
+        e2e_ev[i][0].record(stream)
+        for name in STAGES:
+            for dst, src in zip(d[name], host[name]):
+                dst.copy_(src, non_blocking=True)
+        step()
+        for name in STAGES:
+            host_out[name].copy_(outs[name], non_blocking=True)
+        e2e_ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / K
+    if dist is not None:
+        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    # ------------------------------------------------------------ parity of the timed outputs + CPU baseline
+    result = {}
+    if rank == 0:
+        peaks, peak_kind = load_peaks()
+        got = {name: outs[name].cpu().numpy().view(np.uint16) for name in STAGES}
+        cpu = None
+        parity = {}
+        rows, ref, f_cpu, t_cpu = oracle_sample(data, kc_h, vc_h, args.cpu_rows, max(1, args.cpu_rows // 4))
+        for name in STAGES:
+            r = rows[name]
+            g = gen.bf16_bits_to_f32(got[name][r[:, 0], r[:, 1], r[:, 2]]).astype(np.float64)
+            e = gen.bf16_bits_to_f32(ref[name]).astype(np.float64)
+            err = np.abs(g - e)
+            rel = float(np.linalg.norm(g - e) / max(np.linalg.norm(e), 1e-30))
+            parity[name] = {"rows": int(len(r)), "max_abs": float(err.max()), "mean_abs": float(err.mean()),
+                            "rel": rel}
+            if not (err.max() <= 2e-2 and err.mean() <= 2e-3 and rel <= 1e-2 and np.isfinite(g).all()):
+                raise SystemExit(f"parity check failed for {name}: {parity[name]}")
+        if world == 1 and not args.no_cpu_baseline:
+            cpu = {"value": f_cpu / t_cpu / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                   "sample": (f"{args.cpu_rows} prefill_kv rows + {max(1, args.cpu_rows // 4)} prefill rows + "
+                              f"{S.n_q_heads} decode rows of the step, single-threaded, {t_cpu:.1f} s")}
+        value = world * STEP_FLOPS / (ms * 1e-3) / 1e12
+        flash_ms = kern["flash_fwd"][0]
+        flash_n = kern["flash_fwd"][1]
+        flash_flops = (FLOPS["prefill"] + FLOPS["prefill_kv"]) * K
+        flash_tflops = flash_flops / (flash_ms * 1e-3) / 1e12
+        tc_peak = float(peaks["bf16_tflops"])
+        traffic = flash_traffic_from_profile()
+        hbm = float(peaks["hbm_gbs"])
+        stages = {}
+        for name in STAGES:
+            t_s = stage_ms[name] * 1e-3
+            if name == "decode":
+                gbs = DECODE_BYTES / t_s / 1e9
+                stages[name] = {"ms": stage_ms[name], "GB/s": gbs, "frac_hbm": gbs / hbm,
+                                "kernel_ms": {k: kern[k][0] / K for k in ("decode_split", "decode_combine")}}
+            else:
+                tf = FLOPS[name] / t_s / 1e12
+                stages[name] = {"ms": stage_ms[name], "TFLOP/s": tf, "frac_tensor": tf / tc_peak}
+        launches = int(sum(n for _, n in kern.values()))
+        result = {
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "l2": "flushed between steps (256 MB write, untimed)",
+                       "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       "step_gflop": STEP_FLOPS / 1e9},
+            "roofline": {"bound": "tensor", "achieved": flash_tflops, "peak": tc_peak, "unit": "TFLOP/s",
+                         "frac": flash_tflops / tc_peak, "traffic": traffic, "kernel": "flash_fwd",
+                         "peak_source": f"{peak_kind} bf16_tflops (burst)",
+                         "launch_ms_avg": flash_ms / max(flash_n, 1)},
+            "stages": stages,
+            "kernels_ms_per_step": {k: v[0] / K for k, v in kern.items()},
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * STEP_FLOPS / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "parity": parity,
+        }
+        print(json.dumps(result), flush=True)
+    attn.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--cpu-rows", type=int, default=192, help="prefill_kv rows in the oracle's timed sample")
+    ap.add_argument("--ref-rows", type=int, default=48, help="prefill_kv rows per reference-arm step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

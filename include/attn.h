@@ -135,6 +135,30 @@ int attn_decode(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint1
  */
 int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
 
+/*
+ * Kernel timing (tracing).  The library launches four kernels:
+ *   ATTN_KERNEL_ROPE_APPEND     RoPE of the new keys + in-place cache append (every stage)
+ *   ATTN_KERNEL_FLASH_FWD       causal flash attention (prefill, prefill_kv)
+ *   ATTN_KERNEL_DECODE_SPLIT    split-KV decode partials (decode)
+ *   ATTN_KERNEL_DECODE_COMBINE  log-sum-exp combine of the partials (decode)
+ * attn_timing_enable(ctx, n) creates n pairs of CUDA events (blocking, the only
+ * allocation it makes) and from then on every stage call records one pair
+ * around each kernel it enqueues, on the call's stream; n = 0 disables timing
+ * and frees the events.  Launches beyond n pairs are counted but not timed.
+ * attn_timing_read synchronises the device, adds up the elapsed time of every
+ * recorded pair per kernel into ms[ATTN_NUM_KERNELS] and the launches counted
+ * since the last read (timed or not, enabled or not) into
+ * launches[ATTN_NUM_KERNELS], then starts a new period.  Either array may be
+ * NULL.  Both return ATTN_OK, ATTN_EINVAL or ATTN_ECUDA.
+ */
+#define ATTN_KERNEL_ROPE_APPEND 0
+#define ATTN_KERNEL_FLASH_FWD 1
+#define ATTN_KERNEL_DECODE_SPLIT 2
+#define ATTN_KERNEL_DECODE_COMBINE 3
+#define ATTN_NUM_KERNELS 4
+int attn_timing_enable(attn_ctx* ctx, int max_launches);
+int attn_timing_read(attn_ctx* ctx, double* ms, long long* launches);
+
 /* Static text for an ATTN_* code. */
 const char* attn_strerror(int code);
 

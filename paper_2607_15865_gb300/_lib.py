@@ -17,7 +17,9 @@ ATTN_OK, ATTN_EINVAL, ATTN_EARCH, ATTN_ECUDA, ATTN_ENOMEM, ATTN_EDEVICE = 0, -1,
 DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
-            "attn_device_error", "attn_strerror", "attn_last_cuda_error_string")
+            "attn_device_error", "attn_timing_enable", "attn_timing_read", "attn_strerror",
+            "attn_last_cuda_error_string")
+KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
 
 
 class AttnCfg(ctypes.Structure):
@@ -61,6 +63,10 @@ def load(path: str = LIB_PATH):
     lib.attn_decode.restype = i32
     lib.attn_device_error.argtypes = [vp, vp, ctypes.POINTER(ctypes.c_int)]
     lib.attn_device_error.restype = i32
+    lib.attn_timing_enable.argtypes = [vp, i32]
+    lib.attn_timing_enable.restype = i32
+    lib.attn_timing_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_longlong)]
+    lib.attn_timing_read.restype = i32
     lib.attn_strerror.argtypes = [i32]
     lib.attn_strerror.restype = ctypes.c_char_p
     lib.attn_last_cuda_error_string.argtypes = []

@@ -114,6 +114,17 @@ class Attention:
         self._check(rc, "attn_decode")
         return out
 
+    def timing_enable(self, max_launches: int):
+        """Record CUDA events around every kernel of the following calls (0 disables)."""
+        self._check(self.lib.attn_timing_enable(self._ctx, int(max_launches)), "attn_timing_enable")
+
+    def timing_read(self):
+        """Synchronise; returns {kernel: (milliseconds, launches)} since the last read."""
+        ms = (ctypes.c_double * 4)()
+        n = (ctypes.c_longlong * 4)()
+        self._check(self.lib.attn_timing_read(self._ctx, ms, n), "attn_timing_read")
+        return {name: (ms[i], n[i]) for i, name in enumerate(_lib.KERNELS)}
+
     def device_error(self, stream=None) -> int:
         """Synchronise, read and clear the device error word; returns its DEVERR_* bits."""
         flags = ctypes.c_int(0)

@@ -34,6 +34,11 @@ struct attn_ctx {
     float* d_part_ml;
     int* d_err;
     PFN_cuTensorMapEncodeTiled_v12000 encode;
+    // kernel timing: event pairs recorded around each launch while enabled
+    std::vector<cudaEvent_t> ev;
+    std::vector<int> ev_kind;
+    int ev_used;
+    long long launches[ATTN_NUM_KERNELS];
 };
 
 namespace {
@@ -70,6 +75,32 @@ int decode_nsplit(const attn_ctx* c) {
     if (ns > c->nsplit_max) ns = c->nsplit_max;
     if (ns < 1) ns = 1;
     return static_cast<int>(ns);
+}
+
+// Enqueue one kernel through `launch`, bracketed by a timing event pair when enabled.
+template <typename F>
+cudaError_t timed(attn_ctx* c, int kind, cudaStream_t st, F&& launch) {
+    const bool rec = !c->ev_kind.empty() && c->ev_used < static_cast<int>(c->ev_kind.size());
+    if (rec) {
+        const cudaError_t e = cudaEventRecord(c->ev[2 * c->ev_used], st);
+        if (e != cudaSuccess) return e;
+    }
+    const cudaError_t e = launch();
+    if (e != cudaSuccess) return e;
+    ++c->launches[kind];
+    if (rec) {
+        const cudaError_t e2 = cudaEventRecord(c->ev[2 * c->ev_used + 1], st);
+        if (e2 != cudaSuccess) return e2;
+        c->ev_kind[c->ev_used++] = kind;
+    }
+    return cudaSuccess;
+}
+
+void free_events(attn_ctx* c) {
+    for (cudaEvent_t e : c->ev) cudaEventDestroy(e);
+    c->ev.clear();
+    c->ev_kind.clear();
+    c->ev_used = 0;
 }
 
 int encode_map(const attn_ctx* c, CUtensorMap* map, const void* gaddr, cuuint32_t rank, const cuuint64_t* dims,
@@ -114,9 +145,13 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         if (rc == ATTN_OK) rc = encode_map(c, &maps.v, vc, 3, dims, strides, box);
         if (rc != ATTN_OK) return rc;
     }
-    cudaError_t e = attn::launch_rope_append(s, k, v, hist, nullptr, chunk, c->d_cos, c->d_sin, kc, vc, c->d_err, st);
+    cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&] {
+        return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, c->d_cos, c->d_sin, kc, vc, c->d_err, st);
+    });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
-    e = attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_err, c->num_sms, st);
+    e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&] {
+        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_err, c->num_sms, st);
+    });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
     return ATTN_OK;
 }
@@ -198,6 +233,7 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
 void attn_destroy(attn_ctx* c) {
     if (c == nullptr) return;
     cudaDeviceSynchronize();
+    free_events(c);
     cudaFree(c->d_cos);
     cudaFree(c->d_sin);
     cudaFree(c->d_part_o);
@@ -226,12 +262,21 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         !aligned16(out) || (reinterpret_cast<uintptr_t>(d_hist_len) & 3u))
         return ATTN_EINVAL;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = attn::launch_rope_append(c->shape, k, v, 0, d_hist_len, 1, c->d_cos, c->d_sin, k_cache, v_cache,
-                                             c->d_err, st);
+    const int nsplit = decode_nsplit(c);
+    cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&] {
+        return attn::launch_rope_append(c->shape, k, v, 0, d_hist_len, 1, c->d_cos, c->d_sin, k_cache, v_cache,
+                                        c->d_err, st);
+    });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
-    e = attn::launch_decode(c->shape, q, d_hist_len, k_cache, v_cache, c->d_cos, c->d_sin, c->d_part_o, c->d_part_ml,
-                            decode_nsplit(c), out, st);
-    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&] {
+        return attn::launch_decode_split(c->shape, q, d_hist_len, k_cache, v_cache, c->d_cos, c->d_sin, c->d_part_o,
+                                         c->d_part_ml, nsplit, st);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
+    e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&] {
+        return attn::launch_decode_combine(c->shape, d_hist_len, c->d_part_o, c->d_part_ml, nsplit, out, st);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "decode_combine launch");
     return ATTN_OK;
 }
 
@@ -246,6 +291,45 @@ int attn_device_error(attn_ctx* c, attn_stream_t stream, int* flags) {
     if (e != cudaSuccess) return cuda_fail(e, "attn_device_error");
     if (flags != nullptr) *flags = h;
     return h ? ATTN_EDEVICE : ATTN_OK;
+}
+
+int attn_timing_enable(attn_ctx* c, int max_launches) {
+    if (c == nullptr || max_launches < 0 || max_launches > (1 << 20)) return ATTN_EINVAL;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "attn_timing_enable");
+    free_events(c);
+    if (max_launches == 0) return ATTN_OK;
+    c->ev.resize(2 * static_cast<size_t>(max_launches), nullptr);
+    c->ev_kind.assign(static_cast<size_t>(max_launches), -1);
+    for (cudaEvent_t& ev : c->ev) {
+        e = cudaEventCreate(&ev);
+        if (e != cudaSuccess) {
+            ev = nullptr;
+            free_events(c);
+            return cuda_fail(e, "cudaEventCreate");
+        }
+    }
+    return ATTN_OK;
+}
+
+int attn_timing_read(attn_ctx* c, double* ms, long long* launches) {
+    if (c == nullptr) return ATTN_EINVAL;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "attn_timing_read");
+    double acc[ATTN_NUM_KERNELS] = {0.0, 0.0, 0.0, 0.0};
+    for (int i = 0; i < c->ev_used; ++i) {
+        float t = 0.f;
+        e = cudaEventElapsedTime(&t, c->ev[2 * i], c->ev[2 * i + 1]);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+        acc[c->ev_kind[i]] += t;
+    }
+    for (int k = 0; k < ATTN_NUM_KERNELS; ++k) {
+        if (ms != nullptr) ms[k] = acc[k];
+        if (launches != nullptr) launches[k] = c->launches[k];
+        c->launches[k] = 0;
+    }
+    c->ev_used = 0;
+    return ATTN_OK;
 }
 
 const char* attn_strerror(int code) {

@@ -321,16 +321,19 @@ void launch_split_d(const Shape& s, const uint16_t* q, const int32_t* d_hist, co
 
 }  // namespace
 
-cudaError_t launch_decode(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
-                          const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
-                          float* part_ml, int nsplit, uint16_t* out, cudaStream_t st) {
+cudaError_t launch_decode_split(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
+                                const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
+                                float* part_ml, int nsplit, cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(s.head_dim)));
     if (s.head_dim == 128)
         launch_split_d<128>(s, q, d_hist, k_cache, v_cache, cos_tab, sin_tab, nsplit, scale_log2, part_o, part_ml, st);
     else
         launch_split_d<64>(s, q, d_hist, k_cache, v_cache, cos_tab, sin_tab, nsplit, scale_log2, part_o, part_ml, st);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
+                                  int nsplit, uint16_t* out, cudaStream_t st) {
     const dim3 grid(static_cast<unsigned>(s.n_q_heads), static_cast<unsigned>(s.batch));
     const size_t smem = sizeof(float) * static_cast<size_t>(nsplit);
     if (s.head_dim == 128)

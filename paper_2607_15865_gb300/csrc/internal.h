@@ -35,9 +35,11 @@ cudaError_t configure_flash_fwd();
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
                              const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st);
 
-// K3 + K4: split-KV decode over slots [0, hist[b]] and the log-sum-exp combine.
-cudaError_t launch_decode(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
-                          const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
-                          float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
+// K3: split-KV decode partials over slots [0, hist[b]]; K4: log-sum-exp combine into out.
+cudaError_t launch_decode_split(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
+                                const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
+                                float* part_ml, int nsplit, cudaStream_t st);
+cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
+                                  int nsplit, uint16_t* out, cudaStream_t st);
 
 }  // namespace attn

@@ -12,6 +12,13 @@ from synthetic import gen
 
 MAX_ABS = 2e-2
 MEAN_ABS = 2e-3
+# The absolute bar alone is loose here: outputs average N(0,1)/sqrt(D) values over
+# hundreds of keys, so |out| is ~1e-2..1e-3 and a zero output would pass it.  The
+# relative bar follows from the arithmetic: P is rounded to bf16 (relative error
+# <= 2^-9 per weight) and out is rounded to bf16 (<= 2^-9), so the error norm
+# stays well under 2^-7 of the output norm; 1e-2 leaves margin for float
+# accumulation order.
+REL = 1e-2
 f32 = gen.bf16_bits_to_f32
 
 
@@ -31,7 +38,9 @@ def assert_out_close(got_bits, ref_bits, what):
     err = np.abs(g - r)
     mx, mean = float(err.max()), float(err.mean())
     rel = float(np.linalg.norm(g - r) / max(np.linalg.norm(r), 1e-30))
+    print(f"[parity] {what}: max-abs {mx:.3e} mean-abs {mean:.3e} rel {rel:.3e} |ref|max {np.abs(r).max():.3e}")
     assert mx <= MAX_ABS and mean <= MEAN_ABS, f"{what}: max-abs {mx:.3e} mean-abs {mean:.3e} rel {rel:.3e}"
+    assert rel <= REL, f"{what}: relative error {rel:.3e} above {REL}"
     return mx, mean, rel
 
 
