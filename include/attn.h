@@ -159,6 +159,38 @@ int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
 int attn_timing_enable(attn_ctx* ctx, int max_launches);
 int attn_timing_read(attn_ctx* ctx, double* ms, long long* launches);
 
+/*
+ * Decode for callers that cannot allocate device memory.  The paper has no
+ * counterpart to this entry point; it exists for the library's users.
+ *
+ * Some callers cannot call cudaMalloc: code running inside a framework that owns
+ * all device memory and hands out only its own pre-reserved buffers, processes
+ * whose device memory is provisioned once up front, or callbacks that must not
+ * enter the allocator.  They cannot use attn_create, which allocates.  This call
+ * computes exactly what attn_decode computes, with no context and no allocation:
+ *   - the caller passes every input and output, including the RoPE tables d_cos,
+ *     d_sin (float [max_len][head_dim/2], row p column j holding cos / sin of
+ *     p * theta^(-2j/head_dim) evaluated in double and rounded to float -- the
+ *     table attn_create builds) and d_err, an int32 the caller zeroes and reads
+ *     back (it receives the ATTN_DEVERR_* bits, as attn_device_error reports);
+ *   - the split-KV partials live in a static device array of
+ *     ATTN_NOALLOC_SCRATCH_FLOATS floats (4 MiB) that every GPU which loads this
+ *     library holds until the process exits.  Shapes whose partials do not fit
+ *     even with one split (batch * n_q_heads * (head_dim + 2) > that size) are
+ *     rejected with ATTN_EINVAL; larger ones use fewer splits.
+ * All calls share that one array and nothing in it has to start at zero (every
+ * call rewrites the part it reads).  Calls whose kernels overlap on the GPU --
+ * on different streams, or from several threads -- race on it and must be
+ * serialised by the caller.  The first call on each device looks up the array's
+ * device address (cudaGetSymbolAddress, with that device current) and caches
+ * it; make that first call before any stream capture.  The other arguments and
+ * the errors are those of attn_decode; cfg is read on the host only.
+ */
+#define ATTN_NOALLOC_SCRATCH_FLOATS (1 << 20)
+int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_sin, const uint16_t* q,
+                        const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len, uint16_t* k_cache,
+                        uint16_t* v_cache, uint16_t* out, int32_t* d_err, attn_stream_t stream);
+
 /* Static text for an ATTN_* code. */
 const char* attn_strerror(int code);
 

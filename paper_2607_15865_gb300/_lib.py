@@ -18,7 +18,8 @@ DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
             "attn_device_error", "attn_timing_enable", "attn_timing_read", "attn_strerror",
-            "attn_last_cuda_error_string")
+            "attn_last_cuda_error_string", "attn_decode_noalloc")
+NOALLOC_SCRATCH_FLOATS = 1 << 20
 KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
 
 
@@ -67,6 +68,9 @@ def load(path: str = LIB_PATH):
     lib.attn_timing_enable.restype = i32
     lib.attn_timing_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_longlong)]
     lib.attn_timing_read.restype = i32
+    lib.attn_decode_noalloc.argtypes = [ctypes.POINTER(AttnCfg), vp, vp, u16p, u16p, u16p, vp, u16p, u16p, u16p,
+                                        vp, vp]
+    lib.attn_decode_noalloc.restype = i32
     lib.attn_strerror.argtypes = [i32]
     lib.attn_strerror.restype = ctypes.c_char_p
     lib.attn_last_cuda_error_string.argtypes = []

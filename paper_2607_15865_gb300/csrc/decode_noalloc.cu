@@ -1,0 +1,108 @@
+// decode_noalloc.cu -- attn_decode_noalloc: the decode stage for callers that cannot
+// allocate device memory.
+//
+// Who needs it: code that runs where cudaMalloc is not available or not allowed --
+// for example inside an allocator-owning framework that hands out only its own
+// pre-reserved buffers, in a process whose device memory is fully provisioned up
+// front, or in a callback that must not touch the allocator.  Such a caller cannot
+// create an attn_ctx (attn_create allocates the tables and the split-KV partials).
+//
+// This entry point runs the same kernels as attn_decode (K1 rope_append, K3
+// decode_split, K4 decode_combine) but needs no context: the caller passes every
+// input and output, including the RoPE tables and the error word, and the split-KV
+// partials live in the file-scope array below, which the library holds on every
+// device that loads it until the process exits.  Nothing is allocated or freed.
+//
+// Host code must not pass `g_noalloc_scratch` itself to a kernel: in host code that
+// name denotes a host-side shadow, not device memory.  The device address is looked
+// up with cudaGetSymbolAddress once per device (with that device current) on the
+// first call made on that device, and cached.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "../../include/attn.h"
+#include "internal.h"
+
+namespace {
+
+// Split-KV partials of attn_decode_noalloc: [B*Hq*nsplit*D] accumulators followed by
+// [B*Hq*nsplit*2] (max, sum) pairs.  Shared by every call on the device.
+static __device__ __align__(256) float g_noalloc_scratch[ATTN_NOALLOC_SCRATCH_FLOATS];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_setup_mutex;
+float* g_scratch_ptr[kMaxDevices] = {};
+int g_num_sms[kMaxDevices] = {};
+
+// Per-device set-up, on the current device: the device address of the scratch
+// array and the SM count.  Returns ATTN_OK, ATTN_EARCH or ATTN_ECUDA.
+int setup_device(int dev, float** scratch, int* num_sms) {
+    std::lock_guard<std::mutex> lock(g_setup_mutex);
+    if (g_scratch_ptr[dev] == nullptr) {
+        int major = 0, minor = 0, sms = 0;
+        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return ATTN_ECUDA;
+        if (major != 10 || minor != 3) return ATTN_EARCH;
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ATTN_ECUDA;
+        g_num_sms[dev] = sms;
+        g_scratch_ptr[dev] = static_cast<float*>(p);
+    }
+    *scratch = g_scratch_ptr[dev];
+    *num_sms = g_num_sms[dev];
+    return ATTN_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_sin, const uint16_t* q,
+                                   const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
+                                   uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, int32_t* d_err,
+                                   attn_stream_t stream) {
+    if (cfg == nullptr || d_cos == nullptr || d_sin == nullptr || q == nullptr || k == nullptr || v == nullptr ||
+        d_hist_len == nullptr || k_cache == nullptr || v_cache == nullptr || out == nullptr || d_err == nullptr)
+        return ATTN_EINVAL;
+    if (cfg->batch < 1 || cfg->batch > 65535 || cfg->n_q_heads < 1 || cfg->n_kv_heads < 1 ||
+        cfg->n_q_heads % cfg->n_kv_heads != 0 || cfg->n_q_heads / cfg->n_kv_heads > 16 ||
+        (cfg->head_dim != 64 && cfg->head_dim != 128) || cfg->max_len < 1 || cfg->max_len > (1 << 20))
+        return ATTN_EINVAL;
+    if (!aligned16(d_cos) || !aligned16(d_sin) || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+        !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out) ||
+        (reinterpret_cast<uintptr_t>(d_hist_len) & 3u) || (reinterpret_cast<uintptr_t>(d_err) & 3u))
+        return ATTN_EINVAL;
+    // Partials need B*Hq*(D+2) floats per split; at least one split must fit.
+    const long long per_split = static_cast<long long>(cfg->batch) * cfg->n_q_heads * (cfg->head_dim + 2);
+    if (per_split > ATTN_NOALLOC_SCRATCH_FLOATS) return ATTN_EINVAL;
+
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ATTN_ECUDA;
+    float* scratch = nullptr;
+    int num_sms = 0;
+    const int rc = setup_device(dev, &scratch, &num_sms);
+    if (rc != ATTN_OK) return rc;
+
+    // Same split rule as attn_decode, further capped by what the scratch array holds.
+    const int G = cfg->n_q_heads / cfg->n_kv_heads;
+    const long long items = static_cast<long long>(cfg->batch) * cfg->n_kv_heads * ((G + 7) / 8);
+    long long ns = (4LL * num_sms + items - 1) / items;
+    ns = ns > (cfg->max_len + 63) / 64 ? (cfg->max_len + 63) / 64 : ns;
+    ns = ns > 256 ? 256 : ns;
+    ns = ns > ATTN_NOALLOC_SCRATCH_FLOATS / per_split ? ATTN_NOALLOC_SCRATCH_FLOATS / per_split : ns;
+    ns = ns < 1 ? 1 : ns;
+    const int nsplit = static_cast<int>(ns);
+    float* part_o = scratch;
+    float* part_ml = scratch + static_cast<size_t>(cfg->batch) * cfg->n_q_heads * nsplit * cfg->head_dim;
+
+    const attn::Shape s{cfg->batch, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, cfg->max_len};
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = attn::launch_rope_append(s, k, v, 0, d_hist_len, 1, d_cos, d_sin, k_cache, v_cache, d_err, st);
+    if (e == cudaSuccess)
+        e = attn::launch_decode_split(s, q, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o, part_ml, nsplit, st);
+    if (e == cudaSuccess) e = attn::launch_decode_combine(s, d_hist_len, part_o, part_ml, nsplit, out, st);
+    return e == cudaSuccess ? ATTN_OK : ATTN_ECUDA;
+}
