@@ -5,8 +5,8 @@
 // the kernels of each stage on the caller's stream:
 //   prefill / prefill_kv : K1 rope_append (new k rotated + k, v appended in place)
 //                          -> K2 flash_fwd (q rotated in-kernel, causal attention)
-//   decode               : K1 rope_append (slot hist_len[b], read on the device)
-//                          -> K3 decode_split -> K4 decode_combine
+//   decode               : K3 decode_split (new k rotated + k, v appended at slot
+//                          hist_len[b], read on the device) -> K4 decode_combine
 // No call allocates, frees or synchronises except attn_create/attn_destroy and
 // attn_device_error.
 #include <cuda.h>
@@ -34,6 +34,10 @@ struct attn_ctx {
     float* d_part_ml;
     int* d_err;
     PFN_cuTensorMapEncodeTiled_v12000 encode;
+    // decode tensor maps of the last cache pair seen
+    const uint16_t* dec_k;
+    const uint16_t* dec_v;
+    attn::DecodeMaps dec_maps;
     // kernel timing: event pairs recorded around each launch while enabled
     std::vector<cudaEvent_t> ev;
     std::vector<int> ev_kind;
@@ -61,20 +65,6 @@ bool cfg_valid(const attn_cfg* c) {
     if (c->max_len < 1 || c->max_len > (1 << 20)) return false;
     if (!(c->rope_theta > 0.0) || !std::isfinite(c->rope_theta)) return false;
     return true;
-}
-
-// Split count of the decode: enough CTAs for ~4 per SM over B*Hkv*passes work
-// items, at most one split per 64 cache slots of the static maximum length.
-int decode_nsplit(const attn_ctx* c) {
-    const int G = c->cfg.n_q_heads / c->cfg.n_kv_heads;
-    const int passes = (G + 7) / 8;
-    const long items = static_cast<long>(c->cfg.batch) * c->cfg.n_kv_heads * passes;
-    long ns = (4L * c->num_sms + items - 1) / items;
-    const long cap = (c->cfg.max_len + 63) / 64;
-    if (ns > cap) ns = cap;
-    if (ns > c->nsplit_max) ns = c->nsplit_max;
-    if (ns < 1) ns = 1;
-    return static_cast<int>(ns);
 }
 
 // Enqueue one kernel through `launch`, bracketed by a timing event pair when enabled.
@@ -189,9 +179,10 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     }
     c->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     e = attn::configure_flash_fwd();
+    if (e == cudaSuccess) e = attn::configure_decode();
     if (e != cudaSuccess) {
         delete c;
-        return cuda_fail(e, "configure flash_fwd");
+        return cuda_fail(e, "configure kernels");
     }
 
     // RoPE tables (Section 4.6.2): cos/sin of p * theta^(-2j/D), evaluated in double, stored as float.
@@ -262,15 +253,19 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         !aligned16(out) || (reinterpret_cast<uintptr_t>(d_hist_len) & 3u))
         return ATTN_EINVAL;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    const int nsplit = decode_nsplit(c);
-    cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&] {
-        return attn::launch_rope_append(c->shape, k, v, 0, d_hist_len, 1, c->d_cos, c->d_sin, k_cache, v_cache,
-                                        c->d_err, st);
-    });
-    if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
-    e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&] {
-        return attn::launch_decode_split(c->shape, q, d_hist_len, k_cache, v_cache, c->d_cos, c->d_sin, c->d_part_o,
-                                         c->d_part_ml, nsplit, st);
+    if (k_cache != c->dec_k || v_cache != c->dec_v) {
+        if (attn::make_decode_maps(c->encode, c->shape, k_cache, v_cache, &c->dec_maps) != cudaSuccess) {
+            c->dec_k = c->dec_v = nullptr;
+            std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "cuTensorMapEncodeTiled failed for the decode caches");
+            return ATTN_ECUDA;
+        }
+        c->dec_k = k_cache;
+        c->dec_v = v_cache;
+    }
+    const int nsplit = attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
+    cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&] {
+        return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
+                                         c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
     e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&] {

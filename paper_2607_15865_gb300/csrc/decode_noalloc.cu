@@ -7,8 +7,8 @@
 // front, or in a callback that must not touch the allocator.  Such a caller cannot
 // create an attn_ctx (attn_create allocates the tables and the split-KV partials).
 //
-// This entry point runs the same kernels as attn_decode (K1 rope_append, K3
-// decode_split, K4 decode_combine) but needs no context: the caller passes every
+// This entry point runs the same kernels as attn_decode (K3 decode_split with the
+// new token's append, K4 decode_combine) but needs no context: the caller passes every
 // input and output, including the RoPE tables and the error word, and the split-KV
 // partials live in the file-scope array below, which the library holds on every
 // device that loads it until the process exits.  Nothing is allocated or freed.
@@ -34,11 +34,22 @@ constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
 float* g_scratch_ptr[kMaxDevices] = {};
 int g_num_sms[kMaxDevices] = {};
+attn::PFN_encodeTiled g_encode = nullptr;
 
 // Per-device set-up, on the current device: the device address of the scratch
-// array and the SM count.  Returns ATTN_OK, ATTN_EARCH or ATTN_ECUDA.
+// array, the SM count, the kernels' shared-memory limits and (once per process)
+// the driver's tensor-map encoder.  Returns ATTN_OK, ATTN_EARCH or ATTN_ECUDA.
 int setup_device(int dev, float** scratch, int* num_sms) {
     std::lock_guard<std::mutex> lock(g_setup_mutex);
+    if (g_encode == nullptr) {
+        cudaDriverEntryPointQueryResult qres;
+        void* fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qres) !=
+                cudaSuccess ||
+            qres != cudaDriverEntryPointSuccess || fn == nullptr)
+            return ATTN_ECUDA;
+        g_encode = reinterpret_cast<attn::PFN_encodeTiled>(fn);
+    }
     if (g_scratch_ptr[dev] == nullptr) {
         int major = 0, minor = 0, sms = 0;
         if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
@@ -48,6 +59,7 @@ int setup_device(int dev, float** scratch, int* num_sms) {
         if (major != 10 || minor != 3) return ATTN_EARCH;
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ATTN_ECUDA;
+        if (attn::configure_decode() != cudaSuccess) return ATTN_ECUDA;
         g_num_sms[dev] = sms;
         g_scratch_ptr[dev] = static_cast<float*>(p);
     }
@@ -86,23 +98,18 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     const int rc = setup_device(dev, &scratch, &num_sms);
     if (rc != ATTN_OK) return rc;
 
-    // Same split rule as attn_decode, further capped by what the scratch array holds.
-    const int G = cfg->n_q_heads / cfg->n_kv_heads;
-    const long long items = static_cast<long long>(cfg->batch) * cfg->n_kv_heads * ((G + 7) / 8);
-    long long ns = (4LL * num_sms + items - 1) / items;
-    ns = ns > (cfg->max_len + 63) / 64 ? (cfg->max_len + 63) / 64 : ns;
-    ns = ns > 256 ? 256 : ns;
-    ns = ns > ATTN_NOALLOC_SCRATCH_FLOATS / per_split ? ATTN_NOALLOC_SCRATCH_FLOATS / per_split : ns;
-    ns = ns < 1 ? 1 : ns;
-    const int nsplit = static_cast<int>(ns);
+    // Same split rule as attn_decode, capped by what the scratch array holds.
+    const attn::Shape s{cfg->batch, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, cfg->max_len};
+    const long long fit = ATTN_NOALLOC_SCRATCH_FLOATS / per_split;
+    const int nsplit = attn::decode_num_splits(s, num_sms, static_cast<int>(fit < 256 ? fit : 256));
     float* part_o = scratch;
     float* part_ml = scratch + static_cast<size_t>(cfg->batch) * cfg->n_q_heads * nsplit * cfg->head_dim;
 
-    const attn::Shape s{cfg->batch, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, cfg->max_len};
+    attn::DecodeMaps maps;
+    if (attn::make_decode_maps(g_encode, s, k_cache, v_cache, &maps) != cudaSuccess) return ATTN_ECUDA;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = attn::launch_rope_append(s, k, v, 0, d_hist_len, 1, d_cos, d_sin, k_cache, v_cache, d_err, st);
-    if (e == cudaSuccess)
-        e = attn::launch_decode_split(s, q, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o, part_ml, nsplit, st);
+    cudaError_t e = attn::launch_decode_split(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o,
+                                              part_ml, nsplit, d_err, st);
     if (e == cudaSuccess) e = attn::launch_decode_combine(s, d_hist_len, part_o, part_ml, nsplit, out, st);
     return e == cudaSuccess ? ATTN_OK : ATTN_ECUDA;
 }

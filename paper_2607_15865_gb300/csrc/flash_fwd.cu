@@ -104,9 +104,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int qt = n_qtiles - 1 - static_cast<int>(blockIdx.x);  // longest rows first
-    const int h = blockIdx.y;
-    const int b = blockIdx.z;
+    // Longest rows first across every (head, sequence): with a causal mask the last
+    // query tiles see the most keys, so they are dispatched before all shorter ones.
+    const int heads_x_batch = static_cast<int>(gridDim.x) / n_qtiles;  // Hq * B
+    const int lin = static_cast<int>(blockIdx.x);
+    const int qt = n_qtiles - 1 - lin / heads_x_batch;
+    const int h = (lin % heads_x_batch) % Hq;
+    const int b = (lin % heads_x_batch) / Hq;
     const int g = h / (Hq / Hkv);
     const int q0 = qt * BM;
     const int rows_valid = min(BM, S - q0);
@@ -314,8 +318,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(r[c][e]));
             }
-            const float m_new = fmaxf(m_run, mx * scale_log2);
-            const float alpha = fast_exp2(m_run - m_new);
+            // Lazy rescaling: P is taken relative to a reference max m_run that only moves
+            // when the row max exceeds it by more than 2^8 (P <= 256 otherwise, exact in
+            // bf16/fp32 ranges), so O and l are rescaled rarely; the result is unchanged.
+            const float m_cand = fmaxf(m_run, mx * scale_log2);
+            const bool move = m_cand > m_run + 8.f;  // always true on the first tile
+            const float m_new = move ? m_cand : m_run;
+            const float alpha = move ? fast_exp2(m_run - m_new) : 1.f;
             const float neg_m = -m_new;
             float rowsum = 0.f;
             uint8_t* pbuf = gbase + L::OFF_P + st * L::P_BYTES;
@@ -397,8 +406,7 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
                      const float* sin_tab, uint16_t* out, int* err, cudaStream_t st) {
     const int n_qtiles = (chunk + BM - 1) / BM;
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
-    const dim3 grid(static_cast<unsigned>(n_qtiles), static_cast<unsigned>(s.n_q_heads),
-                    static_cast<unsigned>(s.batch));
+    const dim3 grid(static_cast<unsigned>(n_qtiles) * s.n_q_heads * s.batch);
     flash_fwd_kernel<D><<<grid, kThreads, Layout<D>::ALLOC, st>>>(maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads,
                                                                    s.n_kv_heads, n_qtiles, scale_log2, cos_tab,
                                                                    sin_tab, out, err);

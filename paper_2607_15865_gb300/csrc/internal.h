@@ -4,6 +4,7 @@
 
 #include <cstdint>
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 namespace attn {
@@ -35,10 +36,22 @@ cudaError_t configure_flash_fwd();
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
                              const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st);
 
-// K3: split-KV decode partials over slots [0, hist[b]]; K4: log-sum-exp combine into out.
-cudaError_t launch_decode_split(const Shape& s, const uint16_t* q, const int32_t* d_hist, const uint16_t* k_cache,
-                                const uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
-                                float* part_ml, int nsplit, cudaStream_t st);
+// K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
+// with 64-key boxes (built once per cache pair).  K3 also rotates the new key and
+// appends k and v at slot hist[b]; K4 merges the splits (programmatic dependent launch).
+using PFN_encodeTiled = PFN_cuTensorMapEncodeTiled_v12000;
+struct DecodeMaps {
+    CUtensorMap k;
+    CUtensorMap v;
+};
+cudaError_t configure_decode();  // dynamic shared-memory limits of K3 (once per device)
+int decode_num_splits(const Shape& s, int num_sms, int max_splits);
+cudaError_t make_decode_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
+                             const uint16_t* v_cache, DecodeMaps* maps);
+cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
+                                const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
+                                const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
+                                int nsplit, int* err, cudaStream_t st);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
                                   int nsplit, uint16_t* out, cudaStream_t st);
 
