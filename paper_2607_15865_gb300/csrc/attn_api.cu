@@ -19,7 +19,7 @@
 #include <new>
 #include <vector>
 
-#include "../../include/attn.h"
+#include "attn.h"
 #include "internal.h"
 
 struct attn_ctx {

@@ -21,7 +21,7 @@
 
 #include <mutex>
 
-#include "../../include/attn.h"
+#include "attn.h"
 #include "internal.h"
 
 namespace {

@@ -1,6 +1,6 @@
 // flash_fwd.cu -- K2: causal flash attention for prefill and prefill_kv on sm_103a.
 //
-// What it computes (Section 4.2-4.3; FAttention of Section 2.2 with the causal
+// What it computes (Sections 4.2-4.3; FAttention of Section 2.2 with the causal
 // mask of Section 4.6.1): for the chunk's query rows i at positions p = hist + i
 // and every query head h, out[b, i, h, :] = softmax_j(q_rot . k_j / sqrt(D)) v_j
 // over cache slots j <= p of kv head h / G.  The caches already hold the chunk's
@@ -9,26 +9,34 @@
 // in-place layout itself.  prefill is the same kernel with hist = 0 (the paper's
 // with_history template, Section 4.2).
 //
-// Design (one CTA = one 128-row query tile of one head; 192 threads):
-//   warp 4      TMA producer: the q tile (4-D map straight from q [B,S,Hq,D]),
-//               then K and V tiles of 128 keys into a 2-stage ring (128-byte
-//               swizzle; rows past hist+chunk are zero-filled by the map bounds,
-//               so unwritten cache slots are never read);
-//   warp 5      tcgen05 issuer: S = Q K^T into one of two TMEM score buffers
-//               (M=128, N=128, K=16 steps), then O += P V into the TMEM
-//               accumulator (V as an MN-major operand);
-//   warps 0-3   one thread per query row (= TMEM lane): RoPE of the q row in
-//               shared memory before the first MMA (cos/sin gathered by position,
-//               Section 4.6.2, float arithmetic, bf16 rounding as K1), then per
-//               KV tile: scores from TMEM, causal mask by index compare (no mask
-//               tensor), online softmax in the log2 domain, P as bf16 into a
-//               swizzled shared buffer (double-buffered), rescale of the O row in
-//               TMEM when the running maximum grew; finally O / l -> bf16 -> out.
-// The MMA of tile j+1 overlaps the softmax of tile j (two score buffers).
+// Design.  A persistent CTA per SM walks a static list of work items sorted
+// longest-first.  An item is two 128-row query tiles (A, B) of one head, so each
+// K/V tile is brought in once for 256 queries.  384 threads, three warpgroups:
+//   WG0 (warps 0-3)   softmax + epilogue of tile A (one thread per row = TMEM lane)
+//   WG1 (warps 4-7)   softmax + epilogue of tile B
+//   WG2 (warps 8-11)  warp 8: TMA producer (lane 0: q tiles from a 4-D map of
+//                     q [B,S,Hq,D] and the K ring; lane 1: the V ring), warp 9:
+//                     tcgen05 issuer, warps 10-11 idle.  WG2 gives registers to
+//                     the softmax warpgroups (setmaxnreg 56 / 224 of 168 at launch).
+// K tiles (128 keys, 2-stage ring) and V tiles (3-stage ring) use the 128-byte
+// swizzle; rows past hist+chunk are zero-filled by the map bounds, never read.
+// Per KV tile j the issuer runs PV_A(j-1), S_A(j), PV_B(j-1), S_B(j).
+// TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [256+D,256+2D).
+// P is written back as bf16 over the first 64 columns of its S and fed to the PV
+// MMA from TMEM, so the two warpgroups ping-pong: while one turns its scores into
+// P, the tensor core runs the other tile's MMAs.  A commit covers every earlier
+// MMA of the issuing thread, so "S_T(j) complete" implies "PV_T(j-1) complete":
+// the softmax warpgroup may rescale O_T right away.  O is rescaled lazily (only
+// when the running max grows by more than 2^8, exact in value).
+// Per row: RoPE of the q row in shared memory before the first MMA (cos/sin
+// gathered by position, Section 4.6.2, float arithmetic and bf16 rounding as K1),
+// scores from TMEM, causal mask by index compare on diagonal tiles (no mask
+// tensor), online softmax in the log2 domain, O / l -> bf16 -> out.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its
 // in-flight copies and MMAs finish, releases TMEM and exits.
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cmath>
 
 #include "internal.h"
@@ -39,47 +47,50 @@ namespace {
 
 constexpr int BM = 128;  // query rows per tile (TMEM lanes)
 constexpr int BN = 128;  // keys per KV tile
-constexpr int kThreads = 192;
-constexpr int kWarpTma = 4;
-constexpr int kWarpMma = 5;
-constexpr uint32_t kTmemCols = 512;  // S0 [0,128) S1 [128,256) O [256,256+D)
+constexpr int kThreads = 384;
+constexpr int kWarpTma = 8;
+constexpr int kWarpMma = 9;
+constexpr uint32_t kTmemCols = 512;
+constexpr int KS = 2;  // K ring stages
+constexpr int VS = 3;  // V ring stages
+// Register budgets: 168 per thread at launch (65536 / 384, rounded down to 8);
+// WG2 gives back 112 per thread, the two softmax warpgroups take 56 each.
+constexpr int kLaunchRegs = 168;
+constexpr uint32_t kRegsLow = 56;
+constexpr uint32_t kRegsHigh = 224;
+static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split exceeds the launch total");
 
 enum Bar {
-    B_QFULL, B_QREADY,
+    B_QFULL, B_QREADY, B_QEMPTY,
     B_KFULL0, B_KFULL1, B_KEMPTY0, B_KEMPTY1,
-    B_VFULL0, B_VFULL1, B_VEMPTY0, B_VEMPTY1,
+    B_VFULL0, B_VFULL1, B_VFULL2, B_VEMPTY0, B_VEMPTY1, B_VEMPTY2,
     B_SFULL0, B_SFULL1, B_PFULL0, B_PFULL1,
-    B_PVDONE, B_DRAIN, NBAR
+    B_OFULL0, B_OFULL1, B_OEMPTY0, B_OEMPTY1,
+    B_DRAIN, NBAR
 };
 
 template <int D>
 struct Layout {
-    static constexpr int DCH = D / 64;          // 64-column (128-byte) chunks of a row
-    static constexpr int CHUNK = 128 * 128;     // bytes of one 128-row x 128-byte chunk
-    static constexpr int Q_BYTES = DCH * CHUNK;
-    static constexpr int KV_BYTES = DCH * CHUNK;
-    static constexpr int P_BYTES = (BN / 64) * CHUNK;
-    static constexpr int OFF_Q = 0;
-    static constexpr int OFF_K = OFF_Q + Q_BYTES;
-    static constexpr int OFF_V = OFF_K + 2 * KV_BYTES;
-    static constexpr int OFF_P = OFF_V + 2 * KV_BYTES;
-    static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
+    static constexpr int DCH = D / 64;       // 64-column (128-byte) chunks of a row
+    static constexpr int CHUNK = 128 * 128;  // bytes of one 128-row x 128-byte chunk
+    static constexpr int Q_TILE = DCH * CHUNK;
+    static constexpr int KV_TILE = DCH * CHUNK;
+    static constexpr int OFF_Q = 0;                      // q tiles A, B
+    static constexpr int OFF_K = OFF_Q + 2 * Q_TILE;     // K ring
+    static constexpr int OFF_V = OFF_K + KS * KV_TILE;   // V ring
+    static constexpr int OFF_BAR = OFF_V + VS * KV_TILE;
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
     static constexpr int OFF_ABORT = OFF_TMEM + 8;
     static constexpr int BYTES = OFF_ABORT + 8;
     static constexpr int ALLOC = BYTES + 1024;  // slack to align the base to 1024 bytes
+    static constexpr uint32_t TM_O = 2 * BN;    // TMEM column of O_A; O_B at TM_O + D
 };
 static_assert(Layout<128>::ALLOC <= 232448, "shared memory budget of one CTA");
 
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    const __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&t);
-}
-
-// Byte offset of the 16-byte unit holding columns [8u, 8u+8) of row r inside a
+// Byte offset of the 16-byte unit holding columns [col, col+8) of row `row` inside a
 // 128-row tile stored as 128-byte-swizzled 64-column chunks (TMA SWIZZLE_128B).
 __device__ __forceinline__ uint32_t sw128_offset(int row, int col) {
     const int chunk = col >> 6;
@@ -87,12 +98,100 @@ __device__ __forceinline__ uint32_t sw128_offset(int row, int col) {
     return static_cast<uint32_t>(chunk * (128 * 128) + row * 128 + ((unit ^ (row & 7)) << 4));
 }
 
+// One work item: query tiles A (rows q0(0)..) and B (rows q0(1)..) of head h, sequence b.
+// Scalar fields with select accessors keep every field in registers when the tile
+// index is only known at run time.
+struct Item {
+    int h, b, g;
+    int q0a, q0b;
+    int rowsa, rowsb;  // valid rows of each tile (0: tile absent)
+    int nkva, nkvb;    // KV tiles each tile attends to
+    int n_kv;          // KV tiles loaded for the item
+    __device__ __forceinline__ int q0(int t) const { return t ? q0b : q0a; }
+    __device__ __forceinline__ int rows(int t) const { return t ? rowsb : rowsa; }
+    __device__ __forceinline__ int nkv(int t) const { return t ? nkvb : nkva; }
+};
+
+// Item order: longest query-tile pairs first across every (head, sequence), so a
+// causal launch starts its longest items first and ends with the shortest.
+__device__ __forceinline__ Item decode_item(int lin, int S, int H, int Hq, int G, int hq_b, int n_pairs) {
+    Item it;
+    const int pt = n_pairs - 1 - lin / hq_b;
+    const int rem = lin % hq_b;
+    it.h = rem % Hq;
+    it.b = rem / Hq;
+    it.g = it.h / G;
+    it.q0a = pt * 2 * BM;
+    it.q0b = it.q0a + BM;
+    it.rowsa = max(0, min(BM, S - it.q0a));
+    it.rowsb = max(0, min(BM, S - it.q0b));
+    it.nkva = it.rowsa ? (H + it.q0a + it.rowsa + BN - 1) / BN : 0;
+    it.nkvb = it.rowsb ? (H + it.q0b + it.rowsb + BN - 1) / BN : 0;
+    it.n_kv = max(it.nkva, it.nkvb);
+    return it;
+}
+
+// RoPE of one q row of a tile in shared memory (pairs j, j + D/2, table row of its
+// position, float arithmetic with each product and the difference/sum rounded
+// separately, bf16 result), as K1 applies to keys.
+template <int D>
+__device__ __forceinline__ void rope_row_smem(uint8_t* qtile, int row, int pos, const float* __restrict__ cos_tab,
+                                              const float* __restrict__ sin_tab) {
+    constexpr int HALF = D / 2;
+    const float* crow = cos_tab + static_cast<size_t>(pos) * HALF;
+    const float* srow = sin_tab + static_cast<size_t>(pos) * HALF;
+#pragma unroll
+    for (int u = 0; u < HALF / 8; ++u) {
+        const int jlo = 8 * u;
+        uint4* plo = reinterpret_cast<uint4*>(qtile + sw128_offset(row, jlo));
+        uint4* phi = reinterpret_cast<uint4*>(qtile + sw128_offset(row, jlo + HALF));
+        const uint4 xa = *plo, xb = *phi;
+        const float4 c0 = *reinterpret_cast<const float4*>(crow + jlo);
+        const float4 c1 = *reinterpret_cast<const float4*>(crow + jlo + 4);
+        const float4 s0 = *reinterpret_cast<const float4*>(srow + jlo);
+        const float4 s1 = *reinterpret_cast<const float4*>(srow + jlo + 4);
+        const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+        const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        const uint32_t wa[4] = {xa.x, xa.y, xa.z, xa.w};
+        const uint32_t wb[4] = {xb.x, xb.y, xb.z, xb.w};
+        uint32_t ya[4], yb[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            float lo[2], hi[2];
+#pragma unroll
+            for (int k2 = 0; k2 < 2; ++k2) {
+                const float a = k2 ? bf_hi(wa[e]) : bf_lo(wa[e]);
+                const float bb = k2 ? bf_hi(wb[e]) : bf_lo(wb[e]);
+                const float cc = c[2 * e + k2], ss = s[2 * e + k2];
+                lo[k2] = __fsub_rn(__fmul_rn(a, cc), __fmul_rn(bb, ss));
+                hi[k2] = __fadd_rn(__fmul_rn(bb, cc), __fmul_rn(a, ss));
+            }
+            ya[e] = pack_bf16x2(lo[0], lo[1]);
+            yb[e] = pack_bf16x2(hi[0], hi[1]);
+        }
+        *plo = make_uint4(ya[0], ya[1], ya[2], ya[3]);
+        *phi = make_uint4(yb[0], yb[1], yb[2], yb[3]);
+    }
+}
+
+// Wait for an item's q tiles, rotate this thread's row, hand Q to the MMA warp.
+template <int D>
+__device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint32_t parity, const volatile int* abort,
+                                          uint8_t* qtile, int row, int rows, int pos0,
+                                          const float* __restrict__ cos_tab, const float* __restrict__ sin_tab) {
+    const bool w = __all_sync(0xFFFFFFFFu, mbar_wait(qfull, parity, abort));
+    if (w && row < rows) rope_row_smem<D>(qtile, row, pos0 + row, cos_tab, sin_tab);
+    fence_proxy_async_smem();
+    mbar_arrive(qready);
+    return w;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                     const __grid_constant__ CUtensorMap map_v, int S, int H, int Hq, int Hkv, int n_qtiles,
-                     float scale_log2, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab,
-                     uint16_t* __restrict__ out, int* __restrict__ err) {
+                     const __grid_constant__ CUtensorMap map_v, int S, int H, int Hq, int Hkv, int batch,
+                     int n_pairs, float scale_log2, const float* __restrict__ cos_tab,
+                     const float* __restrict__ sin_tab, uint16_t* __restrict__ out, int* __restrict__ err) {
     using L = Layout<D>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -104,31 +203,29 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    // Longest rows first across every (head, sequence): with a causal mask the last
-    // query tiles see the most keys, so they are dispatched before all shorter ones.
-    const int heads_x_batch = static_cast<int>(gridDim.x) / n_qtiles;  // Hq * B
-    const int lin = static_cast<int>(blockIdx.x);
-    const int qt = n_qtiles - 1 - lin / heads_x_batch;
-    const int h = (lin % heads_x_batch) % Hq;
-    const int b = (lin % heads_x_batch) / Hq;
-    const int g = h / (Hq / Hkv);
-    const int q0 = qt * BM;
-    const int rows_valid = min(BM, S - q0);
-    const int n_kv = (H + q0 + rows_valid + BN - 1) / BN;
+    const int G = Hq / Hkv;
+    const int hq_b = Hq * batch;
+    const int n_items = n_pairs * hq_b;
 
     if (threadIdx.x == 0) {
         *abort_flag = 0;
         mbar_init(bar(B_QFULL), 1);
-        mbar_init(bar(B_QREADY), BM);
-        for (int st = 0; st < 2; ++st) {
+        mbar_init(bar(B_QREADY), 2 * BM);
+        mbar_init(bar(B_QEMPTY), 1);
+        for (int st = 0; st < KS; ++st) {
             mbar_init(bar(B_KFULL0 + st), 1);
             mbar_init(bar(B_KEMPTY0 + st), 1);
+        }
+        for (int st = 0; st < VS; ++st) {
             mbar_init(bar(B_VFULL0 + st), 1);
             mbar_init(bar(B_VEMPTY0 + st), 1);
-            mbar_init(bar(B_SFULL0 + st), 1);
-            mbar_init(bar(B_PFULL0 + st), BM);
         }
-        mbar_init(bar(B_PVDONE), 1);
+        for (int t = 0; t < 2; ++t) {
+            mbar_init(bar(B_SFULL0 + t), 1);
+            mbar_init(bar(B_PFULL0 + t), BM);
+            mbar_init(bar(B_OFULL0 + t), 1);
+            mbar_init(bar(B_OEMPTY0 + t), BM);
+        }
         mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
     }
@@ -141,94 +238,155 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
 
-    if (warp == kWarpTma) {
-        // ------------------------------------------------------------ TMA producer
-        if (lane == 0) {
+    if (warp >= 8) {
+        warpgroup_reg_dec<kRegsLow>();
+        if (warp == kWarpTma && lane == 0) {
+            // ---------------------------------------------------- q tiles and the K ring
             tma_prefetch_desc(&map_q);
             tma_prefetch_desc(&map_k);
-            tma_prefetch_desc(&map_v);
-            mbar_arrive_expect_tx(bar(B_QFULL), L::Q_BYTES);
-#pragma unroll
-            for (int c = 0; c < L::DCH; ++c)
-                tma_load_4d(base + L::OFF_Q + c * L::CHUNK, &map_q, c * 64, h, q0, b, bar(B_QFULL));
-            const int kv_row = b * Hkv + g;
-            int issued_k[2] = {0, 0}, issued_v[2] = {0, 0};
+            uint32_t kc = 0;  // K tiles issued
+            int items = 0;
             bool ok = true;
-            for (int j = 0; j < n_kv; ++j) {
-                const int st = j & 1;
-                const uint32_t ph_free = static_cast<uint32_t>((j - 2) >> 1) & 1u;
-                if (j >= 2 && !mbar_wait(bar(B_KEMPTY0 + st), ph_free, abort_flag)) { ok = false; break; }
-                mbar_arrive_expect_tx(bar(B_KFULL0 + st), L::KV_BYTES);
+            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
+                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+                if (items > 0 && !mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                mbar_arrive_expect_tx(bar(B_QFULL), 2 * L::Q_TILE);
 #pragma unroll
-                for (int c = 0; c < L::DCH; ++c)
-                    tma_load_3d(base + L::OFF_K + st * L::KV_BYTES + c * L::CHUNK, &map_k, c * 64, j * BN, kv_row,
-                                bar(B_KFULL0 + st));
-                ++issued_k[st];
-                if (j >= 2 && !mbar_wait(bar(B_VEMPTY0 + st), ph_free, abort_flag)) { ok = false; break; }
-                mbar_arrive_expect_tx(bar(B_VFULL0 + st), L::KV_BYTES);
+                for (int t = 0; t < 2; ++t)
 #pragma unroll
-                for (int c = 0; c < L::DCH; ++c)
-                    tma_load_3d(base + L::OFF_V + st * L::KV_BYTES + c * L::CHUNK, &map_v, c * 64, j * BN, kv_row,
-                                bar(B_VFULL0 + st));
-                ++issued_v[st];
+                    for (int c = 0; c < L::DCH; ++c)
+                        tma_load_4d(base + L::OFF_Q + t * L::Q_TILE + c * L::CHUNK, &map_q, c * 64, it.h, it.q0(t),
+                                    it.b, bar(B_QFULL));
+                ++items;
+                const int kv_row = it.b * Hkv + it.g;
+                for (int j = 0; j < it.n_kv; ++j, ++kc) {
+                    const int st = static_cast<int>(kc % KS);
+                    if (kc >= KS && !mbar_wait(bar(B_KEMPTY0 + st), (kc / KS - 1u) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(bar(B_KFULL0 + st), L::KV_TILE);
+#pragma unroll
+                    for (int c = 0; c < L::DCH; ++c)
+                        tma_load_3d(base + L::OFF_K + st * L::KV_TILE + c * L::CHUNK, &map_k, c * 64, j * BN, kv_row,
+                                    bar(B_KFULL0 + st));
+                }
             }
             if (!ok) {
                 *abort_flag = 1;
                 atomicOr(err, kDevErrTimeout);
+                // every copy issued must land before the CTA may exit
+                if (items > 0) mbar_wait(bar(B_QFULL), static_cast<uint32_t>(items - 1) & 1u, nullptr);
+                for (uint32_t t = kc >= KS ? kc - KS : 0; t < kc; ++t)
+                    mbar_wait(bar(B_KFULL0 + static_cast<int>(t % KS)), (t / KS) & 1u, nullptr);
             }
-            // Every copy this thread issued must have landed before the CTA may exit.
-            mbar_wait(bar(B_QFULL), 0, nullptr);
-            for (int st = 0; st < 2; ++st) {
-                if (issued_k[st]) mbar_wait(bar(B_KFULL0 + st), static_cast<uint32_t>(issued_k[st] - 1) & 1u, nullptr);
-                if (issued_v[st]) mbar_wait(bar(B_VFULL0 + st), static_cast<uint32_t>(issued_v[st] - 1) & 1u, nullptr);
+        } else if (warp == kWarpTma && lane == 1) {
+            // ---------------------------------------------------- the V ring
+            tma_prefetch_desc(&map_v);
+            uint32_t vc = 0;  // V tiles issued
+            bool ok = true;
+            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
+                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+                const int kv_row = it.b * Hkv + it.g;
+                for (int j = 0; j < it.n_kv; ++j, ++vc) {
+                    const int st = static_cast<int>(vc % VS);
+                    if (vc >= VS && !mbar_wait(bar(B_VEMPTY0 + st), (vc / VS - 1u) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(bar(B_VFULL0 + st), L::KV_TILE);
+#pragma unroll
+                    for (int c = 0; c < L::DCH; ++c)
+                        tma_load_3d(base + L::OFF_V + st * L::KV_TILE + c * L::CHUNK, &map_v, c * 64, j * BN, kv_row,
+                                    bar(B_VFULL0 + st));
+                }
             }
-        }
-    } else if (warp == kWarpMma) {
-        // ------------------------------------------------------------ tcgen05 issuer
-        if (lane == 0) {
+            if (!ok) {
+                *abort_flag = 1;
+                atomicOr(err, kDevErrTimeout);
+                for (uint32_t t = vc >= VS ? vc - VS : 0; t < vc; ++t)
+                    mbar_wait(bar(B_VFULL0 + static_cast<int>(t % VS)), (t / VS) & 1u, nullptr);
+            }
+        } else if (warp == kWarpMma && lane == 0) {
+            // ---------------------------------------------------- tcgen05 issuer
             constexpr uint32_t kIdS = idesc_bf16_f32(BM, BN, false, false);
             constexpr uint32_t kIdPV = idesc_bf16_f32(BM, D, false, true);
-            const uint32_t sQ = base + L::OFF_Q;
-            const uint32_t o_tmem = tmem + 2 * BN;
-            auto issue_pv = [&](int jj) -> bool {
-                const int st = jj & 1;
-                const uint32_t ph = static_cast<uint32_t>(jj >> 1) & 1u;
-                if (!mbar_wait(bar(B_PFULL0 + st), ph, abort_flag)) return false;
-                if (!mbar_wait(bar(B_VFULL0 + st), ph, abort_flag)) return false;
-                tc_fence_after();
-                const uint32_t sP = base + L::OFF_P + st * L::P_BYTES;
-                const uint32_t sV = base + L::OFF_V + st * L::KV_BYTES;
+            uint32_t kvc = 0;
+            uint32_t p_cnt[2] = {0u, 0u};  // P tiles consumed per query tile
+            uint32_t o_cnt[2] = {0u, 0u};  // items whose O was handed to the epilogue
+            int items = 0;
+            bool ok = true;
+            auto issue_s = [&](int t, uint32_t slot) {
+                const uint32_t sQ = base + L::OFF_Q + t * L::Q_TILE;
+                const uint32_t sK = base + L::OFF_K + static_cast<uint32_t>(slot % KS) * L::KV_TILE;
 #pragma unroll
-                for (int kk = 0; kk < BN / 16; ++kk) {
-                    const uint64_t a = smem_desc_sw128(sP + (kk >> 2) * L::CHUNK + (kk & 3) * 32, 16, 1024);
-                    const uint64_t bd = smem_desc_sw128(sV + kk * 16 * 128, L::CHUNK, 1024);
-                    umma_ss(o_tmem, a, bd, kIdPV, (jj > 0 || kk > 0) ? 1u : 0u);
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * L::CHUNK + (kk & 3) * 32;
+                    umma_ss(tmem + t * BN, smem_desc_sw128(sQ + off, 16, 1024), smem_desc_sw128(sK + off, 16, 1024),
+                            kIdS, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(bar(B_PVDONE));
-                umma_commit(bar(B_VEMPTY0 + st));
+                umma_commit(bar(B_SFULL0 + t));
+            };
+            auto issue_pv = [&](int t, int jj, uint32_t slot) -> bool {
+                if (!mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag)) return false;
+                ++p_cnt[t];
+                if (jj == 0 && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag))
+                    return false;
+                const int vs = static_cast<int>(slot % VS);
+                if (!mbar_wait(bar(B_VFULL0 + vs), (slot / VS) & 1u, abort_flag)) return false;
+                tc_fence_after();
+                const uint32_t sV = base + L::OFF_V + vs * L::KV_TILE;
+#pragma unroll
+                for (int kk = 0; kk < BN / 16; ++kk)
+                    umma_ts(tmem + L::TM_O + t * D, tmem + t * BN + kk * 8,
+                            smem_desc_sw128(sV + kk * 16 * 128, L::CHUNK, 1024), kIdPV, (jj > 0 || kk > 0) ? 1u : 0u);
                 return true;
             };
-            bool ok = mbar_wait(bar(B_QREADY), 0, abort_flag);
-            if (ok) {
-                tc_fence_after();
-                for (int j = 0; j < n_kv; ++j) {
-                    const int st = j & 1;
-                    const uint32_t ph = static_cast<uint32_t>(j >> 1) & 1u;
-                    if (!mbar_wait(bar(B_KFULL0 + st), ph, abort_flag)) { ok = false; break; }
-                    tc_fence_after();
-                    const uint32_t sK = base + L::OFF_K + st * L::KV_BYTES;
-                    const uint32_t s_tmem = tmem + st * BN;
-#pragma unroll
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * L::CHUNK + (kk & 3) * 32;
-                        umma_ss(s_tmem, smem_desc_sw128(sQ + off, 16, 1024), smem_desc_sw128(sK + off, 16, 1024),
-                                kIdS, kk > 0 ? 1u : 0u);
-                    }
-                    umma_commit(bar(B_SFULL0 + st));
-                    umma_commit(bar(B_KEMPTY0 + st));
-                    if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
+                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+                if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag)) {
+                    ok = false;
+                    break;
                 }
-                if (ok) ok = issue_pv(n_kv - 1);
+                tc_fence_after();
+                uint32_t prev = 0;
+                for (int j = 0; j < it.n_kv && ok; ++j, ++kvc) {
+                    const int ks = static_cast<int>(kvc % KS);
+                    if (!mbar_wait(bar(B_KFULL0 + ks), (kvc / KS) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+#pragma unroll
+                    for (int t = 0; t < 2; ++t) {
+                        if (j >= 1 && j - 1 < it.nkv(t) && !issue_pv(t, j - 1, prev)) {
+                            ok = false;
+                            break;
+                        }
+                        if (j < it.nkv(t)) issue_s(t, kvc);
+                    }
+                    if (!ok) break;
+                    umma_commit(bar(B_KEMPTY0 + ks));
+                    if (j >= 1) umma_commit(bar(B_VEMPTY0 + static_cast<int>(prev % VS)));
+                    prev = kvc;
+                }
+                if (!ok) break;
+                umma_commit(bar(B_QEMPTY));  // every S MMA of the item is issued
+#pragma unroll
+                for (int t = 0; t < 2; ++t)
+                    if (it.n_kv - 1 < it.nkv(t) && !issue_pv(t, it.n_kv - 1, prev)) ok = false;
+                if (!ok) break;
+                umma_commit(bar(B_VEMPTY0 + static_cast<int>(prev % VS)));
+#pragma unroll
+                for (int t = 0; t < 2; ++t)
+                    if (it.rows(t)) {
+                        umma_commit(bar(B_OFULL0 + t));
+                        ++o_cnt[t];
+                    }
+                ++items;
             }
             if (!ok) {
                 *abort_flag = 1;
@@ -239,155 +397,146 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait(bar(B_DRAIN), 0, nullptr);
         }
     } else {
-        // ------------------------------------------------------------ softmax / epilogue warps
-        constexpr int HALF = D / 2;
-        const int t = threadIdx.x;  // query row in the tile == TMEM lane
-        const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-        bool ok = mbar_wait(bar(B_QFULL), 0, abort_flag);
-        ok = __all_sync(0xFFFFFFFFu, ok);
-        if (ok && t < rows_valid) {
-            // RoPE of this query row in place (pairs j, j + D/2), as K1 does for keys.
-            const int pos = H + q0 + t;
-            const float* crow = cos_tab + static_cast<size_t>(pos) * HALF;
-            const float* srow = sin_tab + static_cast<size_t>(pos) * HALF;
-#pragma unroll
-            for (int u = 0; u < HALF / 8; ++u) {
-                const int jlo = 8 * u;
-                uint4* plo = reinterpret_cast<uint4*>(gbase + L::OFF_Q + sw128_offset(t, jlo));
-                uint4* phi = reinterpret_cast<uint4*>(gbase + L::OFF_Q + sw128_offset(t, jlo + HALF));
-                const uint4 xa = *plo, xb = *phi;
-                const float4 c0 = *reinterpret_cast<const float4*>(crow + jlo);
-                const float4 c1 = *reinterpret_cast<const float4*>(crow + jlo + 4);
-                const float4 s0 = *reinterpret_cast<const float4*>(srow + jlo);
-                const float4 s1 = *reinterpret_cast<const float4*>(srow + jlo + 4);
-                const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-                const uint32_t wa[4] = {xa.x, xa.y, xa.z, xa.w};
-                const uint32_t wb[4] = {xb.x, xb.y, xb.z, xb.w};
-                uint32_t ya[4], yb[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    float lo[2], hi[2];
-#pragma unroll
-                    for (int k2 = 0; k2 < 2; ++k2) {
-                        const float a = k2 ? bf_hi(wa[e]) : bf_lo(wa[e]);
-                        const float bb = k2 ? bf_hi(wb[e]) : bf_lo(wb[e]);
-                        const float cc = c[2 * e + k2], ss = s[2 * e + k2];
-                        lo[k2] = __fsub_rn(__fmul_rn(a, cc), __fmul_rn(bb, ss));
-                        hi[k2] = __fadd_rn(__fmul_rn(bb, cc), __fmul_rn(a, ss));
-                    }
-                    ya[e] = pack_bf16(lo[0], lo[1]);
-                    yb[e] = pack_bf16(hi[0], hi[1]);
-                }
-                *plo = make_uint4(ya[0], ya[1], ya[2], ya[3]);
-                *phi = make_uint4(yb[0], yb[1], yb[2], yb[3]);
-            }
-        }
-        fence_proxy_async_smem();
-        mbar_arrive(bar(B_QREADY));
+        // ------------------------------------------------------------ softmax / epilogue warpgroups
+        warpgroup_reg_inc<kRegsHigh>();
+        const int t = warp >> 2;            // query tile of this warpgroup
+        const int row = threadIdx.x & 127;  // row in the tile == TMEM lane
+        const uint32_t lane_base = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const uint32_t s_col = tmem + lane_base + t * BN;
+        const uint32_t o_col = tmem + lane_base + L::TM_O + t * D;
+        uint8_t* qtile = gbase + L::OFF_Q + t * L::Q_TILE;
+        uint32_t s_cnt = 0, o_cnt = 0;
+        int items = 0;
+        bool ok = true;
 
-        const int pos_row = H + q0 + t;  // last key this row may see
-        const int min_pos = H + q0;      // smallest row position of the tile
-        float m_run = -INFINITY;         // running maximum, log2 domain
-        float l_run = 0.f;
-        for (int j = 0; j < n_kv && ok; ++j) {
-            const int st = j & 1;
-            const uint32_t ph = static_cast<uint32_t>(j >> 1) & 1u;
-            ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + st), ph, abort_flag));
-            if (!ok) break;
-            tc_fence_after();
-            uint32_t r[BN / 32][32];
-#pragma unroll
-            for (int c = 0; c < BN / 32; ++c) tmem_ld32(tmem + lane_base + st * BN + 32 * c, r[c]);
-            tmem_wait_ld();
-            const int kb = j * BN;
-            float mx = -INFINITY;
-            if (kb + BN - 1 > min_pos) {  // the tile crosses the diagonal: mask by index
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        float v = __uint_as_float(r[c][e]);
-                        v = (kb + 32 * c + e > pos_row) ? -INFINITY : v;
-                        r[c][e] = __float_as_uint(v);
-                        mx = fmaxf(mx, v);
-                    }
-            } else {
-#pragma unroll
-                for (int c = 0; c < BN / 32; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(r[c][e]));
-            }
-            // Lazy rescaling: P is taken relative to a reference max m_run that only moves
-            // when the row max exceeds it by more than 2^8 (P <= 256 otherwise, exact in
-            // bf16/fp32 ranges), so O and l are rescaled rarely; the result is unchanged.
-            const float m_cand = fmaxf(m_run, mx * scale_log2);
-            const bool move = m_cand > m_run + 8.f;  // always true on the first tile
-            const float m_new = move ? m_cand : m_run;
-            const float alpha = move ? fast_exp2(m_run - m_new) : 1.f;
-            const float neg_m = -m_new;
-            float rowsum = 0.f;
-            uint8_t* pbuf = gbase + L::OFF_P + st * L::P_BYTES;
-#pragma unroll
-            for (int u8 = 0; u8 < BN / 8; ++u8) {
-                const int c = u8 >> 2;
-                const int e0 = (u8 & 3) * 8;
-                float p[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    p[e] = fast_exp2(fmaf(__uint_as_float(r[c][e0 + e]), scale_log2, neg_m));
-                    rowsum += p[e];
-                }
-                *reinterpret_cast<uint4*>(pbuf + sw128_offset(t, 8 * u8)) =
-                    make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]), pack_bf16(p[4], p[5]),
-                               pack_bf16(p[6], p[7]));
-            }
-            l_run = l_run * alpha + rowsum;
-            if (j >= 1) {
-                // O holds the sum through tile j-1 once PV(j-1) completes; rescale it.
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(j - 1) & 1u, abort_flag));
+        int lin = blockIdx.x;
+        Item it;
+        if (lin < n_items) {
+            it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+            ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
+                              it.rows(t), H + it.q0(t), cos_tab, sin_tab);
+            ++items;
+        }
+        while (lin < n_items && ok) {
+            float m_run = -INFINITY;  // reference max of P (log2 domain)
+            float l_run = 0.f;
+            const int pos_row = H + it.q0(t) + row;  // last key this row may see
+            const int min_pos = H + it.q0(t);        // smallest row position of the tile
+            for (int j = 0; j < it.nkv(t); ++j) {
+                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + t), s_cnt & 1u, abort_flag));
                 if (!ok) break;
+                ++s_cnt;
                 tc_fence_after();
-                if (__any_sync(0xFFFFFFFFu, alpha < 1.f)) {
+                uint32_t r[BN / 32][32];
+#pragma unroll
+                for (int c = 0; c < BN / 32; ++c) tmem_ld32(s_col + 32 * c, r[c]);
+                tmem_wait_ld();
+                const int kb = j * BN;
+                if (kb + BN - 1 > min_pos) {  // the tile crosses the diagonal: mask by index
+#pragma unroll
+                    for (int c = 0; c < BN / 32; ++c)
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            if (kb + 32 * c + e > pos_row) r[c][e] = __float_as_uint(-INFINITY);
+                }
+                // row max: four independent chains, one per 32-column chunk
+                float mxc[BN / 32];
+#pragma unroll
+                for (int c = 0; c < BN / 32; ++c) {
+                    mxc[c] = __uint_as_float(r[c][0]);
+#pragma unroll
+                    for (int e = 1; e < 31; e += 2)
+                        mxc[c] = fmax3(mxc[c], __uint_as_float(r[c][e]), __uint_as_float(r[c][e + 1]));
+                    mxc[c] = fmaxf(mxc[c], __uint_as_float(r[c][31]));
+                }
+                const float mx = fmaxf(fmaxf(mxc[0], mxc[1]), fmaxf(mxc[2], mxc[3]));
+                const float m_cand = fmaxf(m_run, mx * scale_log2);
+                const bool move = m_cand > m_run + 8.f;  // always on the first tile
+                const float m_new = move ? m_cand : m_run;
+                const float alpha = move ? fast_exp2(m_run - m_new) : 1.f;
+                if (j > 0 && __any_sync(0xFFFFFFFFu, move)) {
+                    // O_T holds the sum through tile j-1 (PV_T(j-1) completed before S_T(j)).
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         uint32_t o[32];
-                        const uint32_t ta = tmem + lane_base + 2 * BN + 32 * c;
-                        tmem_ld32(ta, o);
+                        tmem_ld32(o_col + 32 * c, o);
                         tmem_wait_ld();
 #pragma unroll
                         for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        tmem_st32(ta, o);
+                        tmem_st32(o_col + 32 * c, o);
                     }
-                    tmem_wait_st();
                 }
+                // P = 2^(s*scale - m) as bf16 pairs over the first 64 columns of S (keys 2c, 2c+1
+                // in column c), stored a quarter (16 columns) at a time; the scores are all in
+                // registers, so overwriting S is safe.  Row sums in independent accumulators.
+                const float2 sc2 = make_float2(scale_log2, scale_log2);
+                const float2 nm2 = make_float2(-m_new, -m_new);
+                float2 sum2[BN / 32];
+#pragma unroll
+                for (int c = 0; c < BN / 32; ++c) {
+                    uint32_t pw[16];
+                    float2 acc2 = make_float2(0.f, 0.f);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const float2 x =
+                            ffma2(make_float2(__uint_as_float(r[c][2 * i]), __uint_as_float(r[c][2 * i + 1])), sc2, nm2);
+                        const float2 pp = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+                        acc2 = ffma2(pp, make_float2(1.f, 1.f), acc2);
+                        pw[i] = pack_bf16x2(pp.x, pp.y);
+                    }
+                    sum2[c] = acc2;
+                    tmem_st16(s_col + 16 * c, pw);
+                }
+                const float2 sum2a = make_float2(sum2[0].x + sum2[1].x, sum2[0].y + sum2[1].y);
+                const float2 sum2b = make_float2(sum2[2].x + sum2[3].x, sum2[2].y + sum2[3].y);
+                const float2 sum2t = make_float2(sum2a.x + sum2b.x, sum2a.y + sum2b.y);
+                tmem_wait_st();
+                l_run = l_run * alpha + (sum2t.x + sum2t.y);
+                m_run = m_new;
+                tc_fence_before();
+                mbar_arrive(bar(B_PFULL0 + t));
             }
-            m_run = m_new;
-            fence_proxy_async_smem();
-            tc_fence_before();
-            mbar_arrive(bar(B_PFULL0 + st));
+            if (!ok) break;
+            // next item's q rows (its loads overlap this item's last MMAs)
+            const int next = lin + static_cast<int>(gridDim.x);
+            Item nit;
+            if (next < n_items) {
+                nit = decode_item(next, S, H, Hq, G, hq_b, n_pairs);
+                ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
+                                  row, nit.rows(t), H + nit.q0(t), cos_tab, sin_tab);
+                ++items;
+                if (!ok) break;
+            }
+            // epilogue of this item: O_T / l -> bf16 -> out
+            if (it.rows(t)) {
+                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL0 + t), o_cnt & 1u, abort_flag));
+                if (!ok) break;
+                ++o_cnt;
+                tc_fence_after();
+                const float inv_l = 1.f / l_run;
+                uint16_t* orow = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D;
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t o[32];
+                    tmem_ld32(o_col + 32 * c, o);
+                    tmem_wait_ld();
+                    if (row < it.rows(t)) {
+#pragma unroll
+                        for (int v4 = 0; v4 < 4; ++v4) {
+                            const float* f = reinterpret_cast<const float*>(o) + 8 * v4;
+                            *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
+                                pack_bf16x2(f[0] * inv_l, f[1] * inv_l), pack_bf16x2(f[2] * inv_l, f[3] * inv_l),
+                                pack_bf16x2(f[4] * inv_l, f[5] * inv_l), pack_bf16x2(f[6] * inv_l, f[7] * inv_l));
+                        }
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(bar(B_OEMPTY0 + t));
+            }
+            lin = next;
+            it = nit;
         }
-        if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(n_kv - 1) & 1u, abort_flag));
-        if (ok) {
-            tc_fence_after();
-            const float inv_l = 1.f / l_run;
-            uint16_t* orow = out + ((static_cast<size_t>(b) * S + q0 + t) * Hq + h) * D;
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t o[32];
-                tmem_ld32(tmem + lane_base + 2 * BN + 32 * c, o);
-                tmem_wait_ld();
-                if (t < rows_valid) {
-#pragma unroll
-                    for (int v4 = 0; v4 < 4; ++v4) {
-                        const float* f = reinterpret_cast<const float*>(o) + 8 * v4;
-                        *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) =
-                            make_uint4(pack_bf16(f[0] * inv_l, f[1] * inv_l), pack_bf16(f[2] * inv_l, f[3] * inv_l),
-                                       pack_bf16(f[4] * inv_l, f[5] * inv_l), pack_bf16(f[6] * inv_l, f[7] * inv_l));
-                    }
-                }
-            }
-        } else {
+        if (!ok) {
             *abort_flag = 1;
             atomicOr(err, kDevErrTimeout);
         }
@@ -403,30 +552,40 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int D>
 cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                     const float* sin_tab, uint16_t* out, int* err, cudaStream_t st) {
+                     const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st) {
     const int n_qtiles = (chunk + BM - 1) / BM;
+    const int n_pairs = (n_qtiles + 1) / 2;
+    const long n_items = static_cast<long>(n_pairs) * s.n_q_heads * s.batch;
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
-    const dim3 grid(static_cast<unsigned>(n_qtiles) * s.n_q_heads * s.batch);
+    const dim3 grid(static_cast<unsigned>(std::min<long>(n_items, num_sms)));
     flash_fwd_kernel<D><<<grid, kThreads, Layout<D>::ALLOC, st>>>(maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads,
-                                                                   s.n_kv_heads, n_qtiles, scale_log2, cos_tab,
+                                                                   s.n_kv_heads, s.batch, n_pairs, scale_log2, cos_tab,
                                                                    sin_tab, out, err);
     return cudaGetLastError();
+}
+
+// The register split of the warpgroups is only safe when the kernel is launched
+// with exactly kLaunchRegs registers per thread: check before any launch.
+template <int D>
+cudaError_t configure_d() {
+    cudaFuncAttributes attr;
+    cudaError_t e = cudaFuncGetAttributes(&attr, flash_fwd_kernel<D>);
+    if (e != cudaSuccess) return e;
+    if (attr.numRegs != kLaunchRegs || attr.maxThreadsPerBlock < kThreads) return cudaErrorInvalidConfiguration;
+    return cudaFuncSetAttribute(flash_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Layout<D>::ALLOC);
 }
 
 }  // namespace
 
 cudaError_t configure_flash_fwd() {
-    cudaError_t e = cudaFuncSetAttribute(flash_fwd_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Layout<128>::ALLOC);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(flash_fwd_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                Layout<64>::ALLOC);
+    const cudaError_t e = configure_d<128>();
+    return e != cudaSuccess ? e : configure_d<64>();
 }
 
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                             const float* sin_tab, uint16_t* out, int* err, int /*num_sms*/, cudaStream_t st) {
-    if (s.head_dim == 128) return launch_d<128>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, st);
-    return launch_d<64>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, st);
+                             const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st) {
+    if (s.head_dim == 128) return launch_d<128>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, num_sms, st);
+    return launch_d<64>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, num_sms, st);
 }
 
 }  // namespace attn
