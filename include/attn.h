@@ -37,6 +37,7 @@
  * Ownership.  The caller owns every device buffer passed to a call.  The
  * context owns only its own device memory: the RoPE tables (2 x max_len x
  * head_dim/2 floats), the decode split-KV partials (batch x n_q_heads x 256 x
+ * (head_dim + 2) floats), the prefill partials of split work (SM count x 256 x
  * (head_dim + 2) floats) and a device error word; all allocated by attn_create
  * and freed by attn_destroy.  No stage call allocates, frees or synchronises: each one only
  * enqueues kernels on `stream` and returns.  Calls that use the same context
@@ -141,6 +142,8 @@ int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
  *   ATTN_KERNEL_FLASH_FWD       causal flash attention (prefill, prefill_kv)
  *   ATTN_KERNEL_DECODE_SPLIT    split-KV decode partials (decode)
  *   ATTN_KERNEL_DECODE_COMBINE  log-sum-exp combine of the partials (decode)
+ * (ATTN_KERNEL_FLASH_FWD also covers the small merge kernel that follows it when
+ * the last round of its work is split across CTAs; both count as launches.)
  * attn_timing_enable(ctx, n) creates n pairs of CUDA events (blocking, the only
  * allocation it makes) and from then on every stage call records one pair
  * around each kernel it enqueues, on the call's stream; n = 0 disables timing

@@ -32,6 +32,8 @@ struct attn_ctx {
     float* d_sin;
     float* d_part_o;
     float* d_part_ml;
+    float* d_flash_o;   // flash tail pieces: [num_sms * 256, D] partial O
+    float* d_flash_ml;  // and [num_sms * 256, 2] (m, l)
     int* d_err;
     PFN_cuTensorMapEncodeTiled_v12000 encode;
     // decode tensor maps of the last cache pair seen
@@ -68,6 +70,7 @@ bool cfg_valid(const attn_cfg* c) {
 }
 
 // Enqueue one kernel through `launch`, bracketed by a timing event pair when enabled.
+// `launch` returns the CUDA status and may report how many kernels it enqueued.
 template <typename F>
 cudaError_t timed(attn_ctx* c, int kind, cudaStream_t st, F&& launch) {
     const bool rec = !c->ev_kind.empty() && c->ev_used < static_cast<int>(c->ev_kind.size());
@@ -75,9 +78,10 @@ cudaError_t timed(attn_ctx* c, int kind, cudaStream_t st, F&& launch) {
         const cudaError_t e = cudaEventRecord(c->ev[2 * c->ev_used], st);
         if (e != cudaSuccess) return e;
     }
-    const cudaError_t e = launch();
+    int n = 1;
+    const cudaError_t e = launch(&n);
     if (e != cudaSuccess) return e;
-    ++c->launches[kind];
+    c->launches[kind] += n;
     if (rec) {
         const cudaError_t e2 = cudaEventRecord(c->ev[2 * c->ev_used + 1], st);
         if (e2 != cudaSuccess) return e2;
@@ -135,12 +139,13 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         if (rc == ATTN_OK) rc = encode_map(c, &maps.v, vc, 3, dims, strides, box);
         if (rc != ATTN_OK) return rc;
     }
-    cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&] {
+    cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&](int*) {
         return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, c->d_cos, c->d_sin, kc, vc, c->d_err, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
-    e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&] {
-        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_err, c->num_sms, st);
+    e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&](int* n) {
+        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_flash_o, c->d_flash_ml,
+                                      c->d_err, c->num_sms, st, n);
     });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
     return ATTN_OK;
@@ -203,6 +208,9 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     oom |= cudaMalloc(&c->d_sin, ntab * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_part_o, part_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_part_ml, part_rows * 2 * sizeof(float)) != cudaSuccess;
+    const size_t piece_rows = static_cast<size_t>(c->num_sms) * 256;
+    oom |= cudaMalloc(&c->d_flash_o, piece_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_flash_ml, piece_rows * 2 * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_err, sizeof(int)) != cudaSuccess;
     if (oom) {
         cudaGetLastError();
@@ -229,6 +237,8 @@ void attn_destroy(attn_ctx* c) {
     cudaFree(c->d_sin);
     cudaFree(c->d_part_o);
     cudaFree(c->d_part_ml);
+    cudaFree(c->d_flash_o);
+    cudaFree(c->d_flash_ml);
     cudaFree(c->d_err);
     delete c;
 }
@@ -263,12 +273,12 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         c->dec_v = v_cache;
     }
     const int nsplit = attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
-    cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&] {
+    cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
-    e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&] {
+    e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&](int*) {
         return attn::launch_decode_combine(c->shape, d_hist_len, c->d_part_o, c->d_part_ml, nsplit, out, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_combine launch");

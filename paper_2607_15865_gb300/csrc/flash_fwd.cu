@@ -131,6 +131,35 @@ __device__ __forceinline__ Item decode_item(int lin, int S, int H, int Hq, int G
     return it;
 }
 
+// A work unit: a whole item, or one KV-range piece of an item from the tail of the
+// list.  Items fill whole rounds of CTAs first (`head` of them); the remaining
+// items are cut into `nsplit` pieces each, so every CTA ends at about the same
+// time.  Pieces write unnormalised partial results that a second kernel merges.
+struct Unit {
+    Item it;
+    int kv_lo, kv_hi;  // KV tiles [kv_lo, kv_hi) of the item
+    int piece;         // index of the piece in the partial workspace, -1 for a whole item
+    __device__ __forceinline__ int cnt(int t) const { return max(0, min(kv_hi, it.nkv(t)) - kv_lo); }
+};
+
+__device__ __forceinline__ Unit decode_unit(int lin, int S, int H, int Hq, int G, int hq_b, int n_pairs, int head,
+                                            int nsplit) {
+    Unit u;
+    int item = lin, s = 0, ns = 1;
+    u.piece = -1;
+    if (lin >= head) {
+        const int v = lin - head;
+        item = head + v / nsplit;
+        s = v % nsplit;
+        ns = nsplit;
+        if (nsplit > 1) u.piece = v;
+    }
+    u.it = decode_item(item, S, H, Hq, G, hq_b, n_pairs);
+    u.kv_lo = (u.it.n_kv * s) / ns;
+    u.kv_hi = (u.it.n_kv * (s + 1)) / ns;
+    return u;
+}
+
 // RoPE of one q row of a tile in shared memory (pairs j, j + D/2, table row of its
 // position, float arithmetic with each product and the difference/sum rounded
 // separately, bf16 result), as K1 applies to keys.
@@ -190,8 +219,9 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                      const __grid_constant__ CUtensorMap map_v, int S, int H, int Hq, int Hkv, int batch,
-                     int n_pairs, float scale_log2, const float* __restrict__ cos_tab,
-                     const float* __restrict__ sin_tab, uint16_t* __restrict__ out, int* __restrict__ err) {
+                     int n_pairs, int head, int nsplit, float scale_log2, const float* __restrict__ cos_tab,
+                     const float* __restrict__ sin_tab, uint16_t* __restrict__ out, float* __restrict__ ws_o,
+                     float* __restrict__ ws_ml, int* __restrict__ err) {
     using L = Layout<D>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -206,6 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int G = Hq / Hkv;
     const int hq_b = Hq * batch;
     const int n_items = n_pairs * hq_b;
+    const int n_units = head + (n_items - head) * nsplit;
 
     if (threadIdx.x == 0) {
         *abort_flag = 0;
@@ -247,8 +278,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t kc = 0;  // K tiles issued
             int items = 0;
             bool ok = true;
-            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
-                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+            for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
+                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Item& it = un.it;
                 if (items > 0 && !mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
                     ok = false;
                     break;
@@ -262,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     it.b, bar(B_QFULL));
                 ++items;
                 const int kv_row = it.b * Hkv + it.g;
-                for (int j = 0; j < it.n_kv; ++j, ++kc) {
+                for (int j = un.kv_lo; j < un.kv_hi; ++j, ++kc) {
                     const int st = static_cast<int>(kc % KS);
                     if (kc >= KS && !mbar_wait(bar(B_KEMPTY0 + st), (kc / KS - 1u) & 1u, abort_flag)) {
                         ok = false;
@@ -288,10 +320,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_prefetch_desc(&map_v);
             uint32_t vc = 0;  // V tiles issued
             bool ok = true;
-            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
-                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
-                const int kv_row = it.b * Hkv + it.g;
-                for (int j = 0; j < it.n_kv; ++j, ++vc) {
+            for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
+                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const int kv_row = un.it.b * Hkv + un.it.g;
+                for (int j = un.kv_lo; j < un.kv_hi; ++j, ++vc) {
                     const int st = static_cast<int>(vc % VS);
                     if (vc >= VS && !mbar_wait(bar(B_VEMPTY0 + st), (vc / VS - 1u) & 1u, abort_flag)) {
                         ok = false;
@@ -330,10 +362,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 umma_commit(bar(B_SFULL0 + t));
             };
-            auto issue_pv = [&](int t, int jj, uint32_t slot) -> bool {
+            auto issue_pv = [&](int t, bool first, uint32_t slot) -> bool {
                 if (!mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag)) return false;
                 ++p_cnt[t];
-                if (jj == 0 && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag))
+                if (first && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag))
                     return false;
                 const int vs = static_cast<int>(slot % VS);
                 if (!mbar_wait(bar(B_VFULL0 + vs), (slot / VS) & 1u, abort_flag)) return false;
@@ -342,18 +374,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk)
                     umma_ts(tmem + L::TM_O + t * D, tmem + t * BN + kk * 8,
-                            smem_desc_sw128(sV + kk * 16 * 128, L::CHUNK, 1024), kIdPV, (jj > 0 || kk > 0) ? 1u : 0u);
+                            smem_desc_sw128(sV + kk * 16 * 128, L::CHUNK, 1024), kIdPV, (!first || kk > 0) ? 1u : 0u);
                 return true;
             };
-            for (int lin = blockIdx.x; lin < n_items && ok; lin += gridDim.x) {
-                const Item it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+            for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
+                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Item& it = un.it;
                 if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 uint32_t prev = 0;
-                for (int j = 0; j < it.n_kv && ok; ++j, ++kvc) {
+                for (int j = un.kv_lo; j < un.kv_hi && ok; ++j, ++kvc) {
                     const int ks = static_cast<int>(kvc % KS);
                     if (!mbar_wait(bar(B_KFULL0 + ks), (kvc / KS) & 1u, abort_flag)) {
                         ok = false;
@@ -362,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_after();
 #pragma unroll
                     for (int t = 0; t < 2; ++t) {
-                        if (j >= 1 && j - 1 < it.nkv(t) && !issue_pv(t, j - 1, prev)) {
+                        if (j > un.kv_lo && j - 1 < it.nkv(t) && !issue_pv(t, j - 1 == un.kv_lo, prev)) {
                             ok = false;
                             break;
                         }
@@ -370,19 +403,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     if (!ok) break;
                     umma_commit(bar(B_KEMPTY0 + ks));
-                    if (j >= 1) umma_commit(bar(B_VEMPTY0 + static_cast<int>(prev % VS)));
+                    if (j > un.kv_lo) umma_commit(bar(B_VEMPTY0 + static_cast<int>(prev % VS)));
                     prev = kvc;
                 }
                 if (!ok) break;
-                umma_commit(bar(B_QEMPTY));  // every S MMA of the item is issued
+                umma_commit(bar(B_QEMPTY));  // every S MMA of the unit is issued
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
-                    if (it.n_kv - 1 < it.nkv(t) && !issue_pv(t, it.n_kv - 1, prev)) ok = false;
+                    if (un.kv_hi - 1 < it.nkv(t) && !issue_pv(t, un.kv_hi - 1 == un.kv_lo, prev)) ok = false;
                 if (!ok) break;
                 umma_commit(bar(B_VEMPTY0 + static_cast<int>(prev % VS)));
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
-                    if (it.rows(t)) {
+                    if (un.cnt(t) > 0) {
                         umma_commit(bar(B_OFULL0 + t));
                         ++o_cnt[t];
                     }
@@ -410,19 +443,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
 
         int lin = blockIdx.x;
-        Item it;
-        if (lin < n_items) {
-            it = decode_item(lin, S, H, Hq, G, hq_b, n_pairs);
+        Unit un;
+        if (lin < n_units) {
+            un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
             ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
-                              it.rows(t), H + it.q0(t), cos_tab, sin_tab);
+                              un.it.rows(t), H + un.it.q0(t), cos_tab, sin_tab);
             ++items;
         }
-        while (lin < n_items && ok) {
+        while (lin < n_units && ok) {
+            const Item& it = un.it;
             float m_run = -INFINITY;  // reference max of P (log2 domain)
             float l_run = 0.f;
             const int pos_row = H + it.q0(t) + row;  // last key this row may see
             const int min_pos = H + it.q0(t);        // smallest row position of the tile
-            for (int j = 0; j < it.nkv(t); ++j) {
+            const int n_tiles = un.cnt(t);
+            for (int j = un.kv_lo; j < un.kv_lo + n_tiles; ++j) {
                 ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + t), s_cnt & 1u, abort_flag));
                 if (!ok) break;
                 ++s_cnt;
@@ -454,7 +489,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool move = m_cand > m_run + 8.f;  // always on the first tile
                 const float m_new = move ? m_cand : m_run;
                 const float alpha = move ? fast_exp2(m_run - m_new) : 1.f;
-                if (j > 0 && __any_sync(0xFFFFFFFFu, move)) {
+                if (j > un.kv_lo && __any_sync(0xFFFFFFFFu, move)) {
                     // O_T holds the sum through tile j-1 (PV_T(j-1) completed before S_T(j)).
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
@@ -469,8 +504,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // P = 2^(s*scale - m) as bf16 pairs over the first 64 columns of S (keys 2c, 2c+1
                 // in column c), stored a quarter (16 columns) at a time; the scores are all in
                 // registers, so overwriting S is safe.  Row sums in independent accumulators.
+                // A row of a piece may have seen no visible key yet (all masked): keep its
+                // reference finite so that P, O and l stay 0 (the merge skips l = 0).
+                const float m_ref = m_new == -INFINITY ? 0.f : m_new;
                 const float2 sc2 = make_float2(scale_log2, scale_log2);
-                const float2 nm2 = make_float2(-m_new, -m_new);
+                const float2 nm2 = make_float2(-m_ref, -m_ref);
                 float2 sum2[BN / 32];
 #pragma unroll
                 for (int c = 0; c < BN / 32; ++c) {
@@ -497,44 +535,61 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(bar(B_PFULL0 + t));
             }
             if (!ok) break;
-            // next item's q rows (its loads overlap this item's last MMAs)
+            // next unit's q rows (its loads overlap this unit's last MMAs)
             const int next = lin + static_cast<int>(gridDim.x);
-            Item nit;
-            if (next < n_items) {
-                nit = decode_item(next, S, H, Hq, G, hq_b, n_pairs);
+            Unit nun;
+            if (next < n_units) {
+                nun = decode_unit(next, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
-                                  row, nit.rows(t), H + nit.q0(t), cos_tab, sin_tab);
+                                  row, nun.it.rows(t), H + nun.it.q0(t), cos_tab, sin_tab);
                 ++items;
                 if (!ok) break;
             }
-            // epilogue of this item: O_T / l -> bf16 -> out
-            if (it.rows(t)) {
+            // epilogue: O_T / l -> bf16 -> out, or for a piece the unnormalised O_T and (m, l)
+            const size_t prow = (static_cast<size_t>(un.piece) * 2 * BM + t * BM + row);
+            if (n_tiles > 0) {
                 ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL0 + t), o_cnt & 1u, abort_flag));
                 if (!ok) break;
                 ++o_cnt;
                 tc_fence_after();
-                const float inv_l = 1.f / l_run;
+                const float inv_l = un.piece < 0 ? 1.f / l_run : 1.f;
                 uint16_t* orow = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D;
+                float* prow_o = ws_o + prow * D;
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t o[32];
                     tmem_ld32(o_col + 32 * c, o);
                     tmem_wait_ld();
                     if (row < it.rows(t)) {
+                        const float* f = reinterpret_cast<const float*>(o);
+                        if (un.piece < 0) {
 #pragma unroll
-                        for (int v4 = 0; v4 < 4; ++v4) {
-                            const float* f = reinterpret_cast<const float*>(o) + 8 * v4;
-                            *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
-                                pack_bf16x2(f[0] * inv_l, f[1] * inv_l), pack_bf16x2(f[2] * inv_l, f[3] * inv_l),
-                                pack_bf16x2(f[4] * inv_l, f[5] * inv_l), pack_bf16x2(f[6] * inv_l, f[7] * inv_l));
+                            for (int v4 = 0; v4 < 4; ++v4)
+                                *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
+                                    pack_bf16x2(f[8 * v4 + 0] * inv_l, f[8 * v4 + 1] * inv_l),
+                                    pack_bf16x2(f[8 * v4 + 2] * inv_l, f[8 * v4 + 3] * inv_l),
+                                    pack_bf16x2(f[8 * v4 + 4] * inv_l, f[8 * v4 + 5] * inv_l),
+                                    pack_bf16x2(f[8 * v4 + 6] * inv_l, f[8 * v4 + 7] * inv_l));
+                        } else {
+#pragma unroll
+                            for (int v4 = 0; v4 < 8; ++v4)
+                                *reinterpret_cast<float4*>(prow_o + 32 * c + 4 * v4) =
+                                    make_float4(f[4 * v4], f[4 * v4 + 1], f[4 * v4 + 2], f[4 * v4 + 3]);
                         }
                     }
                 }
+                if (un.piece >= 0 && row < it.rows(t)) {
+                    ws_ml[prow * 2 + 0] = m_run;
+                    ws_ml[prow * 2 + 1] = l_run;
+                }
                 tc_fence_before();
                 mbar_arrive(bar(B_OEMPTY0 + t));
+            } else if (un.piece >= 0 && row < it.rows(t)) {  // this piece holds no key of tile t
+                ws_ml[prow * 2 + 0] = -INFINITY;
+                ws_ml[prow * 2 + 1] = 0.f;
             }
             lin = next;
-            it = nit;
+            un = nun;
         }
         if (!ok) {
             *abort_flag = 1;
@@ -550,18 +605,110 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// Merges the pieces of each tail item: for every row, m* = max m_s over pieces with
+// l_s > 0, out = sum_s 2^(m_s - m*) O_s / sum_s 2^(m_s - m*) l_s -> bf16.
+// Block (tail item, query tile, group of 8 rows); one warp per row.
+template <int D>
+__global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restrict__ ws_o,
+                                                            const float* __restrict__ ws_ml, int S, int H, int Hq,
+                                                            int G, int hq_b, int n_pairs, int head, int nsplit,
+                                                            uint16_t* __restrict__ out) {
+    constexpr int PER_LANE = D / 32;
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // the pieces are complete and visible
+    const int item = head + static_cast<int>(blockIdx.x) / 2;
+    const int t = static_cast<int>(blockIdx.x) % 2;
+    const Item it = decode_item(item, S, H, Hq, G, hq_b, n_pairs);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int row = static_cast<int>(blockIdx.y) * 8 + warp;
+    if (row < it.rows(t)) {
+        const size_t v0 = static_cast<size_t>(item - head) * nsplit;
+        float m = -INFINITY, l = 0.f;
+        if (lane < nsplit) {
+            const size_t prow = (v0 + lane) * 2 * BM + t * BM + row;
+            m = ws_ml[prow * 2 + 0];
+            l = ws_ml[prow * 2 + 1];
+        }
+        float mm = l > 0.f ? m : -INFINITY;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xFFFFFFFFu, mm, off));
+        const float w = l > 0.f ? fast_exp2(m - mm) : 0.f;
+        float lw = l * w;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) lw += __shfl_xor_sync(0xFFFFFFFFu, lw, off);
+        float acc[PER_LANE];
+#pragma unroll
+        for (int e = 0; e < PER_LANE; ++e) acc[e] = 0.f;
+        for (int sp = 0; sp < nsplit; ++sp) {
+            const float ws = __shfl_sync(0xFFFFFFFFu, w, sp);
+            if (ws == 0.f) continue;  // a piece without keys of this tile: its O was never written
+            const float* src = ws_o + ((v0 + sp) * 2 * BM + t * BM + row) * D + lane * PER_LANE;
+#pragma unroll
+            for (int e = 0; e < PER_LANE; ++e) acc[e] = fmaf(ws, src[e], acc[e]);
+        }
+        const float inv = 1.f / lw;
+        uint16_t* dst = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D + lane * PER_LANE;
+#pragma unroll
+        for (int e = 0; e < PER_LANE; e += 2)
+            *reinterpret_cast<uint32_t*>(dst + e) = pack_bf16x2(acc[e] * inv, acc[e + 1] * inv);
+    }
+}
+
+// Host schedule: `head` items fill whole rounds of the persistent CTAs; the tail
+// items are cut into nsplit KV pieces (at most one piece per CTA, at most 16 per
+// item, never more than the shortest tail item has KV tiles).
+struct Schedule {
+    int n_pairs, n_items, head, nsplit, n_units, grid;
+};
+
+Schedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
+    Schedule sc;
+    const int n_qtiles = (chunk + BM - 1) / BM;
+    sc.n_pairs = (n_qtiles + 1) / 2;
+    sc.n_items = sc.n_pairs * s.n_q_heads * s.batch;
+    sc.head = (sc.n_items / num_sms) * num_sms;
+    const int tail = sc.n_items - sc.head;
+    sc.nsplit = 1;
+    if (tail > 0) {
+        const int nkv_min = (hist + std::min(2 * BM, chunk) + BN - 1) / BN;  // pair 0 is the shortest
+        long nkv_sum = 0;
+        for (int pt = 0; pt < sc.n_pairs; ++pt) nkv_sum += (hist + std::min(2 * BM * (pt + 1), chunk) + BN - 1) / BN;
+        // Split when there are fewer items than CTAs, or when the tail items are long
+        // enough for the last round to matter (not for the short tail of a causal prefill).
+        if (sc.head == 0 || 2L * nkv_min * sc.n_pairs >= nkv_sum)
+            sc.nsplit = std::max(1, std::min({num_sms / tail, 16, nkv_min}));
+    }
+    if (sc.nsplit == 1) sc.head = sc.n_items;
+    sc.n_units = sc.head + (sc.n_items - sc.head) * sc.nsplit;
+    sc.grid = std::min(sc.n_units, num_sms);
+    return sc;
+}
+
 template <int D>
 cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                     const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st) {
-    const int n_qtiles = (chunk + BM - 1) / BM;
-    const int n_pairs = (n_qtiles + 1) / 2;
-    const long n_items = static_cast<long>(n_pairs) * s.n_q_heads * s.batch;
+                     const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+                     cudaStream_t st, int* n_launched) {
+    const Schedule sc = make_schedule(s, hist, chunk, num_sms);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
-    const dim3 grid(static_cast<unsigned>(std::min<long>(n_items, num_sms)));
-    flash_fwd_kernel<D><<<grid, kThreads, Layout<D>::ALLOC, st>>>(maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads,
-                                                                   s.n_kv_heads, s.batch, n_pairs, scale_log2, cos_tab,
-                                                                   sin_tab, out, err);
-    return cudaGetLastError();
+    flash_fwd_kernel<D><<<sc.grid, kThreads, Layout<D>::ALLOC, st>>>(
+        maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head, sc.nsplit,
+        scale_log2, cos_tab, sin_tab, out, ws_o, ws_ml, err);
+    cudaError_t e = cudaGetLastError();
+    *n_launched = 1;
+    if (e != cudaSuccess || sc.nsplit == 1) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(2 * (sc.n_items - sc.head)), BM / 8);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const int G = s.n_q_heads / s.n_kv_heads;
+    e = cudaLaunchKernelEx(&cfg, flash_combine_kernel<D>, ws_o, ws_ml, chunk, hist, s.n_q_heads, G,
+                           s.n_q_heads * s.batch, sc.n_pairs, sc.head, sc.nsplit, out);
+    *n_launched = 2;
+    return e;
 }
 
 // The register split of the warpgroups is only safe when the kernel is launched
@@ -583,9 +730,11 @@ cudaError_t configure_flash_fwd() {
 }
 
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                             const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st) {
-    if (s.head_dim == 128) return launch_d<128>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, num_sms, st);
-    return launch_d<64>(s, maps, hist, chunk, cos_tab, sin_tab, out, err, num_sms, st);
+                             const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+                             cudaStream_t st, int* n_launched) {
+    if (s.head_dim == 128)
+        return launch_d<128>(s, maps, hist, chunk, cos_tab, sin_tab, out, ws_o, ws_ml, err, num_sms, st, n_launched);
+    return launch_d<64>(s, maps, hist, chunk, cos_tab, sin_tab, out, ws_o, ws_ml, err, num_sms, st, n_launched);
 }
 
 }  // namespace attn

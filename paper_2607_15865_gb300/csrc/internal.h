@@ -33,8 +33,12 @@ struct FlashMaps {
 };
 // Raise the dynamic shared-memory limit of K2 on the current device (once per device).
 cudaError_t configure_flash_fwd();
+// Work is split across num_sms persistent CTAs; items of the last, partial round are
+// cut into KV pieces whose partials go to ws_o [num_sms*256, D] / ws_ml [num_sms*256, 2]
+// and are merged by a second kernel (then *n_launched = 2).
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                             const float* sin_tab, uint16_t* out, int* err, int num_sms, cudaStream_t st);
+                             const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+                             cudaStream_t st, int* n_launched);
 
 // K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
 // with 64-key boxes (built once per cache pair).  K3 also rotates the new key and
