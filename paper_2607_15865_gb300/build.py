@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libattn_gb300.so")
-SOURCES = ["attn_api.cu", "rope_append.cu", "decode.cu", "flash_fwd.cu", "decode_noalloc.cu"]
+SOURCES = ["attn_api.cu", "rope_append.cu", "decode.cu", "decode_tc.cu", "flash_fwd.cu", "decode_noalloc.cu"]
 HEADERS = ["internal.h", "sm100_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -13,6 +13,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -185,6 +186,7 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     c->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     e = attn::configure_flash_fwd();
     if (e == cudaSuccess) e = attn::configure_decode();
+    if (e == cudaSuccess) e = attn::configure_decode_tc();
     if (e != cudaSuccess) {
         delete c;
         return cuda_fail(e, "configure kernels");
@@ -263,8 +265,11 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         !aligned16(out) || (reinterpret_cast<uintptr_t>(d_hist_len) & 3u))
         return ATTN_EINVAL;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const bool tc = c->cfg.head_dim == 128;  // tensor-core decode; head_dim 64 on the CUDA cores
     if (k_cache != c->dec_k || v_cache != c->dec_v) {
-        if (attn::make_decode_maps(c->encode, c->shape, k_cache, v_cache, &c->dec_maps) != cudaSuccess) {
+        const cudaError_t me = tc ? attn::make_decode_tc_maps(c->encode, c->shape, k_cache, v_cache, &c->dec_maps)
+                                  : attn::make_decode_maps(c->encode, c->shape, k_cache, v_cache, &c->dec_maps);
+        if (me != cudaSuccess) {
             c->dec_k = c->dec_v = nullptr;
             std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "cuTensorMapEncodeTiled failed for the decode caches");
             return ATTN_ECUDA;
@@ -272,8 +277,12 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         c->dec_k = k_cache;
         c->dec_v = v_cache;
     }
-    const int nsplit = attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
+    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms), c->nsplit_max)
+                          : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
+        if (tc)
+            return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
+                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });

@@ -59,7 +59,7 @@ int setup_device(int dev, float** scratch, int* num_sms) {
         if (major != 10 || minor != 3) return ATTN_EARCH;
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ATTN_ECUDA;
-        if (attn::configure_decode() != cudaSuccess) return ATTN_ECUDA;
+        if (attn::configure_decode() != cudaSuccess || attn::configure_decode_tc() != cudaSuccess) return ATTN_ECUDA;
         g_num_sms[dev] = sms;
         g_scratch_ptr[dev] = static_cast<float*>(p);
     }
@@ -101,15 +101,22 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     // Same split rule as attn_decode, capped by what the scratch array holds.
     const attn::Shape s{cfg->batch, cfg->n_q_heads, cfg->n_kv_heads, cfg->head_dim, cfg->max_len};
     const long long fit = ATTN_NOALLOC_SCRATCH_FLOATS / per_split;
-    const int nsplit = attn::decode_num_splits(s, num_sms, static_cast<int>(fit < 256 ? fit : 256));
+    const int cap = static_cast<int>(fit < 256 ? fit : 256);
+    const bool tc = cfg->head_dim == 128;
+    int nsplit = tc ? attn::decode_tc_num_splits(s, num_sms) : attn::decode_num_splits(s, num_sms, cap);
+    nsplit = nsplit < cap ? nsplit : cap;
     float* part_o = scratch;
     float* part_ml = scratch + static_cast<size_t>(cfg->batch) * cfg->n_q_heads * nsplit * cfg->head_dim;
 
     attn::DecodeMaps maps;
-    if (attn::make_decode_maps(g_encode, s, k_cache, v_cache, &maps) != cudaSuccess) return ATTN_ECUDA;
+    const cudaError_t me = tc ? attn::make_decode_tc_maps(g_encode, s, k_cache, v_cache, &maps)
+                              : attn::make_decode_maps(g_encode, s, k_cache, v_cache, &maps);
+    if (me != cudaSuccess) return ATTN_ECUDA;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = attn::launch_decode_split(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o,
-                                              part_ml, nsplit, d_err, st);
+    cudaError_t e = tc ? attn::launch_decode_tc(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o,
+                                                part_ml, nsplit, d_err, st)
+                       : attn::launch_decode_split(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin,
+                                                   part_o, part_ml, nsplit, d_err, st);
     if (e == cudaSuccess) e = attn::launch_decode_combine(s, d_hist_len, part_o, part_ml, nsplit, out, st);
     return e == cudaSuccess ? ATTN_OK : ATTN_ECUDA;
 }
