@@ -396,6 +396,100 @@ def run_ours(args):
     return 0
 
 
+# ----------------------------------------------------------------------------- per-config sweep
+
+
+def run_sweep(args):
+    """Times every configuration's stage on one GPU (CUDA events around the stage call,
+    inputs resident, L2 flushed before each timed call) and writes a table to
+    --sweep-out; the default JSON line is not printed in this mode."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.attention import Attention
+    from synthetic.workloads import Shape
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    peaks, kind = load_peaks()
+    tc_peak, hbm = float(peaks["bf16_tflops"]), float(peaks["hbm_gbs"])
+
+    def rnd(shape, gen):
+        return (torch.randn(*shape, device=dev, generator=gen) * 0.0884).to(torch.bfloat16)
+
+    def time_calls(fn, reps):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for _ in range(3):
+            flush.zero_()
+            fn()
+        for a, b in evs:
+            flush.zero_()
+            a.record()
+            fn()
+            b.record()
+        torch.cuda.synchronize()
+        return sorted(a.elapsed_time(b) for a, b in evs)[reps // 2]  # median, ms
+
+    rows = []
+    gen = torch.Generator(device=dev).manual_seed(1)
+    cases = [("7B prefill 512", w.PREFILL_7B, 0, 512),
+             ("prefill_kv 512 over 1536", w.PREFILL_KV, 1536, 512),
+             ("long prefill 4096", S, 0, w.LONG_PREFILL),
+             ("long prefill_kv 4096 over 28672", S, w.LONG_PKV_HIST, w.LONG_PKV_CHUNK)]
+    for name, sh, hist, chunk in cases:
+        attn = Attention.for_shape(sh)
+        q = rnd((sh.batch, chunk, sh.n_q_heads, sh.head_dim), gen)
+        k = rnd((sh.batch, chunk, sh.n_kv_heads, sh.head_dim), gen)
+        v = rnd((sh.batch, chunk, sh.n_kv_heads, sh.head_dim), gen)
+        kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        out = torch.empty_like(q)
+        ms = time_calls(lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out), args.sweep_reps)
+        tf = attn_flops(sh, prefill_pairs(hist, chunk)) / (ms * 1e-3) / 1e12
+        rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
+        attn.close()
+    for bsz in w.DECODE_BATCHES:
+        sh = w.decode_shape(bsz)
+        attn = Attention.for_shape(sh)
+        nbuf = max(2, int(2 * 130e6 // (sh.batch * sh.n_kv_heads * sh.max_len * sh.head_dim * 4)) + 1)
+        caches = [(rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen),
+                   rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)) for _ in range(min(nbuf, 8))]
+        q = rnd((sh.batch, 1, sh.n_q_heads, sh.head_dim), gen)
+        k = rnd((sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+        v = rnd((sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+        out = torch.empty_like(q)
+        for hist in w.DECODE_HISTS:
+            hl = torch.full((sh.batch,), hist, dtype=torch.int32, device=dev)
+            it = [0]
+
+            def call():
+                kc, vc = caches[it[0] % len(caches)]
+                it[0] += 1
+                attn.decode(q, k, v, hl, kc, vc, out)
+            ms = time_calls(call, args.sweep_reps)
+            gbs = decode_bytes(sh, hist) / (ms * 1e-3) / 1e9
+            rows.append({"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+        attn.close()
+    attn = Attention.for_shape(S)
+    kc = rnd((1, 8, 32768, 128), gen)
+    vc = rnd((1, 8, 32768, 128), gen)
+    q, k, v = rnd((1, 1, 40, 128), gen), rnd((1, 1, 8, 128), gen), rnd((1, 1, 8, 128), gen)
+    out = torch.empty_like(q)
+    hl = torch.full((1,), w.LONG_DECODE_HIST, dtype=torch.int32, device=dev)
+    ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), args.sweep_reps)
+    gbs = DECODE_BYTES / (ms * 1e-3) / 1e9
+    rows.append({"config": "long decode hist 32767", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+    doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
+    with open(args.sweep_out, "w") as f:
+        json.dump(doc, f, indent=1)
+    for r in rows:
+        extra = f"{r['TFLOP/s']:8.1f} TFLOP/s {100*r['frac_tensor']:5.1f}%" if "TFLOP/s" in r else \
+            f"{r['GB/s']:8.1f} GB/s    {100*r['frac_hbm']:5.1f}%"
+        print(f"{r['config']:36s} {r['ms']*1e3:9.1f} us {extra}", file=sys.stderr)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -405,11 +499,16 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=192, help="prefill_kv rows in the oracle's timed sample")
     ap.add_argument("--ref-rows", type=int, default=48, help="prefill_kv rows per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="time every configuration's stage instead (table to --sweep-out)")
+    ap.add_argument("--sweep-out", default="sweep.json")
+    ap.add_argument("--sweep-reps", type=int, default=20)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     return run_ours(args)
 
 
