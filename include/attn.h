@@ -140,8 +140,9 @@ int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
  * Kernel timing (tracing).  The library launches four kernels:
  *   ATTN_KERNEL_ROPE_APPEND     RoPE of the new keys + in-place cache append (every stage)
  *   ATTN_KERNEL_FLASH_FWD       causal flash attention (prefill, prefill_kv)
- *   ATTN_KERNEL_DECODE_SPLIT    split-KV decode partials (decode)
- *   ATTN_KERNEL_DECODE_COMBINE  log-sum-exp combine of the partials (decode)
+ *   ATTN_KERNEL_DECODE_SPLIT    split-KV decode (decode); with head_dim 128 it also
+ *                               merges the splits and writes out itself
+ *   ATTN_KERNEL_DECODE_COMBINE  log-sum-exp merge of the partials (decode, head_dim 64)
  * (ATTN_KERNEL_FLASH_FWD also covers the small merge kernel that follows it when
  * the last round of its work is split across CTAs; both count as launches.)
  * attn_timing_enable(ctx, n) creates n pairs of CUDA events (blocking, the only
@@ -178,11 +179,14 @@ int attn_timing_read(attn_ctx* ctx, double* ms, long long* launches);
  *     back (it receives the ATTN_DEVERR_* bits, as attn_device_error reports);
  *   - the split-KV partials live in a static device array of
  *     ATTN_NOALLOC_SCRATCH_FLOATS floats (4 MiB) that every GPU which loads this
- *     library holds until the process exits.  Shapes whose partials do not fit
- *     even with one split (batch * n_q_heads * (head_dim + 2) > that size) are
- *     rejected with ATTN_EINVAL; larger ones use fewer splits.
- * All calls share that one array and nothing in it has to start at zero (every
- * call rewrites the part it reads).  Calls whose kernels overlap on the GPU --
+ *     library holds until the process exits, beside 32768 int counters
+ *     (128 KiB).  Shapes whose partials do not fit even with one split
+ *     (batch * n_q_heads * (head_dim + 2) > that size) are rejected with
+ *     ATTN_EINVAL; larger ones use fewer splits.
+ * All calls share those arrays.  Nothing in the partials has to start at zero
+ * (every call rewrites the part it reads); the counters are zero when the
+ * library loads and every completed call leaves them zero.  Calls whose kernels
+ * overlap on the GPU --
  * on different streams, or from several threads -- race on it and must be
  * serialised by the caller.  The first call on each device looks up the array's
  * device address (cudaGetSymbolAddress, with that device current) and caches

@@ -33,6 +33,7 @@ struct attn_ctx {
     float* d_sin;
     float* d_part_o;
     float* d_part_ml;
+    int* d_counters;    // decode counters, [2][B * Hkv] (merge count, tile claims), zero between launches
     float* d_flash_o;   // flash tail pieces: [num_sms * 256, D] partial O
     float* d_flash_ml;  // and [num_sms * 256, 2] (m, l)
     int* d_err;
@@ -214,6 +215,8 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     oom |= cudaMalloc(&c->d_flash_o, piece_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_flash_ml, piece_rows * 2 * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_err, sizeof(int)) != cudaSuccess;
+    const size_t n_counters = 2 * static_cast<size_t>(cfg->batch) * cfg->n_kv_heads;  // merge + tile claims
+    oom |= cudaMalloc(&c->d_counters, n_counters * sizeof(int)) != cudaSuccess;
     if (oom) {
         cudaGetLastError();
         attn_destroy(c);
@@ -222,6 +225,7 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     e = cudaMemcpy(c->d_cos, hc.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->d_sin, hs.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(c->d_counters, 0, n_counters * sizeof(int));
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         attn_destroy(c);
@@ -242,6 +246,7 @@ void attn_destroy(attn_ctx* c) {
     cudaFree(c->d_flash_o);
     cudaFree(c->d_flash_ml);
     cudaFree(c->d_err);
+    cudaFree(c->d_counters);
     delete c;
 }
 
@@ -282,11 +287,13 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
-                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
+                                          c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
+                                          c->d_err, st);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
+    if (tc) return ATTN_OK;  // the tensor-core decode merges its splits itself
     e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&](int*) {
         return attn::launch_decode_combine(c->shape, d_hist_len, c->d_part_o, c->d_part_ml, nsplit, out, st);
     });

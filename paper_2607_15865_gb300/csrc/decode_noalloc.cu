@@ -7,11 +7,12 @@
 // front, or in a callback that must not touch the allocator.  Such a caller cannot
 // create an attn_ctx (attn_create allocates the tables and the split-KV partials).
 //
-// This entry point runs the same kernels as attn_decode (K3 decode_split with the
-// new token's append, K4 decode_combine) but needs no context: the caller passes every
-// input and output, including the RoPE tables and the error word, and the split-KV
-// partials live in the file-scope array below, which the library holds on every
-// device that loads it until the process exits.  Nothing is allocated or freed.
+// This entry point runs the same kernels as attn_decode (K3 with the new token's
+// append; for head_dim 64 also K4, which merges the splits) but needs no context: the
+// caller passes every input and output, including the RoPE tables and the error word,
+// and the split-KV partials and merge counters live in the file-scope arrays below,
+// which the library holds on every device that loads it until the process exits.
+// Nothing is allocated or freed.
 //
 // Host code must not pass `g_noalloc_scratch` itself to a kernel: in host code that
 // name denotes a host-side shadow, not device memory.  The device address is looked
@@ -29,17 +30,23 @@ namespace {
 // Split-KV partials of attn_decode_noalloc: [B*Hq*nsplit*D] accumulators followed by
 // [B*Hq*nsplit*2] (max, sum) pairs.  Shared by every call on the device.
 static __device__ __align__(256) float g_noalloc_scratch[ATTN_NOALLOC_SCRATCH_FLOATS];
+// Counters of the tensor-core decode, two per (sequence, kv head) (merge count, tile
+// claims); zero at load and left zero by every launch.  B*Hkv <= B*Hq <=
+// scratch / (D + 2) < 16384.
+constexpr int kNoallocCounters = 16384;
+static __device__ int g_noalloc_counters[2 * kNoallocCounters] = {0};
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
 float* g_scratch_ptr[kMaxDevices] = {};
+int* g_counter_ptr[kMaxDevices] = {};
 int g_num_sms[kMaxDevices] = {};
 attn::PFN_encodeTiled g_encode = nullptr;
 
 // Per-device set-up, on the current device: the device address of the scratch
 // array, the SM count, the kernels' shared-memory limits and (once per process)
 // the driver's tensor-map encoder.  Returns ATTN_OK, ATTN_EARCH or ATTN_ECUDA.
-int setup_device(int dev, float** scratch, int* num_sms) {
+int setup_device(int dev, float** scratch, int** counters, int* num_sms) {
     std::lock_guard<std::mutex> lock(g_setup_mutex);
     if (g_encode == nullptr) {
         cudaDriverEntryPointQueryResult qres;
@@ -59,11 +66,15 @@ int setup_device(int dev, float** scratch, int* num_sms) {
         if (major != 10 || minor != 3) return ATTN_EARCH;
         void* p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ATTN_ECUDA;
+        void* pc = nullptr;
+        if (cudaGetSymbolAddress(&pc, g_noalloc_counters) != cudaSuccess || pc == nullptr) return ATTN_ECUDA;
+        g_counter_ptr[dev] = static_cast<int*>(pc);
         if (attn::configure_decode() != cudaSuccess || attn::configure_decode_tc() != cudaSuccess) return ATTN_ECUDA;
         g_num_sms[dev] = sms;
         g_scratch_ptr[dev] = static_cast<float*>(p);
     }
     *scratch = g_scratch_ptr[dev];
+    *counters = g_counter_ptr[dev];
     *num_sms = g_num_sms[dev];
     return ATTN_OK;
 }
@@ -94,8 +105,9 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ATTN_ECUDA;
     float* scratch = nullptr;
+    int* counters = nullptr;
     int num_sms = 0;
-    const int rc = setup_device(dev, &scratch, &num_sms);
+    const int rc = setup_device(dev, &scratch, &counters, &num_sms);
     if (rc != ATTN_OK) return rc;
 
     // Same split rule as attn_decode, capped by what the scratch array holds.
@@ -113,10 +125,11 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
                               : attn::make_decode_maps(g_encode, s, k_cache, v_cache, &maps);
     if (me != cudaSuccess) return ATTN_ECUDA;
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (tc && static_cast<long long>(cfg->batch) * cfg->n_kv_heads > kNoallocCounters) return ATTN_EINVAL;
     cudaError_t e = tc ? attn::launch_decode_tc(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin, part_o,
-                                                part_ml, nsplit, d_err, st)
+                                                part_ml, counters, nsplit, out, d_err, st)
                        : attn::launch_decode_split(s, maps, q, k, v, d_hist_len, k_cache, v_cache, d_cos, d_sin,
                                                    part_o, part_ml, nsplit, d_err, st);
-    if (e == cudaSuccess) e = attn::launch_decode_combine(s, d_hist_len, part_o, part_ml, nsplit, out, st);
+    if (e == cudaSuccess && !tc) e = attn::launch_decode_combine(s, d_hist_len, part_o, part_ml, nsplit, out, st);
     return e == cudaSuccess ? ATTN_OK : ATTN_ECUDA;
 }

@@ -1,4 +1,5 @@
-// decode_tc.cu -- K3 for head_dim 128: split-KV decode attention on the tensor cores.
+// decode_tc.cu -- K3 for head_dim 128: split-KV decode attention on the tensor cores,
+// with the merge of the splits fused in.
 //
 // Decode (Section 4.4): one new query per sequence b at position p = hist_len[b]
 // attends to cache slots [0, p] of its kv head; its own k/v go to slot p (the
@@ -9,23 +10,31 @@
 // in swapped form so that the 128 keys of a tile fill the MMA's M dimension:
 //   S^T [128 keys x 16] = K_tile [128 x D] . Q^T       (Q: G heads, zero-padded to 16)
 //   O^T [D x 16]      += V_tile^T [D x 128] . P^T [128 x 16]
-// Both accumulate in TMEM.  CTA (split s, kv head g, sequence b) owns keys
-// [s*per, min((s+1)*per, p+1)), per computed on the device from p.  192 threads:
-//   warps 0-3  one thread per key of the tile: scores from TMEM, per-head tile
-//              max (shuffles + one exchange), lazy running max, P^T (bf16) into
-//              shared memory; per-thread partial row sums; the epilogue (one
-//              thread per output dimension d) writes the split's partial
-//              (m, l, acc[D]) per head for K4 to merge;
-//   warp 4     TMA producer: K and V tiles of 128 keys (128-byte swizzle) into a
-//              3-stage ring, 64 KB per stage;
-//   warp 5     tcgen05 issuer (S^T into one of two TMEM buffers, then O^T += ...).
-// The split that owns slot p rotates the new k (RoPE from the table, the same
-// float arithmetic and bf16 rounding as K1), writes k and v to slot p, uses
-// q.k_new computed on the CUDA cores as that key's score and writes v_new over
-// the loaded V row.  V rows past the split's end are zeroed before the PV MMA
-// (the slots past hist_len may hold anything, and 0 * NaN would poison O).
-// Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its
-// copies and MMAs finish, releases TMEM and exits.
+// Both accumulate in TMEM.  The T = ceil((p+1)/128) key tiles of a sequence are dealt
+// to the nsplit CTAs of (b, kv head) in contiguous, balanced runs (split s owns tiles
+// [s*T/nsplit, (s+1)*T/nsplit)), so no CTA loads keys that another one owns.
+// 192 threads:
+//   warps 0-3  one thread per key of the tile: scores from TMEM, masking, P^T (bf16)
+//              into shared memory, per-thread partial row sums.  The running max m
+//              moves lazily: a tile whose scores all stay within 2^8 of m (checked
+//              with one OR-barrier) is exponentiated against m as it is; otherwise
+//              the per-head tile maxima are reduced (a halving butterfly: 16
+//              shuffles for 16 heads) and O^T is rescaled.  Epilogue: one thread
+//              per output dimension d;
+//   warp 4     TMA producer: K and V tiles of 128 keys (128-byte swizzle) into
+//              rings of 2 (K) and 4 (V) stages of 32 KB;
+//   warp 5     tcgen05 issuer; it also owns the new token: it rotates k (RoPE from
+//              the table, the same float arithmetic and bf16 rounding as K1), writes
+//              k and v to slot p of the cache and into the shared-memory copies of
+//              the tile that holds slot p (whose later rows it zeroes in V: slots
+//              past p may hold anything, and 0 * NaN would poison O), so the MMA
+//              itself produces the new key's score.
+// Merge: with one split the CTA writes the normalised output.  Otherwise each CTA
+// writes its partial (m, l, acc[D]) per head; the last CTA of (b, kv head) to finish
+// (a device counter, reset by that CTA) merges them:
+//   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
+// Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its copies
+// and MMAs finish, releases TMEM and still takes part in the merge count.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -55,22 +64,23 @@ enum Bar { B_QREADY, B_KFULL0, B_KFULL1, B_KEMPTY0, B_KEMPTY1, B_VFULL0, B_VFULL
 struct L {
     static constexpr int BOX = KT * 128;           // [128 keys x 64 dims] bf16, 16 KB
     static constexpr int TILE = 2 * BOX;           // one K (or V) tile, 32 KB
-    static constexpr int OFF_K = 0;                // K ring
+    static constexpr int OFF_K = 0;                // K ring (the merge's weights reuse it)
     static constexpr int OFF_V = KST * TILE;       // V ring
     static constexpr int OFF_Q = OFF_V + VST * TILE;  // Q^T [16 heads x 128] bf16, 2 x 2 KB
     static constexpr int OFF_P = OFF_Q + 2 * NH * 128;          // P^T [16 x 128 keys] x 2 buffers
-    static constexpr int OFF_RED = OFF_P + 2 * 2 * NH * 128;    // float red[4 warps][16]
-    static constexpr int OFF_NEWS = OFF_RED + 4 * NH * 4;       // float score of the new key [16]
-    static constexpr int OFF_LS = OFF_NEWS + NH * 4;            // float l partials [4 warps][16]
-    static constexpr int OFF_M = OFF_LS + 4 * NH * 4;           // float m [16]
-    static constexpr int OFF_VNEW = OFF_M + NH * 4;             // bf16 v_new [128]
-    static constexpr int OFF_BAR = OFF_VNEW + D * 2;
+    static constexpr int OFF_RED = OFF_P + 2 * 2 * NH * 128;    // float tile maxima [16 heads][4 warps]
+    static constexpr int OFF_LS = OFF_RED + NH * 4 * 4;         // float l partials [16 heads][4 warps]
+    static constexpr int OFF_META = OFF_LS + NH * 4 * 4;       // int tile index per local tile, ring of 8
+    static constexpr int OFF_BAR = OFF_META + 8 * 4;
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
-    static constexpr int OFF_ABORT = OFF_TMEM + 8;
-    static constexpr int BYTES = OFF_ABORT + 8;
+    static constexpr int OFF_ABORT = OFF_TMEM + 4;
+    static constexpr int OFF_LAST = OFF_ABORT + 4;
+    static constexpr int BYTES = OFF_LAST + 8;
     static constexpr int ALLOC = BYTES + 1024;
 };
 static_assert(L::ALLOC <= 232448, "shared memory of one CTA");
+static_assert(NH * 256 * 8 + NH * 4 + (kThreads / 32) * NH * D * 4 <= KST * L::TILE + VST * L::TILE,
+              "merge buffers fit in the rings");
 
 __device__ __forceinline__ float bf16_at(const uint16_t* p) { return __uint_as_float(static_cast<uint32_t>(*p) << 16); }
 __device__ __forceinline__ uint16_t to_bf16(float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
@@ -82,21 +92,38 @@ __device__ __forceinline__ uint32_t sw_elem(int row, int col, int rows) {
                                  (col & 7) * 2);
 }
 
-__device__ __forceinline__ float rope_elem(const uint16_t* x, int d, const float* cos_row, const float* sin_row) {
-    constexpr int HALF = D / 2;
-    const int j = d % HALF;
-    const float c = cos_row[j], s = sin_row[j];
-    if (d < HALF) return __fsub_rn(__fmul_rn(bf16_at(x + d), c), __fmul_rn(bf16_at(x + d + HALF), s));
-    return __fadd_rn(__fmul_rn(bf16_at(x + d), c), __fmul_rn(bf16_at(x + d - HALF), s));
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&r)[N]) {
+    static_assert(N == 8 || N == 16, "8 or 16 columns");
+    if constexpr (N == 16) {
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+            "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+            : "r"(taddr));
+    } else {
+        asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                     : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                     : "r"(taddr));
+    }
 }
 
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)[N]) {
+    static_assert(N == 8 || N == 16, "8 or 16 columns");
+    if constexpr (N == 16) {
+        asm volatile(
+            "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+            "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+            "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+            "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+            : "memory");
+    } else {
+        asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+                     "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                     : "memory");
+    }
 }
 
 __device__ __forceinline__ void named_sync_128() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -115,12 +142,56 @@ __device__ __forceinline__ bool named_or_128(bool pred) {
     return r != 0;
 }
 
+// Reduction of N values per lane over the 32 lanes of a warp by recursive halving:
+// at each step a lane keeps half of its values, sends the other half to its partner
+// and combines (N - 1 shuffles for N -> 1), then the remaining lane bits reduce
+// plainly.  Returns the reduction of value index halving_owner<N>(lane) over all
+// 32 lanes; v is clobbered.
+template <int N, bool kMax>
+__device__ __forceinline__ float warp_reduce_halving(float (&v)[N], int lane) {
+    static_assert(N == 8 || N == 16, "8 or 16 values");
+#pragma unroll
+    for (int half = N / 2, mask = 16; half >= 1; half >>= 1, mask >>= 1) {
+        const bool upper = (lane & mask) != 0;
+#pragma unroll
+        for (int i = 0; i < half; ++i) {
+            const float keep = upper ? v[i + half] : v[i];
+            const float send = upper ? v[i] : v[i + half];
+            const float got = __shfl_xor_sync(0xFFFFFFFFu, send, mask);
+            v[i] = kMax ? fmaxf(keep, got) : keep + got;
+        }
+    }
+    float r = v[0];
+    constexpr int kRest = (N == 16) ? 1 : 2;  // lane bits not used by the halving steps
+#pragma unroll
+    for (int mask = kRest; mask > 0; mask >>= 1) {
+        const float got = __shfl_xor_sync(0xFFFFFFFFu, r, mask);
+        r = kMax ? fmaxf(r, got) : r + got;
+    }
+    return r;
+}
+
+// Value index whose reduction lane `lane` holds after warp_reduce_halving<N>, and
+// whether that lane is the first of the lanes holding it.
+template <int N>
+__device__ __forceinline__ int halving_owner(int lane) {
+    return N == 16 ? (lane >> 1) : (lane >> 2);
+}
+template <int N>
+__device__ __forceinline__ bool halving_leader(int lane) {
+    return N == 16 ? (lane & 1) == 0 : (lane & 3) == 0;
+}
+
+// NHP: query heads the softmax processes (8 when G <= 8, else 16); the MMA always
+// runs N = 16 with the rows of Q^T past G zero.
+template <int NHP>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
     const int32_t* __restrict__ d_hist, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
     const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv, int max_len, int nsplit,
-    float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ err) {
+    float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
+    uint16_t* __restrict__ out, int* __restrict__ err) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -128,10 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint8_t* gb = smem_raw + (base - raw);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(gb + L::OFF_ABORT);
     float* red = reinterpret_cast<float*>(gb + L::OFF_RED);
-    float* news = reinterpret_cast<float*>(gb + L::OFF_NEWS);
     float* ls = reinterpret_cast<float*>(gb + L::OFF_LS);
-    float* msh = reinterpret_cast<float*>(gb + L::OFF_M);
-    uint16_t* vnew_s = reinterpret_cast<uint16_t*>(gb + L::OFF_VNEW);
     auto bar = [&](int i) -> uint32_t { return base + L::OFF_BAR + 8u * static_cast<uint32_t>(i); };
 
     const int G = Hq / Hkv;
@@ -142,27 +210,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-
-    const int hist = d_hist[b];
-    if (hist < 0 || hist >= max_len) {
-        if (s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
-        return;  // sequence skipped: nothing written
+    const int hist = d_hist[b];  // in flight while the barriers and TMEM are set up
+    if (warp == kWarpTma && lane == 0) {
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
     }
-    const int nkeys = hist + 1;
-    const int per = max((nkeys + nsplit - 1) / nsplit, KT);
-    const int start = s * per;
-    const int end = min(start + per, nkeys);
-    const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * nsplit + s;  // head h adds h * nsplit
-    if (start >= end) {  // an empty split: weight 0 in the combine
-        if (tid < G) {
-            part_ml[(row0 + static_cast<size_t>(tid) * nsplit) * 2 + 0] = -INFINITY;
-            part_ml[(row0 + static_cast<size_t>(tid) * nsplit) * 2 + 1] = 0.f;
-        }
-        return;
-    }
-    const int ntiles = (end - start + KT - 1) / KT;
-    const int kv_row = b * Hkv + g;
-    const bool own_new = hist >= start && hist < end;
 
     if (tid == 0) {
         *abort_flag = 0;
@@ -193,48 +245,122 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<const uint32_t*>(gb + L::OFF_TMEM);
 
-    if (warp == kWarpTma) {
-        // ------------------------------------------------------------ TMA producer (lane 0: K, lane 1: V)
-        if (lane < 2) {
-            const bool is_k = lane == 0;
-            const CUtensorMap* map = is_k ? &map_k : &map_v;
-            const int nst = is_k ? KST : VST;
-            const int full0 = is_k ? B_KFULL0 : B_VFULL0;
-            const int empty0 = is_k ? B_KEMPTY0 : B_VEMPTY0;
-            const uint32_t ring = base + (is_k ? L::OFF_K : L::OFF_V);
-            tma_prefetch_desc(map);
-            int issued = 0;
+    const bool hist_ok = hist >= 0 && hist < max_len;
+    if (!hist_ok && s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
+    const int nkeys = hist + 1;
+    const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds slot p
+    const int kv_row = b * Hkv + g;
+    const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * nsplit + s;  // head h adds h * nsplit
+    int* meta = reinterpret_cast<int*>(gb + L::OFF_META);  // tile index of local tile j at [j % 8]; -1 ends
+
+    if (!hist_ok) {
+        // sequence skipped: nothing written
+    } else if (warp == kWarpTma) {
+        // ------------------------------------------------------------ TMA producer (lane 0)
+        // Tiles are claimed, not fixed: split s starts with tile s, then takes tickets
+        // nsplit, nsplit+1, ... from the (sequence, kv head)'s tile counter until they run
+        // past T, so CTAs that stream faster take more tiles.  The next ticket is claimed
+        // while the current tile's copies are issued.  One thread feeds both rings: the
+        // V slot of tile j frees (PV(j-4) done) before the K slot does (S(j-2) done).
+        if (lane == 0) {
+            int* tile_ctr = counters + gridDim.y * gridDim.z + kv_row;
+            int cur = s < T ? s : T;
+            int nxt = (nsplit > 1 && cur < T) ? nsplit + atomicAdd(tile_ctr, 1) : cur + 1;
+            int issued_k = 0, issued_v = 0;
             bool ok = true;
-            for (int j = 0; j < ntiles; ++j) {
-                const int st = j % nst;
-                if (j >= nst && !mbar_wait(bar(empty0 + st), static_cast<uint32_t>(j / nst - 1) & 1u, abort_flag)) {
+            for (int j = 0;; ++j) {
+                const int tile = cur < T ? cur : -1;
+                const int ks = j % KST, vs = j % VST;
+                if (j >= KST && !mbar_wait(bar(B_KEMPTY0 + ks), static_cast<uint32_t>(j / KST - 1) & 1u, abort_flag)) {
                     ok = false;
                     break;
                 }
-                mbar_arrive_expect_tx(bar(full0 + st), L::TILE);
+                meta[j % 8] = tile;
+                if (tile < 0) {  // no more tiles: complete the K slot's phase without data
+                    mbar_arrive(bar(B_KFULL0 + ks));
+                    break;
+                }
+                mbar_arrive_expect_tx(bar(B_KFULL0 + ks), L::TILE);
 #pragma unroll
                 for (int c = 0; c < 2; ++c)
-                    tma_load_3d(ring + st * L::TILE + c * L::BOX, map, c * 64, start + j * KT, kv_row, bar(full0 + st));
-                issued = j + 1;
+                    tma_load_3d(base + L::OFF_K + ks * L::TILE + c * L::BOX, &map_k, c * 64, tile * KT, kv_row,
+                                bar(B_KFULL0 + ks));
+                issued_k = j + 1;
+                if (j >= VST && !mbar_wait(bar(B_VEMPTY0 + vs), static_cast<uint32_t>(j / VST - 1) & 1u, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                mbar_arrive_expect_tx(bar(B_VFULL0 + vs), L::TILE);
+#pragma unroll
+                for (int c = 0; c < 2; ++c)
+                    tma_load_3d(base + L::OFF_V + vs * L::TILE + c * L::BOX, &map_v, c * 64, tile * KT, kv_row,
+                                bar(B_VFULL0 + vs));
+                issued_v = j + 1;
+                cur = nxt;
+                if (nsplit > 1) {
+                    if (cur < T) nxt = nsplit + atomicAdd(tile_ctr, 1);
+                } else {
+                    nxt = cur + 1;
+                }
             }
             if (!ok) {
                 *abort_flag = 1;
                 atomicOr(err, kDevErrTimeout);
-                for (int t = max(0, issued - nst); t < issued; ++t)
-                    mbar_wait(bar(full0 + t % nst), static_cast<uint32_t>(t / nst) & 1u, nullptr);
+                for (int t = max(0, issued_k - KST); t < issued_k; ++t)
+                    mbar_wait(bar(B_KFULL0 + t % KST), static_cast<uint32_t>(t / KST) & 1u, nullptr);
+                for (int t = max(0, issued_v - VST); t < issued_v; ++t)
+                    mbar_wait(bar(B_VFULL0 + t % VST), static_cast<uint32_t>(t / VST) & 1u, nullptr);
             }
         }
     } else if (warp == kWarpMma) {
-        // ------------------------------------------------------------ tcgen05 issuer
-        if (lane == 0) {
-            constexpr uint32_t kIdQK = idesc_bf16_f32(KT, NH, false, false);
-            constexpr uint32_t kIdPV = idesc_bf16_f32(D, NH, true, false);
-            const uint32_t sQ = base + L::OFF_Q;
-            auto issue_pv = [&](int jj) -> bool {
-                if (!mbar_wait(bar(B_PFULL0 + (jj & 1)), static_cast<uint32_t>(jj >> 1) & 1u, abort_flag)) return false;
-                if (!mbar_wait(bar(B_VFULL0 + jj % VST), static_cast<uint32_t>(jj / VST) & 1u, abort_flag)) return false;
+        // ------------------------------------------------------------ tcgen05 issuer (+ the new token)
+        // Lane l handles dimensions 4l .. 4l+3 of the new token (rotated by every CTA;
+        // written by the one that gets tile T-1).
+        const int hrow = hist - (T - 1) * KT;  // row of slot p in tile T-1
+        uint2 k_rot, v_val;
+        {
+            const int d0 = 4 * lane;
+            const int dp = d0 < HALF ? d0 + HALF : d0 - HALF;  // RoPE partner dimensions
+            const uint2 kx = *reinterpret_cast<const uint2*>(k_new + static_cast<size_t>(kv_row) * D + d0);
+            const uint2 ky = *reinterpret_cast<const uint2*>(k_new + static_cast<size_t>(kv_row) * D + dp);
+            v_val = *reinterpret_cast<const uint2*>(v_new + static_cast<size_t>(kv_row) * D + d0);
+            const float4 c4 = *reinterpret_cast<const float4*>(cos_tab + static_cast<size_t>(hist) * HALF + d0 % HALF);
+            const float4 s4 = *reinterpret_cast<const float4*>(sin_tab + static_cast<size_t>(hist) * HALF + d0 % HALF);
+            const float xs[4] = {__uint_as_float(kx.x << 16), __uint_as_float(kx.x & 0xFFFF0000u),
+                                 __uint_as_float(kx.y << 16), __uint_as_float(kx.y & 0xFFFF0000u)};
+            const float ys[4] = {__uint_as_float(ky.x << 16), __uint_as_float(ky.x & 0xFFFF0000u),
+                                 __uint_as_float(ky.y << 16), __uint_as_float(ky.y & 0xFFFF0000u)};
+            const float cs[4] = {c4.x, c4.y, c4.z, c4.w}, ss[4] = {s4.x, s4.y, s4.z, s4.w};
+            uint32_t kb[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float r = d0 < HALF ? __fsub_rn(__fmul_rn(xs[e], cs[e]), __fmul_rn(ys[e], ss[e]))
+                                          : __fadd_rn(__fmul_rn(xs[e], cs[e]), __fmul_rn(ys[e], ss[e]));
+                kb[e] = to_bf16(r);
+            }
+            k_rot = make_uint2(kb[0] | (kb[1] << 16), kb[2] | (kb[3] << 16));
+        }
+        constexpr uint32_t kIdQK = idesc_bf16_f32(KT, NH, false, false);
+        constexpr uint32_t kIdPV = idesc_bf16_f32(D, NH, true, false);
+        const uint32_t sQ = base + L::OFF_Q;
+        auto wait_all = [&](int barrier, uint32_t parity) -> bool {
+            return __all_sync(0xFFFFFFFFu, mbar_wait(bar(barrier), parity, abort_flag));
+        };
+        auto issue_pv = [&](int jj) -> bool {
+            if (!wait_all(B_PFULL0 + (jj & 1), static_cast<uint32_t>(jj >> 1) & 1u)) return false;
+            if (!wait_all(B_VFULL0 + jj % VST, static_cast<uint32_t>(jj / VST) & 1u)) return false;
+            const uint32_t sV = base + L::OFF_V + (jj % VST) * L::TILE;
+            if (meta[jj % 8] == T - 1) {
+                // v_new into row hrow; the rows past it (slots past p) zeroed
+                uint8_t* vt = gb + L::OFF_V + (jj % VST) * L::TILE;
+                *reinterpret_cast<uint2*>(vt + sw_elem(hrow, 4 * lane, KT)) = v_val;
+                for (int i = (hrow + 1) * 16 + lane; i < KT * 16; i += 32)
+                    *reinterpret_cast<uint4*>(vt + sw_elem(i >> 4, 8 * (i & 15), KT)) = make_uint4(0, 0, 0, 0);
+                fence_proxy_async_smem();
+            }
+            __syncwarp();
+            if (lane == 0) {
                 tc_fence_after();
-                const uint32_t sV = base + L::OFF_V + (jj % VST) * L::TILE;
                 const uint32_t sP = base + L::OFF_P + (jj & 1) * (2 * NH * 128);
 #pragma unroll
                 for (int kk = 0; kk < KT / 16; ++kk)
@@ -243,19 +369,35 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                             (jj > 0 || kk > 0) ? 1u : 0u);
                 umma_commit(bar(B_PVDONE));
                 umma_commit(bar(B_VEMPTY0 + jj % VST));
-                return true;
-            };
-            bool ok = mbar_wait(bar(B_QREADY), 0, abort_flag);
-            if (ok) {
-                tc_fence_after();
-                for (int j = 0; j < ntiles; ++j) {
-                    const int ks = j % KST;
-                    if (!mbar_wait(bar(B_KFULL0 + ks), static_cast<uint32_t>(j / KST) & 1u, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
+            }
+            __syncwarp();
+            return true;
+        };
+        bool ok = wait_all(B_QREADY, 0);
+        int n = 0;  // tiles this CTA processes
+        if (ok) {
+            for (int j = 0;; ++j) {
+                const int ks = j % KST;
+                if (!wait_all(B_KFULL0 + ks, static_cast<uint32_t>(j / KST) & 1u)) {
+                    ok = false;
+                    break;
+                }
+                const int tile = meta[j % 8];
+                if (tile < 0) {
+                    n = j;
+                    break;
+                }
+                const uint32_t sK = base + L::OFF_K + ks * L::TILE;
+                if (tile == T - 1) {  // the new token: to the cache, and its rotated k into row hrow
+                    const size_t dst = (static_cast<size_t>(kv_row) * max_len + hist) * D + 4 * lane;
+                    *reinterpret_cast<uint2*>(k_cache + dst) = k_rot;
+                    *reinterpret_cast<uint2*>(v_cache + dst) = v_val;
+                    *reinterpret_cast<uint2*>(gb + L::OFF_K + ks * L::TILE + sw_elem(hrow, 4 * lane, KT)) = k_rot;
+                    fence_proxy_async_smem();
+                }
+                __syncwarp();
+                if (lane == 0) {
                     tc_fence_after();
-                    const uint32_t sK = base + L::OFF_K + ks * L::TILE;
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
                         const uint32_t off = (kk >> 2) * L::BOX + (kk & 3) * 32;
@@ -265,138 +407,134 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     }
                     umma_commit(bar(B_SFULL0 + (j & 1)));
                     umma_commit(bar(B_KEMPTY0 + ks));  // K is consumed once S^T(j) completes
-                    if (j >= 1 && !issue_pv(j - 1)) {
-                        ok = false;
-                        break;
-                    }
                 }
-                if (ok) ok = issue_pv(ntiles - 1);
-                if (ok) umma_commit(bar(B_OFULL));  // the epilogue's signal: every PV is complete
+                __syncwarp();
+                if (j >= 1 && !issue_pv(j - 1)) {
+                    ok = false;
+                    break;
+                }
             }
-            if (!ok) {
-                *abort_flag = 1;
-                atomicOr(err, kDevErrTimeout);
+            if (ok) {
+                // the softmax learns the count from the same end marker: S buffer n's phase
+                // completes without an MMA (S(n-2) on that buffer was consumed: PFULL(n-2) seen)
+                if (lane == 0) mbar_arrive(bar(B_SFULL0 + (n & 1)));
+                if (n > 0) ok = issue_pv(n - 1);
+                if (ok && n > 0 && lane == 0) umma_commit(bar(B_OFULL));  // every PV is complete
             }
+        }
+        if (!ok && lane == 0) {
+            *abort_flag = 1;
+            atomicOr(err, kDevErrTimeout);
+        }
+        if (lane == 0) {
             umma_commit(bar(B_DRAIN));
             mbar_wait(bar(B_DRAIN), 0, nullptr);
         }
+        __syncwarp();
     } else {
         // ------------------------------------------------------------ softmax / epilogue (one thread per key)
         const int t = tid;  // key row of a tile; output dimension in the epilogue
         const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-        uint8_t* qs = gb + L::OFF_Q;
-        const float* cos_row = cos_tab + static_cast<size_t>(hist) * HALF;
-        const float* sin_row = sin_tab + static_cast<size_t>(hist) * HALF;
-        // Q^T: row h = rotated q of head h0 + h (bf16), zero rows past G; P^T buffers zeroed.
-        // Each thread owns dimension t of every head: all loads first, then the math.
-        const int tp = t < HALF ? t + HALF : t - HALF;  // RoPE partner dimension
-        const float c_t = cos_row[t % HALF], s_t = sin_row[t % HALF];
-        float qx[NH], qy[NH];
+        {
+            // Q^T: row h = rotated q of head h0 + h (bf16), zero rows past G; P^T buffers zeroed.
+            // Each thread owns dimension t of every head: all loads first, then the math.
+            uint8_t* qs = gb + L::OFF_Q;
+            const float* cos_row = cos_tab + static_cast<size_t>(hist) * HALF;
+            const float* sin_row = sin_tab + static_cast<size_t>(hist) * HALF;
+            const int tp = t < HALF ? t + HALF : t - HALF;  // RoPE partner dimension
+            const float c_t = cos_row[t % HALF], s_t = sin_row[t % HALF];
+            float qx[NHP], qy[NHP];
 #pragma unroll
-        for (int h = 0; h < NH; ++h) {
-            const uint16_t* qrow = q + (static_cast<size_t>(b) * Hq + h0 + min(h, G - 1)) * D;
-            qx[h] = bf16_at(qrow + t);
-            qy[h] = bf16_at(qrow + tp);
-        }
-        float qhat[NH];
-#pragma unroll
-        for (int h = 0; h < NH; ++h) {
-            const float r = t < HALF ? __fsub_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t))
-                                     : __fadd_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t));
-            const uint16_t qb = h < G ? to_bf16(r) : 0;
-            qhat[h] = __uint_as_float(static_cast<uint32_t>(qb) << 16);
-            *reinterpret_cast<uint16_t*>(qs + sw_elem(h, t, NH)) = qb;
-        }
-        for (int i = t; i < 2 * NH * 128 / 16; i += 128)
-            reinterpret_cast<uint4*>(gb + L::OFF_P)[i] = make_uint4(0, 0, 0, 0);
-        if (own_new) {
-            // the new token: rotated k to slot hist, v to slot hist and to shared memory, and
-            // its score q.k_new per head (float, reduced over the 128 dimensions)
-            const uint16_t kr = to_bf16(rope_elem(k_new + static_cast<size_t>(kv_row) * D, t, cos_row, sin_row));
-            const uint16_t vv = v_new[static_cast<size_t>(kv_row) * D + t];
-            const size_t dst = (static_cast<size_t>(kv_row) * max_len + hist) * D + t;
-            k_cache[dst] = kr;
-            v_cache[dst] = vv;
-            vnew_s[t] = vv;
-            const float kf = __uint_as_float(static_cast<uint32_t>(kr) << 16);
+            for (int h = 0; h < NHP; ++h) {
+                const uint16_t* qrow = q + (static_cast<size_t>(b) * Hq + h0 + min(h, G - 1)) * D;
+                qx[h] = bf16_at(qrow + t);
+                qy[h] = bf16_at(qrow + tp);
+            }
 #pragma unroll
             for (int h = 0; h < NH; ++h) {
-                float v = qhat[h] * kf;
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, off);
-                if (lane == 0) red[warp * NH + h] = v;
+                uint16_t qb = 0;
+                if (h < NHP && h < G) {
+                    const float r = t < HALF ? __fsub_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t))
+                                             : __fadd_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t));
+                    qb = to_bf16(r);
+                }
+                *reinterpret_cast<uint16_t*>(qs + sw_elem(h, t, NH)) = qb;
             }
+            for (int i = t; i < 2 * NH * 128 / 16; i += 128)
+                reinterpret_cast<uint4*>(gb + L::OFF_P)[i] = make_uint4(0, 0, 0, 0);
+            fence_proxy_async_smem();
+            mbar_arrive(bar(B_QREADY));
         }
-        fence_proxy_async_smem();
-        named_sync_128();
-        if (own_new && t < NH) news[t] = red[t] + red[NH + t] + red[2 * NH + t] + red[3 * NH + t];
-        mbar_arrive(bar(B_QREADY));
-        named_sync_128();
 
-        float m_run[NH], l_run[NH];
+        float m_run[NHP], l_run[NHP];
 #pragma unroll
-        for (int h = 0; h < NH; ++h) {
+        for (int h = 0; h < NHP; ++h) {
             m_run[h] = -INFINITY;
             l_run[h] = 0.f;
         }
         bool ok = true;
-        for (int j = 0; j < ntiles; ++j) {
+        int n = 0;  // tiles processed
+        for (int j = 0;; ++j) {
             ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + (j & 1)), static_cast<uint32_t>(j >> 1) & 1u, abort_flag));
             if (!ok) break;
+            const int tile = meta[j % 8];
+            if (tile < 0) {
+                n = j;
+                break;
+            }
             tc_fence_after();
-            uint32_t r[NH];
-            tmem_ld16(tmem + lane_base + (j & 1) * NH, r);
+            uint32_t r[NHP];
+            tmem_ld_cols<NHP>(tmem + lane_base + (j & 1) * NH, r);
             tmem_wait_ld();
-            const int key = start + j * KT + t;
-            const bool valid = key < end;
-            float sc[NH];
+            const bool valid = tile * KT + t < nkeys;
+            float sc[NHP];
+            bool exceed = false;
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                const float raw_s = (key == hist) ? news[h] : __uint_as_float(r[h]);
-                sc[h] = (valid && h < G) ? raw_s * scale_log2 : -INFINITY;
+            for (int h = 0; h < NHP; ++h) {
+                sc[h] = (valid && h < G) ? __uint_as_float(r[h]) * scale_log2 : -INFINITY;
+                exceed |= sc[h] > m_run[h] + 8.f;  // lazy: P stays <= 2^8 otherwise
             }
-            // per-head tile max: warp shuffles, then the four warps through shared memory
+            if (named_or_128(exceed)) {
+                // per-head tile maxima: halving butterfly in the warp, then the four warps.
+                // (`red` is rewritten only after the next tile's OR-barrier, which every
+                // thread reaches after its reads below.)
+                float mx[NHP];
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                if (h < G) {  // uniform: padded heads are skipped
-                    float mx = sc[h];
+                for (int h = 0; h < NHP; ++h) mx[h] = sc[h];
+                const float wm = warp_reduce_halving<NHP, true>(mx, lane);
+                if (halving_leader<NHP>(lane)) red[halving_owner<NHP>(lane) * 4 + warp] = wm;
+                named_sync_128();
+                bool any_move = false;
+                float alpha[NHP];
 #pragma unroll
-                    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, off));
-                    if (lane == 0) red[warp * NH + h] = mx;
+                for (int h = 0; h < NHP; ++h) {
+                    const float4 r4 = reinterpret_cast<const float4*>(red)[h];
+                    const float tmx = fmaxf(fmaxf(r4.x, r4.y), fmaxf(r4.z, r4.w));
+                    const bool move = tmx > m_run[h] + 8.f;
+                    alpha[h] = move ? fast_exp2(m_run[h] - tmx) : 1.f;
+                    if (move) m_run[h] = tmx;
+                    any_move |= move;
+                    l_run[h] *= alpha[h];
                 }
-            }
-            named_sync_128();
-            bool any_move = false;
-            float alpha[NH];
+                if (j > 0 && any_move) {  // the same decision in every thread (same tile maxima)
+                    // O^T holds PV through tile j-1 once PV(j-1) completed (S(j) completed after PV(j-2)).
+                    ok = __all_sync(0xFFFFFFFFu,
+                                    mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(j - 1) & 1u, abort_flag));
+                    if (!ok) break;
+                    tc_fence_after();
+                    uint32_t o[NHP];
+                    tmem_ld_cols<NHP>(tmem + lane_base + TM_O, o);
+                    tmem_wait_ld();
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                const float tmx = h < G ? fmaxf(fmaxf(red[h], red[NH + h]), fmaxf(red[2 * NH + h], red[3 * NH + h]))
-                                        : -INFINITY;
-                const float m_cand = fmaxf(m_run[h], tmx);
-                const bool move = m_cand > m_run[h] + 8.f;  // lazy: P stays <= 2^8 otherwise
-                alpha[h] = move ? fast_exp2(m_run[h] - m_cand) : 1.f;
-                if (move) m_run[h] = m_cand;
-                any_move |= move;
-            }
-            named_sync_128();  // every warp has read `red` before the next tile overwrites it
-            if (j > 0 && any_move) {  // the same decision in every thread (same tile maxima)
-                // O^T holds PV through tile j-1 once PV(j-1) completed (S(j) completed after PV(j-2)).
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(j - 1) & 1u, abort_flag));
-                if (!ok) break;
-                tc_fence_after();
-                uint32_t o[NH];
-                tmem_ld16(tmem + lane_base + TM_O, o);
-                tmem_wait_ld();
-#pragma unroll
-                for (int h = 0; h < NH; ++h) o[h] = __float_as_uint(__uint_as_float(o[h]) * alpha[h]);
-                tmem_st16(tmem + lane_base + TM_O, o);
-                tmem_wait_st();
+                    for (int h = 0; h < NHP; ++h) o[h] = __float_as_uint(__uint_as_float(o[h]) * alpha[h]);
+                    tmem_st_cols<NHP>(tmem + lane_base + TM_O, o);
+                    tmem_wait_st();
+                }
             }
             // P^T (bf16, row = head, column = key of the tile); padded heads stay zero
             uint8_t* pbuf = gb + L::OFF_P + (j & 1) * (2 * NH * 128);
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                l_run[h] *= alpha[h];
+            for (int h = 0; h < NHP; ++h) {
                 if (h < G) {
                     const float m_ref = m_run[h] == -INFINITY ? 0.f : m_run[h];
                     const float p = fast_exp2(sc[h] - m_ref);
@@ -404,61 +542,153 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     *reinterpret_cast<uint16_t*>(pbuf + sw_elem(h, t, NH)) = to_bf16(p);
                 }
             }
-            // V rows past the split's end may hold anything: zero them; the new token's v.
-            // (Only the tile that holds them: wait for its V to land first.)
-            uint8_t* vtile = gb + L::OFF_V + (j % VST) * L::TILE;
-            const bool patch = named_or_128(!valid || key == hist);
-            if (patch) {
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_VFULL0 + j % VST), static_cast<uint32_t>(j / VST) & 1u, abort_flag));
-                if (!ok) break;
-            }
-            if (!valid) {
-#pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    *reinterpret_cast<uint4*>(vtile + sw_elem(t, 8 * c, KT)) = make_uint4(0, 0, 0, 0);
-            } else if (key == hist) {
-#pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    *reinterpret_cast<uint4*>(vtile + sw_elem(t, 8 * c, KT)) = reinterpret_cast<const uint4*>(vnew_s)[c];
-            }
             fence_proxy_async_smem();
             tc_fence_before();
             mbar_arrive(bar(B_PFULL0 + (j & 1)));
         }
-        // (PVDONE could be two phases behind here -- PV(ntiles-2) may still run -- so
-        // the epilogue waits on its own barrier, committed once after the last PV.)
-        if (ok) ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL), 0u, abort_flag));
-        if (ok) {
+        if (ok && n == 0) {
+            if (t < G) {  // no tile came to this CTA: weight 0 in the merge
+                part_ml[(row0 + static_cast<size_t>(t) * nsplit) * 2 + 0] = -INFINITY;
+                part_ml[(row0 + static_cast<size_t>(t) * nsplit) * 2 + 1] = 0.f;
+            }
+        } else if (ok) {
+            // (PVDONE could be two phases behind here -- PV(n-2) may still run -- so the
+            // epilogue waits on its own barrier, committed once after the last PV.)
+            ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL), 0u, abort_flag));
+        }
+        if (ok && n > 0) {
             // row sums: every thread holds a partial over its keys
-#pragma unroll
-            for (int h = 0; h < NH; ++h) {
-                if (h < G) {
-                    float v = l_run[h];
-#pragma unroll
-                    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, off);
-                    if (lane == 0) ls[warp * NH + h] = v;
-                }
-            }
-            if (t == 0) {  // every thread holds the same running maxima
-#pragma unroll
-                for (int h = 0; h < NH; ++h) msh[h] = m_run[h];
-            }
+            const float wl = warp_reduce_halving<NHP, false>(l_run, lane);
+            if (halving_leader<NHP>(lane)) ls[halving_owner<NHP>(lane) * 4 + warp] = wl;
             tc_fence_after();
-            uint32_t o[NH];
-            tmem_ld16(tmem + lane_base + TM_O, o);  // thread t = output dimension d
+            uint32_t o[NHP];
+            tmem_ld_cols<NHP>(tmem + lane_base + TM_O, o);  // thread t = output dimension d
             tmem_wait_ld();
             named_sync_128();
-            for (int h = 0; h < G; ++h) {
-                const size_t row = row0 + static_cast<size_t>(h) * nsplit;
-                part_o[row * D + t] = __uint_as_float(o[h]);
-                if (t == 0) {
-                    part_ml[row * 2 + 0] = msh[h];
-                    part_ml[row * 2 + 1] = ls[h] + ls[NH + h] + ls[2 * NH + h] + ls[3 * NH + h];
+#pragma unroll
+            for (int h = 0; h < NHP; ++h) {
+                if (h < G) {
+                    const float4 l4 = reinterpret_cast<const float4*>(ls)[h];
+                    const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
+                    if (nsplit == 1) {
+                        out[(static_cast<size_t>(b) * Hq + h0 + h) * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
+                    } else {
+                        const size_t row = row0 + static_cast<size_t>(h) * nsplit;
+                        part_o[row * D + t] = __uint_as_float(o[h]);
+                        if (t == 0) {
+                            part_ml[row * 2 + 0] = m_run[h];
+                            part_ml[row * 2 + 1] = l_tot;
+                        }
+                    }
                 }
             }
-        } else {
+        } else if (!ok) {
             *abort_flag = 1;
             atomicOr(err, kDevErrTimeout);
+        }
+    }
+
+    // ---------------------------------------------------------------- merge of the splits
+    if (hist_ok && nsplit > 1) {
+        int* last_flag = reinterpret_cast<int*>(gb + L::OFF_LAST);
+        __threadfence();  // this CTA's partials are visible before it is counted
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            int* cnt = counters + kv_row;
+            const int last = atomicAdd(cnt, 1) == nsplit - 1;
+            if (last) {  // every split of this launch has been counted and has claimed its last tile
+                *cnt = 0;
+                counters[gridDim.y * gridDim.z + kv_row] = 0;
+            }
+            *last_flag = last;
+        }
+        __syncthreads();
+        tc_fence_after();
+        if (*last_flag) {
+            // All six warps merge; shared memory of the (idle) K ring holds
+            //   wml  [G][nsplit] float2: (m_s, l_s), then (weight_s, -) per head and split
+            //   winv [G]         1 / L per head
+            //   racc [6 warps][G][D] float: each warp's weighted sum over its splits.
+            // Splits without keys have l = 0 and weight 0; their accumulators were never
+            // written, and what is read there is discarded.
+            __threadfence();
+            float2* wml = reinterpret_cast<float2*>(gb + L::OFF_K);
+            float* winv = reinterpret_cast<float*>(gb + L::OFF_K + NH * 256 * 8);
+            float* racc = winv + NH;
+            const size_t hrow0 = (static_cast<size_t>(b) * Hq + h0) * nsplit;  // row of (head 0, split 0)
+            const int npair = G * nsplit;
+            for (int p = tid; p < npair; p += kThreads)  // pair p = (head p / nsplit, split p % nsplit)
+                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + hrow0 + p);
+            __syncthreads();
+            for (int h = warp; h < G; h += kThreads / 32) {  // per head: M, weights, 1/L
+                float mm = -INFINITY;
+                for (int sp = lane; sp < nsplit; sp += 32) {
+                    const float2 ml = wml[h * nsplit + sp];
+                    if (ml.y > 0.f) mm = fmaxf(mm, ml.x);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xFFFFFFFFu, mm, off));
+                float ll = 0.f;
+                for (int sp = lane; sp < nsplit; sp += 32) {
+                    const float2 ml = wml[h * nsplit + sp];
+                    const float wgt = ml.y > 0.f ? fast_exp2(ml.x - mm) : 0.f;
+                    wml[h * nsplit + sp].x = wgt;
+                    ll += ml.y * wgt;
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) ll += __shfl_xor_sync(0xFFFFFFFFu, ll, off);
+                if (lane == 0) winv[h] = 1.f / ll;
+            }
+            __syncthreads();
+            // warp w: splits w, w+6, ...; lane l: dimensions 4l .. 4l+3 of every head
+            float4 acc[NHP];
+#pragma unroll
+            for (int h = 0; h < NHP; ++h) acc[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+            // (Every load is issued unconditionally -- padded heads re-read head G-1 -- and
+            // weight-0 values are dropped by a select, so that the loads of a split for
+            // all heads are in flight together instead of each waiting on a branch.)
+#pragma unroll 2
+            for (int sp = warp; sp < nsplit; sp += kThreads / 32) {
+                float4 o4[NHP];
+                float wgt[NHP];
+#pragma unroll
+                for (int h = 0; h < NHP; ++h) {
+                    const int hh = min(h, G - 1);
+                    wgt[h] = h < G ? wml[hh * nsplit + sp].x : 0.f;
+                    o4[h] = __ldcg(reinterpret_cast<const float4*>(
+                                       part_o + (hrow0 + static_cast<size_t>(hh) * nsplit + sp) * D) + lane);
+                }
+#pragma unroll
+                for (int h = 0; h < NHP; ++h) {
+                    const bool use = wgt[h] != 0.f;
+                    acc[h].x = use ? fmaf(wgt[h], o4[h].x, acc[h].x) : acc[h].x;
+                    acc[h].y = use ? fmaf(wgt[h], o4[h].y, acc[h].y) : acc[h].y;
+                    acc[h].z = use ? fmaf(wgt[h], o4[h].z, acc[h].z) : acc[h].z;
+                    acc[h].w = use ? fmaf(wgt[h], o4[h].w, acc[h].w) : acc[h].w;
+                }
+            }
+#pragma unroll
+            for (int h = 0; h < NHP; ++h)
+                if (h < G) reinterpret_cast<float4*>(racc + (warp * NH + h) * D)[lane] = acc[h];
+            __syncthreads();
+            for (int p = tid; p < G * (D / 4); p += kThreads) {  // (head, 4 dimensions)
+                const int h = p / (D / 4), c = p % (D / 4);
+                float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int w = 0; w < kThreads / 32; ++w) {
+                    const float4 v4 = reinterpret_cast<const float4*>(racc + (w * NH + h) * D)[c];
+                    sum.x += v4.x;
+                    sum.y += v4.y;
+                    sum.z += v4.z;
+                    sum.w += v4.w;
+                }
+                const float inv = winv[h];
+                const uint2 packed = make_uint2(
+                    to_bf16(sum.x * inv) | (static_cast<uint32_t>(to_bf16(sum.y * inv)) << 16),
+                    to_bf16(sum.z * inv) | (static_cast<uint32_t>(to_bf16(sum.w * inv)) << 16));
+                *reinterpret_cast<uint2*>(out + (static_cast<size_t>(b) * Hq + h0 + h) * D + 4 * c) = packed;
+            }
         }
     }
     tc_fence_before();
@@ -472,26 +702,20 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
 }  // namespace
 
 cudaError_t configure_decode_tc() {
-    return cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
+    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(decode_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
+    return e;
 }
 
+// One wave of CTAs, one per SM: with fewer (sequence, kv head) items than SMs, each
+// item gets floor(SMs / items) splits; otherwise one split per item.
 int decode_tc_num_splits(const Shape& s, int num_sms) {
     const long items = static_cast<long>(s.batch) * s.n_kv_heads;
-    const long slots = num_sms;  // one CTA per SM
-    const long cap = std::max(1L, std::min<long>(256, (s.max_len + KT - 1) / KT));
-    long best = 1;
-    double best_eff = 0.0;
-    for (long ns = 1; ns <= cap; ++ns) {
-        const long ctas = items * ns;
-        if (ctas < slots && ns < cap) continue;
-        const double eff = static_cast<double>(ctas) / static_cast<double>(slots * ((ctas + slots - 1) / slots));
-        if (eff >= 0.9) return static_cast<int>(ns);
-        if (eff > best_eff) {
-            best_eff = eff;
-            best = ns;
-        }
-    }
-    return static_cast<int>(best);
+    const long max_tiles = std::max(1L, static_cast<long>((s.max_len + KT - 1) / KT));
+    long ns = items >= num_sms ? 1 : num_sms / items;
+    ns = std::min(ns, std::min(max_tiles, 256L));
+    return static_cast<int>(std::max(1L, ns));
 }
 
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
@@ -513,13 +737,21 @@ cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const ui
 
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
                              const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
-                             const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml, int nsplit,
-                             int* err, cudaStream_t st) {
+                             const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
+                             int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
-    decode_tc_kernel<<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, k_cache, v_cache,
-                                                       cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads, s.max_len, nsplit,
-                                                       scale_log2, part_o, part_ml, err);
+    const int G = s.n_q_heads / s.n_kv_heads;
+    if (G <= 8)
+        decode_tc_kernel<8><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, k_cache,
+                                                              v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
+                                                              s.max_len, nsplit, scale_log2, part_o, part_ml,
+                                                              counters, out, err);
+    else
+        decode_tc_kernel<16><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, k_cache,
+                                                               v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
+                                                               s.max_len, nsplit, scale_log2, part_o, part_ml,
+                                                               counters, out, err);
     return cudaGetLastError();
 }
 

@@ -57,15 +57,19 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
                                 const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                                 int nsplit, int* err, cudaStream_t st);
 // K3 for head_dim 128 on the tensor cores (decode_tc.cu): one CTA per SM, maps with
-// 128-key boxes; same partial layout as launch_decode_split.
+// 128-key boxes; same partial layout as launch_decode_split, but the merge is fused
+// in (the last CTA of each (b, kv head) merges and writes `out`), so no K4 follows.
+// Splits claim key tiles from a per-(b, kv head) counter.  `counters`: 2*B*Hkv ints
+// (merge counts, then tile claims), zero before the first launch; every launch leaves
+// them zero.
 cudaError_t configure_decode_tc();
 int decode_tc_num_splits(const Shape& s, int num_sms);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                                 const uint16_t* v_cache, DecodeMaps* maps);
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
                              const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
-                             const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml, int nsplit,
-                             int* err, cudaStream_t st);
+                             const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
+                             int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
                                   int nsplit, uint16_t* out, cudaStream_t st);
 

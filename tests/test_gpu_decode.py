@@ -109,3 +109,30 @@ def test_decode_out_of_range_length_sets_error_and_skips(torch):
     r0k, r0v = rk[:1].copy(), rv[:1].copy()
     ref = O.decode(one, q[:1].copy(), k[:1].copy(), v[:1].copy(), np.array([100], np.int32), r0k, r0v)
     assert_out_close(out[:1], ref, "valid sequence next to invalid ones")
+
+
+def test_decode_chain_reuses_merge_state(torch):
+    """Consecutive decode steps on one context and one cache: each step appends its
+    token and attends to the previous steps' tokens; tile boundaries (128, 256) and
+    splits without keys are crossed on the way.  Checks that nothing a step leaves
+    behind on the device (merge counters, partials) changes the next step."""
+    from paper_2607_15865_gb300.attention import Attention
+    shape = Shape("chain", 2, 16, 8, 128, 1024, 1.0e4)
+    hist0 = np.array([126, 254], np.int32)
+    steps = 4
+    kc, vc = w.cache(shape, "chain", int(hist0.max()), fill="random")
+    attn = Attention.for_shape(shape)
+    gk, gv = to_dev(kc), to_dev(vc)
+    rk, rv = kc.copy(), vc.copy()
+    for i in range(steps):
+        hist = hist0 + i
+        q, k, v = w.tokens(shape, f"chain_{i}", 1)
+        hl = torch.from_numpy(hist).cuda()
+        out = to_host(attn.decode(to_dev(q), to_dev(k), to_dev(v), hl, gk, gv))
+        ref = O.decode(shape, q, k, v, hist, rk, rv)  # appends to rk, rv in place
+        assert_out_close(out, ref, f"chain step {i}")
+    torch.cuda.synchronize()
+    assert attn.device_error() == 0
+    assert_cache(to_host(gk), to_host(gv), rk, rv, kc, vc,
+                 [(int(h), int(h) + steps) for h in hist0], "chain cache")
+    attn.close()
