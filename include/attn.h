@@ -36,9 +36,10 @@
  *
  * Ownership.  The caller owns every device buffer passed to a call.  The
  * context owns only its own device memory: the RoPE tables (2 x max_len x
- * head_dim/2 floats), the decode split-KV partials (batch x n_q_heads x 256 x
- * (head_dim + 2) floats), the prefill partials of split work (SM count x 256 x
- * (head_dim + 2) floats) and a device error word; all allocated by attn_create
+ * head_dim/2 floats, held twice: position-major and pair-major), the decode
+ * split-KV partials (batch x n_q_heads x 256 x (head_dim + 2) floats) and counters
+ * (2 x batch x n_kv_heads ints), the prefill partials of split work (SM count x
+ * 256 x (head_dim + 2) floats) and a device error word; all allocated by attn_create
  * and freed by attn_destroy.  No stage call allocates, frees or synchronises: each one only
  * enqueues kernels on `stream` and returns.  Calls that use the same context
  * share its scratch buffers, so they must not run concurrently on different

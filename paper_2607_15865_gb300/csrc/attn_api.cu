@@ -29,8 +29,10 @@ struct attn_ctx {
     int device;
     int num_sms;
     int nsplit_max;
-    float* d_cos;
+    float* d_cos;       // RoPE tables [max_len][D/2]
     float* d_sin;
+    float* d_cos_t;     // the same, pair-major [D/2][max_len] (flash_fwd's q rows)
+    float* d_sin_t;
     float* d_part_o;
     float* d_part_ml;
     int* d_counters;    // decode counters, [2][B * Hkv] (merge count, tile claims), zero between launches
@@ -146,7 +148,7 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
     e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&](int* n) {
-        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos, c->d_sin, out, c->d_flash_o, c->d_flash_ml,
+        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos_t, c->d_sin_t, out, c->d_flash_o, c->d_flash_ml,
                                       c->d_err, c->num_sms, st, n);
     });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
@@ -196,19 +198,23 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     // RoPE tables (Section 4.6.2): cos/sin of p * theta^(-2j/D), evaluated in double, stored as float.
     const int half = cfg->head_dim / 2;
     const size_t ntab = static_cast<size_t>(cfg->max_len) * half;
-    std::vector<float> hc(ntab), hs(ntab);
+    std::vector<float> hc(ntab), hs(ntab), hct(ntab), hst(ntab);
     for (int p = 0; p < cfg->max_len; ++p) {
         for (int j = 0; j < half; ++j) {
             const double inv_freq = std::pow(cfg->rope_theta, -(2.0 * j) / static_cast<double>(cfg->head_dim));
             const double ang = static_cast<double>(p) * inv_freq;
             hc[static_cast<size_t>(p) * half + j] = static_cast<float>(std::cos(ang));
             hs[static_cast<size_t>(p) * half + j] = static_cast<float>(std::sin(ang));
+            hct[static_cast<size_t>(j) * cfg->max_len + p] = hc[static_cast<size_t>(p) * half + j];
+            hst[static_cast<size_t>(j) * cfg->max_len + p] = hs[static_cast<size_t>(p) * half + j];
         }
     }
     const size_t part_rows = static_cast<size_t>(cfg->batch) * cfg->n_q_heads * c->nsplit_max;
     bool oom = false;
     oom |= cudaMalloc(&c->d_cos, ntab * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_sin, ntab * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_cos_t, ntab * sizeof(float)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_sin_t, ntab * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_part_o, part_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_part_ml, part_rows * 2 * sizeof(float)) != cudaSuccess;
     const size_t piece_rows = static_cast<size_t>(c->num_sms) * 256;
@@ -224,6 +230,8 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     }
     e = cudaMemcpy(c->d_cos, hc.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemcpy(c->d_sin, hs.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->d_cos_t, hct.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->d_sin_t, hst.data(), ntab * sizeof(float), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(c->d_counters, 0, n_counters * sizeof(int));
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
@@ -241,6 +249,8 @@ void attn_destroy(attn_ctx* c) {
     free_events(c);
     cudaFree(c->d_cos);
     cudaFree(c->d_sin);
+    cudaFree(c->d_cos_t);
+    cudaFree(c->d_sin_t);
     cudaFree(c->d_part_o);
     cudaFree(c->d_part_ml);
     cudaFree(c->d_flash_o);

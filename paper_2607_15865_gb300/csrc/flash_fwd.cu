@@ -29,7 +29,8 @@
 // the softmax warpgroup may rescale O_T right away.  O is rescaled lazily (only
 // when the running max grows by more than 2^8, exact in value).
 // Per row: RoPE of the q row in shared memory before the first MMA (cos/sin
-// gathered by position, Section 4.6.2, float arithmetic and bf16 rounding as K1),
+// gathered by position from pair-major copies of the tables, Section 4.6.2, float
+// arithmetic and bf16 rounding as K1),
 // scores from TMEM, causal mask by index compare on diagonal tiles (no mask
 // tensor), online softmax in the log2 domain, O / l -> bf16 -> out.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its
@@ -160,27 +161,37 @@ __device__ __forceinline__ Unit decode_unit(int lin, int S, int H, int Hq, int G
     return u;
 }
 
-// RoPE of one q row of a tile in shared memory (pairs j, j + D/2, table row of its
-// position, float arithmetic with each product and the difference/sum rounded
+// RoPE tables of one position in registers: cos/sin of pairs j = 0 .. D/2-1.  They are
+// read from pair-major copies of the tables ([D/2][max_len]: entry (j, p) at
+// j * stride + p), so that the 32 threads of a warp -- 32 consecutive positions --
+// read one coalesced line per pair, and are loaded before the q tile lands.
+template <int D>
+struct RopeRow {
+    float c[D / 2], s[D / 2];
+};
+
+template <int D>
+__device__ __forceinline__ void rope_load(RopeRow<D>& t, int pos, const float* __restrict__ cos_t,
+                                          const float* __restrict__ sin_t, int stride) {
+#pragma unroll
+    for (int j = 0; j < D / 2; ++j) {
+        t.c[j] = __ldg(cos_t + static_cast<size_t>(j) * stride + pos);
+        t.s[j] = __ldg(sin_t + static_cast<size_t>(j) * stride + pos);
+    }
+}
+
+// RoPE of one q row of a tile in shared memory (pairs j, j + D/2, with the tables of
+// its position; float arithmetic with each product and the difference/sum rounded
 // separately, bf16 result), as K1 applies to keys.
 template <int D>
-__device__ __forceinline__ void rope_row_smem(uint8_t* qtile, int row, int pos, const float* __restrict__ cos_tab,
-                                              const float* __restrict__ sin_tab) {
+__device__ __forceinline__ void rope_row_smem(uint8_t* qtile, int row, const RopeRow<D>& t) {
     constexpr int HALF = D / 2;
-    const float* crow = cos_tab + static_cast<size_t>(pos) * HALF;
-    const float* srow = sin_tab + static_cast<size_t>(pos) * HALF;
 #pragma unroll
     for (int u = 0; u < HALF / 8; ++u) {
         const int jlo = 8 * u;
         uint4* plo = reinterpret_cast<uint4*>(qtile + sw128_offset(row, jlo));
         uint4* phi = reinterpret_cast<uint4*>(qtile + sw128_offset(row, jlo + HALF));
         const uint4 xa = *plo, xb = *phi;
-        const float4 c0 = *reinterpret_cast<const float4*>(crow + jlo);
-        const float4 c1 = *reinterpret_cast<const float4*>(crow + jlo + 4);
-        const float4 s0 = *reinterpret_cast<const float4*>(srow + jlo);
-        const float4 s1 = *reinterpret_cast<const float4*>(srow + jlo + 4);
-        const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-        const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
         const uint32_t wa[4] = {xa.x, xa.y, xa.z, xa.w};
         const uint32_t wb[4] = {xb.x, xb.y, xb.z, xb.w};
         uint32_t ya[4], yb[4];
@@ -191,7 +202,7 @@ __device__ __forceinline__ void rope_row_smem(uint8_t* qtile, int row, int pos, 
             for (int k2 = 0; k2 < 2; ++k2) {
                 const float a = k2 ? bf_hi(wa[e]) : bf_lo(wa[e]);
                 const float bb = k2 ? bf_hi(wb[e]) : bf_lo(wb[e]);
-                const float cc = c[2 * e + k2], ss = s[2 * e + k2];
+                const float cc = t.c[jlo + 2 * e + k2], ss = t.s[jlo + 2 * e + k2];
                 lo[k2] = __fsub_rn(__fmul_rn(a, cc), __fmul_rn(bb, ss));
                 hi[k2] = __fadd_rn(__fmul_rn(bb, cc), __fmul_rn(a, ss));
             }
@@ -207,9 +218,12 @@ __device__ __forceinline__ void rope_row_smem(uint8_t* qtile, int row, int pos, 
 template <int D>
 __device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint32_t parity, const volatile int* abort,
                                           uint8_t* qtile, int row, int rows, int pos0,
-                                          const float* __restrict__ cos_tab, const float* __restrict__ sin_tab) {
+                                          const float* __restrict__ cos_t, const float* __restrict__ sin_t,
+                                          int stride) {
+    RopeRow<D> tabs;
+    rope_load<D>(tabs, row < rows ? pos0 + row : pos0, cos_t, sin_t, stride);
     const bool w = __all_sync(0xFFFFFFFFu, mbar_wait(qfull, parity, abort));
-    if (w && row < rows) rope_row_smem<D>(qtile, row, pos0 + row, cos_tab, sin_tab);
+    if (w && row < rows) rope_row_smem<D>(qtile, row, tabs);
     fence_proxy_async_smem();
     mbar_arrive(qready);
     return w;
@@ -219,8 +233,8 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                      const __grid_constant__ CUtensorMap map_v, int S, int H, int Hq, int Hkv, int batch,
-                     int n_pairs, int head, int nsplit, float scale_log2, const float* __restrict__ cos_tab,
-                     const float* __restrict__ sin_tab, uint16_t* __restrict__ out, float* __restrict__ ws_o,
+                     int n_pairs, int head, int nsplit, float scale_log2, const float* __restrict__ cos_t,
+                     const float* __restrict__ sin_t, int tab_stride, uint16_t* __restrict__ out, float* __restrict__ ws_o,
                      float* __restrict__ ws_ml, int* __restrict__ err) {
     using L = Layout<D>;
     extern __shared__ uint8_t smem_raw[];
@@ -447,7 +461,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lin < n_units) {
             un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
             ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
-                              un.it.rows(t), H + un.it.q0(t), cos_tab, sin_tab);
+                              un.it.rows(t), H + un.it.q0(t), cos_t, sin_t, tab_stride);
             ++items;
         }
         while (lin < n_units && ok) {
@@ -541,7 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (next < n_units) {
                 nun = decode_unit(next, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
-                                  row, nun.it.rows(t), H + nun.it.q0(t), cos_tab, sin_tab);
+                                  row, nun.it.rows(t), H + nun.it.q0(t), cos_t, sin_t, tab_stride);
                 ++items;
                 if (!ok) break;
             }
@@ -684,14 +698,14 @@ Schedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
 }
 
 template <int D>
-cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                     const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+                     const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                      cudaStream_t st, int* n_launched) {
     const Schedule sc = make_schedule(s, hist, chunk, num_sms);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     flash_fwd_kernel<D><<<sc.grid, kThreads, Layout<D>::ALLOC, st>>>(
         maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head, sc.nsplit,
-        scale_log2, cos_tab, sin_tab, out, ws_o, ws_ml, err);
+        scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
     cudaError_t e = cudaGetLastError();
     *n_launched = 1;
     if (e != cudaSuccess || sc.nsplit == 1) return e;
@@ -729,12 +743,12 @@ cudaError_t configure_flash_fwd() {
     return e != cudaSuccess ? e : configure_d<64>();
 }
 
-cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                             const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+                             const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                              cudaStream_t st, int* n_launched) {
     if (s.head_dim == 128)
-        return launch_d<128>(s, maps, hist, chunk, cos_tab, sin_tab, out, ws_o, ws_ml, err, num_sms, st, n_launched);
-    return launch_d<64>(s, maps, hist, chunk, cos_tab, sin_tab, out, ws_o, ws_ml, err, num_sms, st, n_launched);
+        return launch_d<128>(s, maps, hist, chunk, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
+    return launch_d<64>(s, maps, hist, chunk, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
 }
 
 }  // namespace attn

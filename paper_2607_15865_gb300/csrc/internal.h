@@ -36,8 +36,9 @@ cudaError_t configure_flash_fwd();
 // Work is split across num_sms persistent CTAs; items of the last, partial round are
 // cut into KV pieces whose partials go to ws_o [num_sms*256, D] / ws_ml [num_sms*256, 2]
 // and are merged by a second kernel (then *n_launched = 2).
-cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_tab,
-                             const float* sin_tab, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+// cos_t / sin_t: the RoPE tables pair-major, [D/2][max_len] (entry (j, p) at j * max_len + p).
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+                             const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                              cudaStream_t st, int* n_launched);
 
 // K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
