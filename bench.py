@@ -148,9 +148,11 @@ class ClockSampler:
 
 
 def flash_traffic_from_profile():
-    """DRAM bytes per flash_fwd launch from the committed ncu summary, if it was taken
-    on the current kernel source (its sha256 is recorded there); else None."""
-    path = os.path.join(ROOT, "profiles", "flash_fwd_long_prefill_kv.md")
+    """DRAM bytes per flash_fwd-kind launch (dram__bytes_read + dram__bytes_write of one
+    step's flash launches, from the committed single-pass ncu capture, divided by the
+    launches per step), if that capture was taken on the current kernel source (its
+    sha256 is recorded there); else None."""
+    path = os.path.join(ROOT, "profiles", "flash_fwd_long_step.md")
     src = os.path.join(ROOT, "paper_2607_15865_gb300", "csrc", "flash_fwd.cu")
     if not os.path.exists(path):
         return None
@@ -163,8 +165,8 @@ def flash_traffic_from_profile():
     if kv.get("kernel_source_sha256_16") != sha:
         return None
     try:
-        return float(kv["dram_bytes_per_launch_full_size"])
-    except (KeyError, ValueError):
+        return float(kv["dram_bytes_per_step_full_size"]) / int(kv["flash_launches_per_step"])
+    except (KeyError, ValueError, ZeroDivisionError):
         return None
 
 
@@ -502,19 +504,67 @@ def run_sweep(args):
     return 0
 
 
+# ----------------------------------------------------------------------------- one stage (profiling)
+
+
+def run_stage(args):
+    """Runs one stage of the long-context workload --warmup + --reps times on random
+    device inputs (no timing, no JSON line): the launch pattern that profiler captures
+    of a single kernel use.  --hist / --chunk override the stage's sizes."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.attention import Attention
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    st = STAGES[args.stage]
+    hist = st["hist"] if args.hist is None else args.hist
+    chunk = st["chunk"] if args.chunk is None else args.chunk
+    g = torch.Generator(device=dev).manual_seed(3)
+
+    def rnd(*shape):
+        return (torch.randn(*shape, device=dev, generator=g) * 0.0884).to(torch.bfloat16)
+
+    attn = Attention.for_shape(S)
+    kc = rnd(S.batch, S.n_kv_heads, S.max_len, S.head_dim)
+    vc = rnd(S.batch, S.n_kv_heads, S.max_len, S.head_dim)
+    q = rnd(S.batch, chunk, S.n_q_heads, S.head_dim)
+    k = rnd(S.batch, chunk, S.n_kv_heads, S.head_dim)
+    v = rnd(S.batch, chunk, S.n_kv_heads, S.head_dim)
+    out = torch.empty_like(q)
+    hl = torch.full((S.batch,), hist, dtype=torch.int32, device=dev)
+    for _ in range(args.warmup + args.reps):
+        if args.stage == "decode":
+            attn.decode(q, k, v, hl, kc, vc, out)
+        else:
+            attn.prefill_kv(q, k, v, hist, kc, vc, out)
+    torch.cuda.synchronize()
+    flags = attn.device_error()
+    attn.close()
+    print(f"stage {args.stage} hist {hist} chunk {chunk}: {args.warmup} + {args.reps} calls, device error word {flags}")
+    return 0 if flags == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--cpu-rows", type=int, default=192, help="prefill_kv rows in the oracle's timed sample")
+    ap.add_argument("--cpu-rows", type=int, default=1536, help="prefill_kv rows in the oracle's timed sample")
     ap.add_argument("--ref-rows", type=int, default=48, help="prefill_kv rows per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="time every configuration's stage instead (table to --sweep-out)")
     ap.add_argument("--sweep-out", default="sweep.json")
     ap.add_argument("--sweep-reps", type=int, default=20)
+    ap.add_argument("--stage", choices=tuple(STAGES), help="run only this stage (for profiler captures)")
+    ap.add_argument("--reps", type=int, default=2)
+    ap.add_argument("--hist", type=int)
+    ap.add_argument("--chunk", type=int)
     args = ap.parse_args()
+    if args.stage:  # no timing in this mode
+        return run_stage(args)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
