@@ -93,6 +93,22 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
 
 
+def max_over_ranks(x: float, dist, device) -> float:
+    """The maximum of x over all ranks (x itself without a process group)."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tflops(world: int, ms: float) -> float:
+    """Whole-job throughput: each of `world` ranks ran one replica of the step (weak
+    scaling, no exchange); the slowest rank's step time counts."""
+    return world * STEP_FLOPS / (ms * 1e-3) / 1e12
+
+
 def make_inputs():
     """Seeded host inputs of the step (bf16 bit patterns)."""
     data = {}
@@ -304,11 +320,7 @@ def run_ours(args):
     step_ms = [ev[i][0].elapsed_time(ev[i][3]) for i in range(K)]
     stage_ms = {name: sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(K)) / K
                 for j, name in enumerate(STAGES)}
-    ms = sum(step_ms) / K
-    if dist is not None:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(sum(step_ms) / K, dist, dev)
     if attn.device_error() != 0:
         raise RuntimeError("device error word set during the timed region")
 
@@ -331,11 +343,7 @@ def run_ours(args):
         e2e_ev[i][1].record(stream)
     torch.cuda.synchronize()
     clocks = sampler.stop()
-    e2e_ms = sum(a.elapsed_time(b) for a, b in e2e_ev) / K
-    if dist is not None:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in e2e_ev) / K, dist, dev)
 
     # ------------------------------------------------------------ parity of the timed outputs + CPU baseline
     result = {}
@@ -359,7 +367,7 @@ def run_ours(args):
             cpu = {"value": f_cpu / t_cpu / 1e12, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
                    "sample": (f"{args.cpu_rows} prefill_kv rows + {max(1, args.cpu_rows // 4)} prefill rows + "
                               f"{S.n_q_heads} decode rows of the step, single-threaded, {t_cpu:.1f} s")}
-        value = world * STEP_FLOPS / (ms * 1e-3) / 1e12
+        value = job_tflops(world, ms)
         flash_ms = kern["flash_fwd"][0]
         flash_n = kern["flash_fwd"][1]
         flash_flops = (FLOPS["prefill"] + FLOPS["prefill_kv"]) * K
@@ -392,7 +400,7 @@ def run_ours(args):
             "stages": stages,
             "kernels_ms_per_step": {k: v[0] / K for k, v in kern.items()},
             "cpu_baseline": cpu,
-            "e2e": {"value": world * STEP_FLOPS / (e2e_ms * 1e-3) / 1e12, "unit": "TFLOP/s",
+            "e2e": {"value": job_tflops(world, e2e_ms), "unit": "TFLOP/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
             "gpu_launches": launches,
             "clocks": clocks,
