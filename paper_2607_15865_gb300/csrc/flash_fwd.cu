@@ -366,23 +366,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             int items = 0;
             bool ok = true;
             // The tensor core holds almost no queue of MMAs, so every cycle this thread spends
-            // between two MMAs -- a barrier wait even when it is already satisfied costs about
-            // 60 -- is a cycle the tensor core idles.  So the barriers of the next group are
-            // tested (never blocking) while the current group still has MMAs to issue, and a
-            // group only blocks on a barrier that such a test did not find complete.
+            // between two MMAs is a cycle the tensor core idles: descriptors are precomputed
+            // words plus constants, and each KV step waits on as few barriers as it can (the
+            // V tile once for both query tiles).
             // Descriptor low words of the operand tiles; a K step adds a constant to them.
             constexpr uint32_t kHi = desc_hi_sw128(1024);
             const uint32_t q_lo0 = desc_lo_sw128(base + L::OFF_Q, 16);
             const uint32_t k_lo0 = desc_lo_sw128(base + L::OFF_K, 16);
             const uint32_t v_lo0 = desc_lo_sw128(base + L::OFF_V, L::CHUNK);
-            auto issue_s = [&](int t, uint32_t slot, auto&& mid) {
+            auto issue_s = [&](int t, uint32_t slot) {
                 const uint32_t a_lo = q_lo0 + t * (L::Q_TILE >> 4);
                 const uint32_t b_lo = k_lo0 + slot * (L::KV_TILE >> 4);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t c = ((kk >> 2) * L::CHUNK + (kk & 3) * 32) >> 4;
                     umma_ss_w(tmem + t * BN, a_lo + c, kHi, b_lo + c, kHi, kIdS, kk > 0 ? 1u : 0u);
-                    if (kk == D / 16 - 3) mid();
                 }
                 umma_commit(bar(B_SFULL0 + t));
             };
@@ -394,18 +392,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                               (!first || kk > 0) ? 1u : 0u);
             };
             // P_t of the previous KV tile in TMEM, and O_t free when it is the unit's first PV
-            auto wait_p = [&](int t, bool first, bool tested) -> bool {
-                if (!tested && !mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag)) return false;
+            auto wait_p = [&](int t, bool first) -> bool {
+                if (!mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag)) return false;
                 ++p_cnt[t];
                 if (first && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag))
                     return false;
                 return true;
             };
             uint32_t kslot = 0, vslot = 0;  // kvc % KS and the V slot of the previous KV tile
-            bool k_tested = false;          // KFULL of the next KV tile found complete early
-            bool pa_tested = false;         // PFULL_A of this KV tile found complete early
-            bool v_tested = false;          // VFULL of this KV tile found complete early
-            auto nothing = [] {};
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
                 const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 const Item& it = un.it;
@@ -415,21 +409,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 uint32_t prev = 0;
-                k_tested = pa_tested = v_tested = false;
                 for (int j = un.kv_lo; j < un.kv_hi && ok; ++j, ++kvc) {
                     const int ks = static_cast<int>(kslot);
-                    if (!k_tested && !mbar_wait(bar(B_KFULL0 + ks), (kvc / KS) & 1u, abort_flag)) {
+                    if (!mbar_wait(bar(B_KFULL0 + ks), (kvc / KS) & 1u, abort_flag)) {
                         ok = false;
                         break;
                     }
-                    k_tested = false;
                     tc_fence_after();
                     const bool pv_a = j > un.kv_lo && j - 1 < it.nkv(0), pv_b = j > un.kv_lo && j - 1 < it.nkv(1);
                     const bool s_a = j < it.nkv(0), s_b = j < it.nkv(1);
                     const bool first = j - 1 == un.kv_lo;
-                    bool v_ok = v_tested, pb_tested = false;
+                    bool v_ok = false;
                     if (pv_a) {
-                        if (!wait_p(0, first, pa_tested) ||
+                        if (!wait_p(0, first) ||
                             (!v_ok && !mbar_wait(bar(B_VFULL0 + vslot), (prev / VS) & 1u, abort_flag))) {
                             ok = false;
                             break;
@@ -438,10 +430,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tc_fence_after();
                         issue_pv(0, first, vslot);
                     }
-                    if (s_a)
-                        issue_s(0, kslot, [&] { if (pv_b) pb_tested = mbar_test(bar(B_PFULL0 + 1), p_cnt[1] & 1u); });
+                    if (s_a) issue_s(0, kslot);
                     if (pv_b) {
-                        if (!wait_p(1, first, pb_tested) ||
+                        if (!wait_p(1, first) ||
                             (!v_ok && !mbar_wait(bar(B_VFULL0 + vslot), (prev / VS) & 1u, abort_flag))) {
                             ok = false;
                             break;
@@ -451,17 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     const uint32_t knext = kslot + 1 == KS ? 0 : kslot + 1;
                     const uint32_t vnext = static_cast<uint32_t>(kvc % VS);  // V slot of this KV tile
-                    pa_tested = v_tested = false;
-                    if (s_b)
-                        issue_s(1, kslot, [&] {
-                            if (j + 1 < un.kv_hi) {
-                                k_tested = mbar_test(bar(B_KFULL0 + knext), ((kvc + 1) / KS) & 1u);
-                                v_tested = mbar_test(bar(B_VFULL0 + vnext), (kvc / VS) & 1u);
-                                if (s_a) pa_tested = mbar_test(bar(B_PFULL0), p_cnt[0] & 1u);
-                            }
-                        });
-                    else
-                        nothing();
+                    if (s_b) issue_s(1, kslot);
                     umma_commit(bar(B_KEMPTY0 + ks));
                     if (j > un.kv_lo) umma_commit(bar(B_VEMPTY0 + vslot));
                     prev = kvc;
@@ -474,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
                     if (ok && un.kv_hi - 1 < it.nkv(t)) {
-                        if (!wait_p(t, un.kv_hi - 1 == un.kv_lo, false)) {
+                        if (!wait_p(t, un.kv_hi - 1 == un.kv_lo)) {
                             ok = false;
                             break;
                         }
