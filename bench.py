@@ -16,6 +16,8 @@ e2e       the same metric through the same C-ABI calls with host buffers: every
           (copies on their own streams, overlapping the neighbouring steps' compute).
 roofline  the dominant kernel (flash_fwd) against the measured bf16 tensor peak.
 stages    per-stage times; prefill stages in TFLOP/s, decode in HBM GB/s.
+          (value comes from a pass with one event pair per step; stages, per-kernel
+          times and the roofline from a second, instrumented pass over the same steps.)
 cpu_baseline  the CPU oracle on a bounded row sample of the same step.
 
 --impl reference times the CPU oracle (the reference arm of this path) instead.
@@ -295,16 +297,33 @@ def run_ours(args):
         raise RuntimeError("device error word set during warm-up")
 
     # ------------------------------------------------------------ timed region (device-resident inputs)
+    # Loop A times the step with one event pair per step and nothing else inside it: the
+    # headline value.  Loop B repeats the same K steps with an event pair around every
+    # stage and the library's own pair around every kernel launch (its kernel timing),
+    # for the per-stage times and the roofline of the dominant kernel.  (Those 16 event
+    # records per step cost 1-2% of the step, which is why they stay out of loop A.)
     K = args.steps
+    ev_a = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
-    attn.timing_read()
-    attn.timing_enable(8 * K)
     sampler = ClockSampler(local_rank)
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
     sampler.start()
     time.sleep(0.3)  # let the sampler start before the GPU gets busy
+    for i in range(K):
+        l2_flush()
+        ev_a[i][0].record(stream)
+        step()
+        ev_a[i][1].record(stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev_a]
+    ms = max_over_ranks(sum(step_ms) / K, dist, dev)
+
+    attn.timing_read()
+    attn.timing_enable(8 * K)
     for i in range(K):
         l2_flush()
         ev[i][0].record(stream)
@@ -315,14 +334,10 @@ def run_ours(args):
         attn.decode(*d["decode"], hist_dec, kc, vc, out=outs["decode"], stream=stream)
         ev[i][3].record(stream)
     torch.cuda.synchronize()
-    if dist is not None:
-        dist.barrier()
     kern = attn.timing_read()
     attn.timing_enable(0)
-    step_ms = [ev[i][0].elapsed_time(ev[i][3]) for i in range(K)]
     stage_ms = {name: sum(ev[i][j].elapsed_time(ev[i][j + 1]) for i in range(K)) / K
                 for j, name in enumerate(STAGES)}
-    ms = max_over_ranks(sum(step_ms) / K, dist, dev)
     if attn.device_error() != 0:
         raise RuntimeError("device error word set during the timed region")
 
