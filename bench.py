@@ -535,7 +535,29 @@ def run_sweep(args):
                 attn.decode(q, k, v, hl, kc, vc, out)
             ms = time_calls(call, args.sweep_reps)
             gbs = decode_bytes(sh, hist) / (ms * 1e-3) / 1e9
-            rows.append({"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+            # the same step replayed from a CUDA graph (one graph per cache pair): what a
+            # serving loop that captures its decode step sees
+            graphs = []
+            for kc, vc in caches:
+                attn.decode(q, k, v, hl, kc, vc, out)  # tensor maps built outside the capture
+                gr = torch.cuda.CUDAGraph()
+                side = torch.cuda.Stream()
+                side.wait_stream(torch.cuda.current_stream())
+                with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+                    attn.decode(q, k, v, hl, kc, vc, out)
+                torch.cuda.current_stream().wait_stream(side)
+                graphs.append(gr)
+            torch.cuda.synchronize()
+            git = [0]
+
+            def replay():
+                graphs[git[0] % len(graphs)].replay()
+                git[0] += 1
+            ms_g = time_calls(replay, args.sweep_reps)
+            gbs_g = decode_bytes(sh, hist) / (ms_g * 1e-3) / 1e9
+            rows.append({"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm,
+                         "graph_ms": ms_g, "graph_GB/s": gbs_g})
+            del graphs
         attn.close()
     attn = Attention.for_shape(S)
     kc = rnd((1, 8, 32768, 128), gen)
@@ -552,6 +574,8 @@ def run_sweep(args):
     for r in rows:
         extra = f"{r['TFLOP/s']:8.1f} TFLOP/s {100*r['frac_tensor']:5.1f}%" if "TFLOP/s" in r else \
             f"{r['GB/s']:8.1f} GB/s    {100*r['frac_hbm']:5.1f}%"
+        if "graph_ms" in r:
+            extra += f"   (CUDA graph: {r['graph_ms']*1e3:6.1f} us {r['graph_GB/s']:7.1f} GB/s)"
         print(f"{r['config']:36s} {r['ms']*1e3:9.1f} us {extra}", file=sys.stderr)
     return 0
 
