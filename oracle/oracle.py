@@ -147,6 +147,26 @@ def append(shape, k, v, hist, k_cache, v_cache, lib=None):
                              _u16(v_cache)), "append")
 
 
+def attend_rows_parallel(shape, q, hist, k_cache, v_cache, rows, threads=None, lib=None):
+    """attend_rows on several host cores: the rows are cut into contiguous blocks and each
+    block is one call of the same C routine on its own thread (ctypes releases the GIL,
+    and the routine keeps all of its state on its own stack and heap).  Row by row the
+    arithmetic is that of attend_rows; only whole rows are distributed."""
+    from concurrent.futures import ThreadPoolExecutor
+    lib = lib or load()
+    r = np.ascontiguousarray(rows, dtype=np.int32).reshape(-1, 3)
+    n = max(1, min(int(threads or os.cpu_count() or 1), len(r)))
+    out = np.zeros((r.shape[0], shape.head_dim), np.uint16)
+    blocks = [ix for ix in np.array_split(np.arange(len(r)), n) if len(ix)]
+
+    def run(ix):
+        out[ix] = attend_rows(shape, q, hist, k_cache, v_cache, r[ix], lib=lib)
+
+    with ThreadPoolExecutor(max_workers=n) as ex:
+        list(ex.map(run, blocks))
+    return out
+
+
 def attend_rows(shape, q, hist, k_cache, v_cache, rows, lib=None):
     """Output rows for the (b, i, h) triples in ``rows`` over caches that already hold the chunk."""
     lib = lib or load()

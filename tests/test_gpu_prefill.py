@@ -155,3 +155,27 @@ def test_long_prefill_4096(torch):
 
 def test_long_prefill_kv_4096_over_28672(torch):
     check_full_size(torch, w.LONG, "long_pkv", w.LONG_PKV_HIST, w.LONG_PKV_CHUNK, n_pos=6, heads=10)
+
+
+def check_every_row(torch, shape, tag, hist, chunk):
+    """Every output row of a full-size stage against the oracle, run on all host cores."""
+    q, k, v = w.tokens(shape, tag, chunk)
+    kc, vc = w.cache(shape, tag, hist, fill="nan")
+    out, gk, gv = gpu_stage(torch, shape, q, k, v, hist, kc, vc)
+    rk, rv = kc.copy(), vc.copy()
+    O.append(shape, k, v, hist, rk, rv)
+    assert_cache(gk, gv, rk, rv, kc, vc, [(hist, hist + chunk)] * shape.batch, f"{tag} cache")
+    rows = np.array([(b, i, h) for b in range(shape.batch) for i in range(chunk) for h in range(shape.n_q_heads)],
+                    np.int32)
+    ref = O.attend_rows_parallel(shape, q, hist, rk, rv, rows).reshape(out.shape)
+    assert_out_close(out, ref, f"{tag} every row")
+
+
+@pytest.mark.slow
+def test_long_prefill_4096_every_row(torch):
+    check_every_row(torch, w.LONG, "long_prefill_all", 0, w.LONG_PREFILL)
+
+
+@pytest.mark.slow
+def test_long_prefill_kv_4096_over_28672_every_row(torch):
+    check_every_row(torch, w.LONG, "long_pkv_all", w.LONG_PKV_HIST, w.LONG_PKV_CHUNK)
