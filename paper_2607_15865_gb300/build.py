@@ -17,7 +17,11 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libattn_gb300.so")
-SOURCES = ["attn_api.cu", "rope_append.cu", "decode.cu", "decode_tc.cu", "flash_fwd.cu", "decode_noalloc.cu"]
+# (source, object name, extra nvcc flags): flash_fwd.cu is built twice, as the 2- and the
+# 3-stage V ring variant of K2.
+SOURCES = [("attn_api.cu", "attn_api", []), ("rope_append.cu", "rope_append", []), ("decode.cu", "decode", []),
+           ("decode_tc.cu", "decode_tc", []), ("flash_fwd.cu", "flash_fwd_v2", ["-DFLASH_V_STAGES=2"]),
+           ("flash_fwd.cu", "flash_fwd_v3", ["-DFLASH_V_STAGES=3"]), ("decode_noalloc.cu", "decode_noalloc", [])]
 HEADERS = ["internal.h", "sm100_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -34,19 +38,20 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def _compile(src: str, verbose_ptxas: bool) -> str:
-    obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+def _compile(unit, verbose_ptxas: bool) -> str:
+    src, name, flags = unit
+    obj = os.path.join(BUILD, name + ".o")
     deps = [os.path.join(CSRC, src)] + [os.path.join(CSRC, h) for h in HEADERS] + [
         os.path.join(ROOT, "include", "attn.h")]
     if not _stale(obj, deps) and not verbose_ptxas:
         return obj
     cmd = [_nvcc(), *ARCH, "-lineinfo", "-O3", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
-           "-I", os.path.join(ROOT, "include"), "-c", os.path.join(CSRC, src), "-o", obj + ".tmp"]
+           *flags, "-I", os.path.join(ROOT, "include"), "-c", os.path.join(CSRC, src), "-o", obj + ".tmp"]
     if verbose_ptxas:
         cmd[1:1] = ["-Xptxas", "-v"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
-        raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+        raise RuntimeError(f"nvcc failed for {name} ({src}):\n{r.stdout}\n{r.stderr}")
     if verbose_ptxas:
         sys.stderr.write(r.stderr)
     os.replace(obj + ".tmp", obj)
@@ -57,7 +62,7 @@ def build(verbose_ptxas: bool = False) -> str:
     """Compile every CUDA source and link the shared library; returns its path."""
     os.makedirs(BUILD, exist_ok=True)
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(lambda s: _compile(s, verbose_ptxas), SOURCES))
+        objs = list(ex.map(lambda u: _compile(u, verbose_ptxas), SOURCES))
     if _stale(LIB, objs):
         tmp = LIB + f".tmp{os.getpid()}"
         r = subprocess.run([_nvcc(), *ARCH, "-shared", "-o", tmp, *objs], capture_output=True, text=True)

@@ -18,7 +18,7 @@
 //                     q [B,S,Hq,D] and the K ring; lane 1: the V ring), warp 9:
 //                     tcgen05 issuer, warps 10-11 idle.  WG2 gives registers to
 //                     the softmax warpgroups (setmaxnreg 56 / 224 of 168 at launch).
-// K tiles (128 keys, 2-stage ring) and V tiles (3-stage ring) use the 128-byte
+// K tiles (128 keys, 2-stage ring) and V tiles (2- or 3-stage ring) use the 128-byte
 // swizzle; rows past hist+chunk are zero-filled by the map bounds, never read.
 // Per KV tile j the issuer runs PV_A(j-1), S_A(j), PV_B(j-1), S_B(j).
 // TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [256+D,256+2D).
@@ -52,8 +52,16 @@ constexpr int kThreads = 384;
 constexpr int kWarpTma = 8;
 constexpr int kWarpMma = 9;
 constexpr uint32_t kTmemCols = 512;
-constexpr int KS = 2;  // K ring stages
-constexpr int VS = 3;  // V ring stages
+// This file is compiled twice (FLASH_V_STAGES = 2 and 3, entry points suffixed _v2 /
+// _v3).  Three V stages suit long KV walks; with two, the freed 32 KB stage the epilogue's
+// output so that each warp store writes 4 whole 128-byte rows instead of 16 bytes of 32
+// rows 10 KB apart -- worth it where work items are short (the causal prefill).
+#ifndef FLASH_V_STAGES
+#define FLASH_V_STAGES 3
+#endif
+constexpr int KS = 2;                      // K ring stages
+constexpr int VS = FLASH_V_STAGES;         // V ring stages
+constexpr bool kStagedEpilogue = VS == 2;  // epilogue through shared memory
 // Register budgets: 168 per thread at launch (65536 / 384, rounded down to 8);
 // WG2 gives back 112 per thread, the two softmax warpgroups take 56 each.
 constexpr int kLaunchRegs = 168;
@@ -63,9 +71,9 @@ static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "regis
 
 enum Bar {
     B_QFULL, B_QREADY, B_QEMPTY,
-    B_KFULL0, B_KFULL1, B_KEMPTY0, B_KEMPTY1,
-    B_VFULL0, B_VFULL1, B_VFULL2, B_VEMPTY0, B_VEMPTY1, B_VEMPTY2,
-    B_SFULL0, B_SFULL1, B_PFULL0, B_PFULL1,
+    B_KFULL0, B_KEMPTY0 = B_KFULL0 + KS,
+    B_VFULL0 = B_KEMPTY0 + KS, B_VEMPTY0 = B_VFULL0 + VS,
+    B_SFULL0 = B_VEMPTY0 + VS, B_SFULL1, B_PFULL0, B_PFULL1,
     B_OFULL0, B_OFULL1, B_OEMPTY0, B_OEMPTY1,
     B_DRAIN, NBAR
 };
@@ -79,7 +87,9 @@ struct Layout {
     static constexpr int OFF_Q = 0;                      // q tiles A, B
     static constexpr int OFF_K = OFF_Q + 2 * Q_TILE;     // K ring
     static constexpr int OFF_V = OFF_K + KS * KV_TILE;   // V ring
-    static constexpr int OFF_BAR = OFF_V + VS * KV_TILE;
+    static constexpr int OFF_STAGE = OFF_V + VS * KV_TILE;  // epilogue staging, 4 KB per softmax warp
+    static constexpr int STAGE_WARP = 32 * 128;             // 32 rows x 64 bf16 columns
+    static constexpr int OFF_BAR = OFF_STAGE + (kStagedEpilogue ? 8 * STAGE_WARP : 0);
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
     static constexpr int OFF_ABORT = OFF_TMEM + 8;
     static constexpr int BYTES = OFF_ABORT + 8;
@@ -603,29 +613,64 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 ++o_cnt;
                 tc_fence_after();
-                const float inv_l = un.piece < 0 ? 1.f / l_run : 1.f;
-                uint16_t* orow = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D;
-                float* prow_o = ws_o + prow * D;
+                if (un.piece < 0 && kStagedEpilogue) {
+                    // O_T / l -> bf16 through this warp's staging area, 64 columns at a time: each
+                    // thread writes its row there, then the warp stores 4 rows (512 contiguous-row
+                    // bytes) per instruction instead of 32 rows 10 KB apart.
+                    const float inv_l = 1.f / l_run;
+                    const int lane = threadIdx.x & 31, r0 = row & ~31;
+                    uint8_t* stage = gbase + L::OFF_STAGE + warp * L::STAGE_WARP;
+                    uint16_t* obase = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + r0) * Hq + it.h) * D;
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t o[32];
-                    tmem_ld32(o_col + 32 * c, o);
-                    tmem_wait_ld();
-                    if (row < it.rows(t)) {
-                        const float* f = reinterpret_cast<const float*>(o);
-                        if (un.piece < 0) {
+                    for (int c2 = 0; c2 < D / 64; ++c2) {
+                        uint32_t o[2][32];
+                        tmem_ld32(o_col + 64 * c2, o[0]);
+                        tmem_ld32(o_col + 64 * c2 + 32, o[1]);
+                        tmem_wait_ld();
 #pragma unroll
-                            for (int v4 = 0; v4 < 4; ++v4)
-                                *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
-                                    pack_bf16x2(f[8 * v4 + 0] * inv_l, f[8 * v4 + 1] * inv_l),
-                                    pack_bf16x2(f[8 * v4 + 2] * inv_l, f[8 * v4 + 3] * inv_l),
-                                    pack_bf16x2(f[8 * v4 + 4] * inv_l, f[8 * v4 + 5] * inv_l),
-                                    pack_bf16x2(f[8 * v4 + 6] * inv_l, f[8 * v4 + 7] * inv_l));
-                        } else {
+                        for (int ch = 0; ch < 8; ++ch) {  // 16-byte chunks, swizzled by the row
+                            const float* f = reinterpret_cast<const float*>(o[ch >> 2]) + (ch & 3) * 8;
+                            *reinterpret_cast<uint4*>(stage + lane * 128 + ((ch ^ (lane & 7)) << 4)) = make_uint4(
+                                pack_bf16x2(f[0] * inv_l, f[1] * inv_l), pack_bf16x2(f[2] * inv_l, f[3] * inv_l),
+                                pack_bf16x2(f[4] * inv_l, f[5] * inv_l), pack_bf16x2(f[6] * inv_l, f[7] * inv_l));
+                        }
+                        __syncwarp();
 #pragma unroll
-                            for (int v4 = 0; v4 < 8; ++v4)
-                                *reinterpret_cast<float4*>(prow_o + 32 * c + 4 * v4) =
-                                    make_float4(f[4 * v4], f[4 * v4 + 1], f[4 * v4 + 2], f[4 * v4 + 3]);
+                        for (int i = 0; i < 8; ++i) {
+                            const int rr = 4 * i + (lane >> 3), ch = lane & 7;
+                            const uint4 u = *reinterpret_cast<const uint4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
+                            if (r0 + rr < it.rows(t))
+                                *reinterpret_cast<uint4*>(obase + static_cast<size_t>(rr) * Hq * D + 64 * c2 + 8 * ch) = u;
+                        }
+                        __syncwarp();
+                    }
+                } else {
+                    // O_T / l -> bf16 -> out straight from each thread's row, or for a piece the
+                    // unnormalised O_T
+                    const float inv_l = un.piece < 0 ? 1.f / l_run : 1.f;
+                    uint16_t* orow = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D;
+                    float* prow_o = ws_o + prow * D;
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(o_col + 32 * c, o);
+                        tmem_wait_ld();
+                        if (row < it.rows(t)) {
+                            const float* f = reinterpret_cast<const float*>(o);
+                            if (un.piece < 0) {
+#pragma unroll
+                                for (int v4 = 0; v4 < 4; ++v4)
+                                    *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
+                                        pack_bf16x2(f[8 * v4 + 0] * inv_l, f[8 * v4 + 1] * inv_l),
+                                        pack_bf16x2(f[8 * v4 + 2] * inv_l, f[8 * v4 + 3] * inv_l),
+                                        pack_bf16x2(f[8 * v4 + 4] * inv_l, f[8 * v4 + 5] * inv_l),
+                                        pack_bf16x2(f[8 * v4 + 6] * inv_l, f[8 * v4 + 7] * inv_l));
+                            } else {
+#pragma unroll
+                                for (int v4 = 0; v4 < 8; ++v4)
+                                    *reinterpret_cast<float4*>(prow_o + 32 * c + 4 * v4) =
+                                        make_float4(f[4 * v4], f[4 * v4 + 1], f[4 * v4 + 2], f[4 * v4 + 3]);
+                            }
                         }
                     }
                 }
@@ -775,12 +820,18 @@ cudaError_t configure_d() {
 
 }  // namespace
 
-cudaError_t configure_flash_fwd() {
+#if FLASH_V_STAGES == 2
+#define FLASH_ENTRY(name) name##_v2
+#else
+#define FLASH_ENTRY(name) name##_v3
+#endif
+
+cudaError_t FLASH_ENTRY(configure_flash_fwd)() {
     const cudaError_t e = configure_d<128>();
     return e != cudaSuccess ? e : configure_d<64>();
 }
 
-cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+cudaError_t FLASH_ENTRY(launch_flash_fwd)(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
                              const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                              cudaStream_t st, int* n_launched) {
     if (s.head_dim == 128)
