@@ -17,11 +17,10 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libattn_gb300.so")
-# (source, object name, extra nvcc flags): flash_fwd.cu is built twice, as the 2- and the
-# 3-stage V ring variant of K2.
+# (source, object name, extra nvcc flags)
 SOURCES = [("attn_api.cu", "attn_api", []), ("rope_append.cu", "rope_append", []), ("decode.cu", "decode", []),
-           ("decode_tc.cu", "decode_tc", []), ("flash_fwd.cu", "flash_fwd_v2", ["-DFLASH_V_STAGES=2"]),
-           ("flash_fwd.cu", "flash_fwd_v3", ["-DFLASH_V_STAGES=3"]), ("decode_noalloc.cu", "decode_noalloc", [])]
+           ("decode_tc.cu", "decode_tc", []), ("flash_fwd.cu", "flash_fwd", []),
+           ("decode_noalloc.cu", "decode_noalloc", [])]
 HEADERS = ["internal.h", "sm100_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -148,9 +148,8 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
     e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&](int* n) {
-        const auto launch = attn::flash_fwd_use_v2(hist, chunk) ? attn::launch_flash_fwd_v2 : attn::launch_flash_fwd_v3;
-        return launch(s, maps, hist, chunk, c->d_cos_t, c->d_sin_t, out, c->d_flash_o, c->d_flash_ml, c->d_err,
-                      c->num_sms, st, n);
+        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos_t, c->d_sin_t, out, c->d_flash_o, c->d_flash_ml,
+                                      c->d_err, c->num_sms, st, n);
     });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
     return ATTN_OK;
@@ -188,8 +187,7 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
         return cuda_fail(e == cudaSuccess ? cudaErrorNotSupported : e, "cuTensorMapEncodeTiled entry point");
     }
     c->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    e = attn::configure_flash_fwd_v2();
-    if (e == cudaSuccess) e = attn::configure_flash_fwd_v3();
+    e = attn::configure_flash_fwd();
     if (e == cudaSuccess) e = attn::configure_decode();
     if (e == cudaSuccess) e = attn::configure_decode_tc();
     if (e != cudaSuccess) {

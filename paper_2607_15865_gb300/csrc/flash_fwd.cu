@@ -15,10 +15,10 @@
 //   WG0 (warps 0-3)   softmax + epilogue of tile A (one thread per row = TMEM lane)
 //   WG1 (warps 4-7)   softmax + epilogue of tile B
 //   WG2 (warps 8-11)  warp 8: TMA producer (lane 0: q tiles from a 4-D map of
-//                     q [B,S,Hq,D] and the K ring; lane 1: the V ring), warp 9:
-//                     tcgen05 issuer, warps 10-11 idle.  WG2 gives registers to
-//                     the softmax warpgroups (setmaxnreg 56 / 224 of 168 at launch).
-// K tiles (128 keys, 2-stage ring) and V tiles (2- or 3-stage ring) use the 128-byte
+//                     q [B,S,Hq,D] and the K/V group ring), warp 9: tcgen05
+//                     issuer, warps 10-11 idle.  WG2 gives registers to
+//                     the softmax warpgroups (setmaxnreg 96 / 200 of 168 at launch).
+// K and V tiles (128 keys, a 2-stage ring of K(j)/V(j-1) groups) use the 128-byte
 // swizzle; rows past hist+chunk are zero-filled by the map bounds, never read.
 // Per KV tile j the issuer runs PV_A(j-1), S_A(j), PV_B(j-1), S_B(j).
 // TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [256+D,256+2D).
@@ -26,8 +26,8 @@
 // MMA from TMEM, so the two warpgroups ping-pong: while one turns its scores into
 // P, the tensor core runs the other tile's MMAs.  A commit covers every earlier
 // MMA of the issuing thread, so "S_T(j) complete" implies "PV_T(j-1) complete":
-// the softmax warpgroup may rescale O_T right away.  O is rescaled lazily (only
-// when the running max grows by more than 2^8, exact in value).
+// the softmax warpgroup may rescale O_T before it hands P over.  O is rescaled lazily
+// (only when the running max grows by more than 2^8, exact in value).
 // Per row: RoPE of the q row in shared memory before the first MMA (cos/sin
 // gathered by position from pair-major copies of the tables, Section 4.6.2, float
 // arithmetic and bf16 rounding as K1),
@@ -52,28 +52,27 @@ constexpr int kThreads = 384;
 constexpr int kWarpTma = 8;
 constexpr int kWarpMma = 9;
 constexpr uint32_t kTmemCols = 512;
-// This file is compiled twice (FLASH_V_STAGES = 2 and 3, entry points suffixed _v2 /
-// _v3).  Three V stages suit long KV walks; with two, the freed 32 KB stage the epilogue's
-// output so that each warp store writes 4 whole 128-byte rows instead of 16 bytes of 32
-// rows 10 KB apart -- worth it where work items are short (the causal prefill).
-#ifndef FLASH_V_STAGES
-#define FLASH_V_STAGES 3
-#endif
-constexpr int KS = 2;                      // K ring stages
-constexpr int VS = FLASH_V_STAGES;         // V ring stages
-constexpr bool kStagedEpilogue = VS == 2;  // epilogue through shared memory
+// K/V ring of "groups": group j holds K tile j and V tile j-1, the operands of KV step
+// j (S(j) and PV(j-1)), so the issuer waits on one barrier and releases one slot per
+// step -- each satisfied wait or extra commit of the issuing thread idles the tensor
+// core for about 100 cycles.  Two 64 KB slots, and 32 KB to stage the epilogue's output
+// (each warp store then writes 4 whole 128-byte rows instead of 16 bytes of 32 rows
+// 10 KB apart).
+constexpr int GS = 2;
 // Register budgets: 168 per thread at launch (65536 / 384, rounded down to 8);
-// WG2 gives back 112 per thread, the two softmax warpgroups take 56 each.
+// WG2 gives back 72 per thread, the two softmax warpgroups take 32 each.  The MMA
+// issuer must not spill: a local-memory reload between two MMA groups idles the
+// tensor core (56 for WG2 cost 8% of the prefill_kv time against 96), and at 200 the
+// softmax fits because O is rescaled after its scores have been consumed.
 constexpr int kLaunchRegs = 168;
-constexpr uint32_t kRegsLow = 56;
-constexpr uint32_t kRegsHigh = 224;
+constexpr uint32_t kRegsLow = 96;
+constexpr uint32_t kRegsHigh = 200;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split exceeds the launch total");
 
 enum Bar {
     B_QFULL, B_QREADY, B_QEMPTY,
-    B_KFULL0, B_KEMPTY0 = B_KFULL0 + KS,
-    B_VFULL0 = B_KEMPTY0 + KS, B_VEMPTY0 = B_VFULL0 + VS,
-    B_SFULL0 = B_VEMPTY0 + VS, B_SFULL1, B_PFULL0, B_PFULL1,
+    B_GFULL0, B_GEMPTY0 = B_GFULL0 + GS,
+    B_SFULL0 = B_GEMPTY0 + GS, B_SFULL1, B_PFULL0, B_PFULL1,
     B_OFULL0, B_OFULL1, B_OEMPTY0, B_OEMPTY1,
     B_DRAIN, NBAR
 };
@@ -85,11 +84,11 @@ struct Layout {
     static constexpr int Q_TILE = DCH * CHUNK;
     static constexpr int KV_TILE = DCH * CHUNK;
     static constexpr int OFF_Q = 0;                      // q tiles A, B
-    static constexpr int OFF_K = OFF_Q + 2 * Q_TILE;     // K ring
-    static constexpr int OFF_V = OFF_K + KS * KV_TILE;   // V ring
-    static constexpr int OFF_STAGE = OFF_V + VS * KV_TILE;  // epilogue staging, 4 KB per softmax warp
+    static constexpr int OFF_G = OFF_Q + 2 * Q_TILE;     // group ring: slot = K tile, V tile
+    static constexpr int G_SLOT = 2 * KV_TILE;
+    static constexpr int OFF_STAGE = OFF_G + GS * G_SLOT;  // epilogue staging, 4 KB per softmax warp
     static constexpr int STAGE_WARP = 32 * 128;             // 32 rows x 64 bf16 columns
-    static constexpr int OFF_BAR = OFF_STAGE + (kStagedEpilogue ? 8 * STAGE_WARP : 0);
+    static constexpr int OFF_BAR = OFF_STAGE + 8 * STAGE_WARP;
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
     static constexpr int OFF_ABORT = OFF_TMEM + 8;
     static constexpr int BYTES = OFF_ABORT + 8;
@@ -267,13 +266,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(bar(B_QFULL), 1);
         mbar_init(bar(B_QREADY), 2 * BM);
         mbar_init(bar(B_QEMPTY), 1);
-        for (int st = 0; st < KS; ++st) {
-            mbar_init(bar(B_KFULL0 + st), 1);
-            mbar_init(bar(B_KEMPTY0 + st), 1);
-        }
-        for (int st = 0; st < VS; ++st) {
-            mbar_init(bar(B_VFULL0 + st), 1);
-            mbar_init(bar(B_VEMPTY0 + st), 1);
+        for (int st = 0; st < GS; ++st) {
+            mbar_init(bar(B_GFULL0 + st), 1);
+            mbar_init(bar(B_GEMPTY0 + st), 1);
         }
         for (int t = 0; t < 2; ++t) {
             mbar_init(bar(B_SFULL0 + t), 1);
@@ -296,10 +291,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp >= 8) {
         warpgroup_reg_dec<kRegsLow>();
         if (warp == kWarpTma && lane == 0) {
-            // ---------------------------------------------------- q tiles and the K ring
+            // ---------------------------------------------------- q tiles and the group ring
+            // A unit of n KV tiles takes n + 1 groups: group j holds K(j) (j < kv_hi) and
+            // V(j-1) (j > kv_lo), the last one only the V the final PV reads.
             tma_prefetch_desc(&map_q);
             tma_prefetch_desc(&map_k);
-            uint32_t kc = 0;  // K tiles issued
+            tma_prefetch_desc(&map_v);
+            uint32_t gc = 0;  // groups issued
             int items = 0;
             bool ok = true;
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
@@ -318,17 +316,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     it.b, bar(B_QFULL));
                 ++items;
                 const int kv_row = it.b * Hkv + it.g;
-                for (int j = un.kv_lo; j < un.kv_hi; ++j, ++kc) {
-                    const int st = static_cast<int>(kc % KS);
-                    if (kc >= KS && !mbar_wait(bar(B_KEMPTY0 + st), (kc / KS - 1u) & 1u, abort_flag)) {
+                for (int j = un.kv_lo; j <= un.kv_hi; ++j, ++gc) {
+                    const int st = static_cast<int>(gc % GS);
+                    if (gc >= GS && !mbar_wait(bar(B_GEMPTY0 + st), (gc / GS - 1u) & 1u, abort_flag)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(bar(B_KFULL0 + st), L::KV_TILE);
+                    const bool has_k = j < un.kv_hi, has_v = j > un.kv_lo;
+                    const uint32_t slot = base + L::OFF_G + st * L::G_SLOT;
+                    mbar_arrive_expect_tx(bar(B_GFULL0 + st), (has_k ? L::KV_TILE : 0) + (has_v ? L::KV_TILE : 0));
+                    if (has_k) {
 #pragma unroll
-                    for (int c = 0; c < L::DCH; ++c)
-                        tma_load_3d(base + L::OFF_K + st * L::KV_TILE + c * L::CHUNK, &map_k, c * 64, j * BN, kv_row,
-                                    bar(B_KFULL0 + st));
+                        for (int c = 0; c < L::DCH; ++c)
+                            tma_load_3d(slot + c * L::CHUNK, &map_k, c * 64, j * BN, kv_row, bar(B_GFULL0 + st));
+                    }
+                    if (has_v) {
+#pragma unroll
+                        for (int c = 0; c < L::DCH; ++c)
+                            tma_load_3d(slot + L::KV_TILE + c * L::CHUNK, &map_v, c * 64, (j - 1) * BN, kv_row,
+                                        bar(B_GFULL0 + st));
+                    }
                 }
             }
             if (!ok) {
@@ -336,41 +343,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 atomicOr(err, kDevErrTimeout);
                 // every copy issued must land before the CTA may exit
                 if (items > 0) mbar_wait(bar(B_QFULL), static_cast<uint32_t>(items - 1) & 1u, nullptr);
-                for (uint32_t t = kc >= KS ? kc - KS : 0; t < kc; ++t)
-                    mbar_wait(bar(B_KFULL0 + static_cast<int>(t % KS)), (t / KS) & 1u, nullptr);
-            }
-        } else if (warp == kWarpTma && lane == 1) {
-            // ---------------------------------------------------- the V ring
-            tma_prefetch_desc(&map_v);
-            uint32_t vc = 0;  // V tiles issued
-            bool ok = true;
-            for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
-                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
-                const int kv_row = un.it.b * Hkv + un.it.g;
-                for (int j = un.kv_lo; j < un.kv_hi; ++j, ++vc) {
-                    const int st = static_cast<int>(vc % VS);
-                    if (vc >= VS && !mbar_wait(bar(B_VEMPTY0 + st), (vc / VS - 1u) & 1u, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    mbar_arrive_expect_tx(bar(B_VFULL0 + st), L::KV_TILE);
-#pragma unroll
-                    for (int c = 0; c < L::DCH; ++c)
-                        tma_load_3d(base + L::OFF_V + st * L::KV_TILE + c * L::CHUNK, &map_v, c * 64, j * BN, kv_row,
-                                    bar(B_VFULL0 + st));
-                }
-            }
-            if (!ok) {
-                *abort_flag = 1;
-                atomicOr(err, kDevErrTimeout);
-                for (uint32_t t = vc >= VS ? vc - VS : 0; t < vc; ++t)
-                    mbar_wait(bar(B_VFULL0 + static_cast<int>(t % VS)), (t / VS) & 1u, nullptr);
+                for (uint32_t t = gc >= GS ? gc - GS : 0; t < gc; ++t)
+                    mbar_wait(bar(B_GFULL0 + static_cast<int>(t % GS)), (t / GS) & 1u, nullptr);
             }
         } else if (warp == kWarpMma && lane == 0) {
             // ---------------------------------------------------- tcgen05 issuer
             constexpr uint32_t kIdS = idesc_bf16_f32(BM, BN, false, false);
             constexpr uint32_t kIdPV = idesc_bf16_f32(BM, D, false, true);
-            uint32_t kvc = 0;
+            uint32_t gc = 0;  // groups consumed
             uint32_t p_cnt[2] = {0u, 0u};  // P tiles consumed per query tile
             uint32_t o_cnt[2] = {0u, 0u};  // items whose O was handed to the epilogue
             int items = 0;
@@ -382,11 +362,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Descriptor low words of the operand tiles; a K step adds a constant to them.
             constexpr uint32_t kHi = desc_hi_sw128(1024);
             const uint32_t q_lo0 = desc_lo_sw128(base + L::OFF_Q, 16);
-            const uint32_t k_lo0 = desc_lo_sw128(base + L::OFF_K, 16);
-            const uint32_t v_lo0 = desc_lo_sw128(base + L::OFF_V, L::CHUNK);
+            const uint32_t k_lo0 = desc_lo_sw128(base + L::OFF_G, 16);
+            const uint32_t v_lo0 = desc_lo_sw128(base + L::OFF_G + L::KV_TILE, L::CHUNK);
             auto issue_s = [&](int t, uint32_t slot) {
                 const uint32_t a_lo = q_lo0 + t * (L::Q_TILE >> 4);
-                const uint32_t b_lo = k_lo0 + slot * (L::KV_TILE >> 4);
+                const uint32_t b_lo = k_lo0 + slot * (L::G_SLOT >> 4);
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t c = ((kk >> 2) * L::CHUNK + (kk & 3) * 32) >> 4;
@@ -394,8 +374,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 umma_commit(bar(B_SFULL0 + t));
             };
-            auto issue_pv = [&](int t, bool first, uint32_t vslot) {
-                const uint32_t b_lo = v_lo0 + vslot * (L::KV_TILE >> 4);
+            auto issue_pv = [&](int t, bool first, uint32_t slot) {
+                const uint32_t b_lo = v_lo0 + slot * (L::G_SLOT >> 4);
 #pragma unroll
                 for (int kk = 0; kk < BN / 16; ++kk)
                     umma_ts_w(tmem + L::TM_O + t * D, tmem + t * BN + kk * 8, b_lo + kk * ((16 * 128) >> 4), kHi, kIdPV,
@@ -409,7 +389,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     return false;
                 return true;
             };
-            uint32_t kslot = 0, vslot = 0;  // kvc % KS and the V slot of the previous KV tile
+            uint32_t gslot = 0;  // gc % GS
+            auto next_group = [&]() {
+                ++gc;
+                gslot = gslot + 1 == GS ? 0 : gslot + 1;
+            };
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
                 const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 const Item& it = un.it;
@@ -418,10 +402,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                uint32_t prev = 0;
-                for (int j = un.kv_lo; j < un.kv_hi && ok; ++j, ++kvc) {
-                    const int ks = static_cast<int>(kslot);
-                    if (!mbar_wait(bar(B_KFULL0 + ks), (kvc / KS) & 1u, abort_flag)) {
+                for (int j = un.kv_lo; j < un.kv_hi && ok; ++j) {
+                    // group j: K(j), and V(j-1) for the PV MMAs of the previous tile
+                    if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag)) {
                         ok = false;
                         break;
                     }
@@ -429,39 +412,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const bool pv_a = j > un.kv_lo && j - 1 < it.nkv(0), pv_b = j > un.kv_lo && j - 1 < it.nkv(1);
                     const bool s_a = j < it.nkv(0), s_b = j < it.nkv(1);
                     const bool first = j - 1 == un.kv_lo;
-                    bool v_ok = false;
                     if (pv_a) {
-                        if (!wait_p(0, first) ||
-                            (!v_ok && !mbar_wait(bar(B_VFULL0 + vslot), (prev / VS) & 1u, abort_flag))) {
+                        if (!wait_p(0, first)) {
                             ok = false;
                             break;
                         }
-                        v_ok = true;
                         tc_fence_after();
-                        issue_pv(0, first, vslot);
+                        issue_pv(0, first, gslot);
                     }
-                    if (s_a) issue_s(0, kslot);
+                    if (s_a) issue_s(0, gslot);
                     if (pv_b) {
-                        if (!wait_p(1, first) ||
-                            (!v_ok && !mbar_wait(bar(B_VFULL0 + vslot), (prev / VS) & 1u, abort_flag))) {
+                        if (!wait_p(1, first)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        issue_pv(1, first, vslot);
+                        issue_pv(1, first, gslot);
                     }
-                    const uint32_t knext = kslot + 1 == KS ? 0 : kslot + 1;
-                    const uint32_t vnext = static_cast<uint32_t>(kvc % VS);  // V slot of this KV tile
-                    if (s_b) issue_s(1, kslot);
-                    umma_commit(bar(B_KEMPTY0 + ks));
-                    if (j > un.kv_lo) umma_commit(bar(B_VEMPTY0 + vslot));
-                    prev = kvc;
-                    kslot = knext;
-                    vslot = vnext;
+                    if (s_b) issue_s(1, gslot);
+                    umma_commit(bar(B_GEMPTY0 + gslot));
+                    next_group();
                 }
                 if (!ok) break;
                 umma_commit(bar(B_QEMPTY));  // every S MMA of the unit is issued
-                if (!mbar_wait(bar(B_VFULL0 + vslot), (prev / VS) & 1u, abort_flag)) ok = false;
+                // the last group: V of the final tile
+                if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag)) ok = false;
+                tc_fence_after();
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
                     if (ok && un.kv_hi - 1 < it.nkv(t)) {
@@ -470,10 +446,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                             break;
                         }
                         tc_fence_after();
-                        issue_pv(t, un.kv_hi - 1 == un.kv_lo, vslot);
+                        issue_pv(t, un.kv_hi - 1 == un.kv_lo, gslot);
                     }
                 if (!ok) break;
-                umma_commit(bar(B_VEMPTY0 + vslot));
+                umma_commit(bar(B_GEMPTY0 + gslot));
+                next_group();
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
                     if (un.cnt(t) > 0) {
@@ -550,18 +527,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool move = m_cand > m_run + 8.f;  // always on the first tile
                 const float m_new = move ? m_cand : m_run;
                 const float alpha = move ? fast_exp2(m_run - m_new) : 1.f;
-                if (j > un.kv_lo && __any_sync(0xFFFFFFFFu, move)) {
-                    // O_T holds the sum through tile j-1 (PV_T(j-1) completed before S_T(j)).
-#pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        uint32_t o[32];
-                        tmem_ld32(o_col + 32 * c, o);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-                        tmem_st32(o_col + 32 * c, o);
-                    }
-                }
                 // P = 2^(s*scale - m) as bf16 pairs over the first 64 columns of S (keys 2c, 2c+1
                 // in column c), stored a quarter (16 columns) at a time; the scores are all in
                 // registers, so overwriting S is safe.  Row sums in independent accumulators.
@@ -589,6 +554,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float2 sum2a = make_float2(sum2[0].x + sum2[1].x, sum2[0].y + sum2[1].y);
                 const float2 sum2b = make_float2(sum2[2].x + sum2[3].x, sum2[2].y + sum2[3].y);
                 const float2 sum2t = make_float2(sum2a.x + sum2b.x, sum2a.y + sum2b.y);
+                if (j > un.kv_lo && __any_sync(0xFFFFFFFFu, move)) {
+                    // O_T holds the sum through tile j-1 (PV_T(j-1) completed before S_T(j)),
+                    // and PV_T(j) waits for this thread's arrive below.  Done after P, when the
+                    // scores no longer hold registers.
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t o[32];
+                        tmem_ld32(o_col + 32 * c, o);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+                        tmem_st32(o_col + 32 * c, o);
+                    }
+                }
                 tmem_wait_st();
                 l_run = l_run * alpha + (sum2t.x + sum2t.y);
                 m_run = m_new;
@@ -613,7 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 ++o_cnt;
                 tc_fence_after();
-                if (un.piece < 0 && kStagedEpilogue) {
+                if (un.piece < 0) {
                     // O_T / l -> bf16 through this warp's staging area, 64 columns at a time: each
                     // thread writes its row there, then the warp stores 4 rows (512 contiguous-row
                     // bytes) per instruction instead of 32 rows 10 KB apart.
@@ -820,18 +799,12 @@ cudaError_t configure_d() {
 
 }  // namespace
 
-#if FLASH_V_STAGES == 2
-#define FLASH_ENTRY(name) name##_v2
-#else
-#define FLASH_ENTRY(name) name##_v3
-#endif
-
-cudaError_t FLASH_ENTRY(configure_flash_fwd)() {
+cudaError_t configure_flash_fwd() {
     const cudaError_t e = configure_d<128>();
     return e != cudaSuccess ? e : configure_d<64>();
 }
 
-cudaError_t FLASH_ENTRY(launch_flash_fwd)(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
                              const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                              cudaStream_t st, int* n_launched) {
     if (s.head_dim == 128)

@@ -31,25 +31,15 @@ struct FlashMaps {
     CUtensorMap k;  // k_cache as 3-D {D, hist+chunk, B*Hkv}; box {64, 128, 1}
     CUtensorMap v;  // v_cache, same as k
 };
-// K2 is built twice from one source: _v3 keeps three V stages in its ring and stores the
-// output from registers (long KV walks); _v2 keeps two and stages the output through the
-// freed shared memory for coalesced stores (short walks: the causal prefill).  Results
-// are identical; flash_fwd_use_v2 picks one per call.
 // Raise the dynamic shared-memory limit of K2 on the current device (once per device).
-cudaError_t configure_flash_fwd_v2();
-cudaError_t configure_flash_fwd_v3();
+cudaError_t configure_flash_fwd();
 // Work is split across num_sms persistent CTAs; items of the last, partial round are
 // cut into KV pieces whose partials go to ws_o [num_sms*256, D] / ws_ml [num_sms*256, 2]
 // and are merged by a second kernel (then *n_launched = 2).
 // cos_t / sin_t: the RoPE tables pair-major, [D/2][max_len] (entry (j, p) at j * max_len + p).
-cudaError_t launch_flash_fwd_v2(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
-                                const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
-                                int num_sms, cudaStream_t st, int* n_launched);
-cudaError_t launch_flash_fwd_v3(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
-                                const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
-                                int num_sms, cudaStream_t st, int* n_launched);
-// True when the mean KV walk of a work item (query tile) is at most 64 tiles of 128 keys.
-inline bool flash_fwd_use_v2(int hist, int chunk) { return hist + chunk / 2 <= 64 * 128; }
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+                             const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
+                             cudaStream_t st, int* n_launched);
 
 // K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
 // with 64-key boxes (built once per cache pair).  K3 also rotates the new key and
