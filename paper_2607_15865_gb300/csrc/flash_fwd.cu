@@ -234,7 +234,8 @@ __device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint3
     const bool w = __all_sync(0xFFFFFFFFu, mbar_wait(qfull, parity, abort));
     if (w && row < rows) rope_row_smem<D>(qtile, row, tabs);
     fence_proxy_async_smem();
-    mbar_arrive(qready);
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(qready);
     return w;
 }
 
@@ -264,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         *abort_flag = 0;
         mbar_init(bar(B_QFULL), 1);
-        mbar_init(bar(B_QREADY), 2 * BM);
+        mbar_init(bar(B_QREADY), 2 * BM / 32);
         mbar_init(bar(B_QEMPTY), 1);
         for (int st = 0; st < GS; ++st) {
             mbar_init(bar(B_GFULL0 + st), 1);
@@ -272,9 +273,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int t = 0; t < 2; ++t) {
             mbar_init(bar(B_SFULL0 + t), 1);
-            mbar_init(bar(B_PFULL0 + t), BM);
+            mbar_init(bar(B_PFULL0 + t), BM / 32);  // one arrive per softmax warp
             mbar_init(bar(B_OFULL0 + t), 1);
-            mbar_init(bar(B_OEMPTY0 + t), BM);
+            mbar_init(bar(B_OEMPTY0 + t), BM / 32);
         }
         mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
@@ -572,7 +573,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 l_run = l_run * alpha + (sum2t.x + sum2t.y);
                 m_run = m_new;
                 tc_fence_before();
-                mbar_arrive(bar(B_PFULL0 + t));
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(B_PFULL0 + t));
             }
             if (!ok) break;
             // next unit's q rows (its loads overlap this unit's last MMAs)
@@ -658,7 +660,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ws_ml[prow * 2 + 1] = l_run;
                 }
                 tc_fence_before();
-                mbar_arrive(bar(B_OEMPTY0 + t));
+                __syncwarp();
+                if ((threadIdx.x & 31) == 0) mbar_arrive(bar(B_OEMPTY0 + t));
             } else if (un.piece >= 0 && row < it.rows(t)) {  // this piece holds no key of tile t
                 ws_ml[prow * 2 + 0] = -INFINITY;
                 ws_ml[prow * 2 + 1] = 0.f;
