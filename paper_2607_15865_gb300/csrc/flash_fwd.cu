@@ -10,7 +10,7 @@
 // with_history template, Section 4.2).
 //
 // Design.  A persistent CTA per SM walks a static list of work items sorted
-// longest-first.  An item is two 128-row query tiles (A, B) of one head, so each
+// longest-first, dealt out in rounds of alternating direction.  An item is two 128-row query tiles (A, B) of one head, so each
 // K/V tile is brought in once for 256 queries.  384 threads, three warpgroups:
 //   WG0 (warps 0-3)   softmax + epilogue of tile A (one thread per row = TMEM lane)
 //   WG1 (warps 4-7)   softmax + epilogue of tile B
@@ -170,6 +170,17 @@ __device__ __forceinline__ Unit decode_unit(int lin, int S, int H, int Hq, int G
     return u;
 }
 
+// Unit taken by a CTA in its round r = lin / gridDim.x.  Rounds alternate direction
+// (odd rounds reversed), so the CTA that took one of the longest units of a round takes
+// one of the shortest of the next: with items sorted longest-first this evens out the
+// CTAs' totals (causal prefill 4096, 40 heads: the slowest CTA walks 74 KV tiles instead
+// of 88).  The last, partial round keeps its order.  A bijection on [0, n_units).
+__device__ __forceinline__ int unit_of(int lin, int n_units) {
+    const int g = static_cast<int>(gridDim.x), r = lin / g;
+    if ((r & 1) == 0 || (r + 1) * g > n_units) return lin;
+    return r * g + (g - 1 - lin % g);
+}
+
 // RoPE tables of one position in registers: cos/sin of pairs j = 0 .. D/2-1.  They are
 // read from pair-major copies of the tables ([D/2][max_len]: entry (j, p) at
 // j * stride + p), so that the 32 threads of a warp -- 32 consecutive positions --
@@ -302,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int items = 0;
             bool ok = true;
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
-                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Unit un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 const Item& it = un.it;
                 if (items > 0 && !mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
                     ok = false;
@@ -396,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 gslot = gslot + 1 == GS ? 0 : gslot + 1;
             };
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
-                const Unit un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Unit un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 const Item& it = un.it;
                 if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag)) {
                     ok = false;
@@ -484,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int lin = blockIdx.x;
         Unit un;
         if (lin < n_units) {
-            un = decode_unit(lin, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+            un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
             ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
                               un.it.rows(t), H + un.it.q0(t), cos_t, sin_t, tab_stride);
             ++items;
@@ -581,7 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int next = lin + static_cast<int>(gridDim.x);
             Unit nun;
             if (next < n_units) {
-                nun = decode_unit(next, S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                nun = decode_unit(unit_of(next, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
                                   row, nun.it.rows(t), H + nun.it.q0(t), cos_t, sin_t, tab_stride);
                 ++items;
