@@ -131,6 +131,45 @@ int attn_decode(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint1
                 attn_stream_t stream);
 
 /*
+ * Stage driver, long prompts (Section 4.1, the third scenario: a prompt longer than
+ * the stages' static chunk length runs as 1 prefill + N prefill_kv).  The prompt's
+ * prompt_len tokens take positions hist_len .. hist_len+prompt_len-1.  They are
+ * processed in segments of seg_len tokens (the last one may be shorter), in order:
+ * the first segment by attn_prefill when hist_len = 0 and by attn_prefill_kv
+ * otherwise (a later session of a conversation, Section 4.1 scenario 2), every
+ * further segment by attn_prefill_kv over all positions before it.
+ *   q   [batch, prompt_len, n_q_heads,  head_dim]   (the whole prompt, dense)
+ *   k,v [batch, prompt_len, n_kv_heads, head_dim]
+ *   out [batch, prompt_len, n_q_heads,  head_dim]
+ * Cache slots [hist_len, hist_len+prompt_len) are written.  The result equals
+ * one attn_prefill_kv of the whole prompt up to the order of float accumulation.
+ * hist_len >= 0, prompt_len >= 1, seg_len >= 1, hist_len + prompt_len <= max_len;
+ * otherwise ATTN_EINVAL before any launch.  A launch failure in segment i returns
+ * ATTN_ECUDA with the earlier segments enqueued.
+ */
+int attn_prompt(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len,
+                int prompt_len, int seg_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
+                attn_stream_t stream);
+
+/*
+ * Stage driver, decode loop (Section 4.5, steps 3-5, the attention part): n_steps
+ * decode steps in a row.  Step t's token of sequence b takes position
+ * d_hist_len[b] + t and attends to slots [0, d_hist_len[b] + t]; d_hist_len is
+ * read, not written.  Inputs are step-major so that each step's operands are
+ * those of one attn_decode:
+ *   q   [n_steps, batch, 1, n_q_heads,  head_dim]
+ *   k,v [n_steps, batch, 1, n_kv_heads, head_dim]
+ *   out [n_steps, batch, 1, n_q_heads,  head_dim]
+ * 1 <= n_steps <= max_len.  A position past max_len - 1 is handled as in
+ * attn_decode (that step skips the sequence and sets ATTN_DEVERR_HIST_RANGE).  Like
+ * every stage call it only enqueues kernels, so a serving loop can capture it into
+ * a CUDA graph once and replay it.
+ */
+int attn_decode_steps(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                      const int32_t* d_hist_len, int n_steps, uint16_t* k_cache, uint16_t* v_cache,
+                      uint16_t* out, attn_stream_t stream);
+
+/*
  * Synchronise `stream`, read and clear the context's device error word.
  * *flags (may be NULL) receives the ATTN_DEVERR_* bits.  Returns ATTN_OK when
  * the word was zero, ATTN_EDEVICE when a bit was set, ATTN_ECUDA on a CUDA error.

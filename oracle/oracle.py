@@ -177,3 +177,29 @@ def attend_rows(shape, q, hist, k_cache, v_cache, rows, lib=None):
     _check(lib.oracle_attend(ctypes.byref(cfg_of(shape)), q, h, q.shape[1], q.shape[1], _u16(k_cache),
                              _u16(v_cache), out, r.shape[0], r.ctypes.data_as(ctypes.c_void_p)), "attend")
     return out
+
+
+def prompt(shape, q, k, v, hist_len: int, seg_len: int, k_cache, v_cache, lib=None):
+    """Section 4.1, third scenario: a prompt in segments of ``seg_len`` tokens, the
+    first by prefill (no history; scenario 1) or prefill_kv (scenario 2), every later
+    one by prefill_kv over all positions before it.  q [B,P,Hq,D], k/v [B,P,Hkv,D];
+    returns out [B,P,Hq,D] and updates the caches in place."""
+    P = q.shape[1]
+    outs = []
+    for s0 in range(0, P, seg_len):
+        sl = slice(s0, min(P, s0 + seg_len))
+        qs, ks, vs = (np.ascontiguousarray(a[:, sl]) for a in (q, k, v))
+        if hist_len + s0 == 0:
+            outs.append(prefill(shape, qs, ks, vs, k_cache, v_cache, lib=lib))
+        else:
+            outs.append(prefill_kv(shape, qs, ks, vs, hist_len + s0, k_cache, v_cache, lib=lib))
+    return np.concatenate(outs, axis=1)
+
+
+def decode_steps(shape, q, k, v, hist_len, k_cache, v_cache, lib=None):
+    """Section 4.5, steps 3-5 restricted to attention: decode steps in a row, step t's
+    token of sequence b at position hist_len[b] + t.  q [n,B,1,Hq,D], k/v [n,B,1,Hkv,D];
+    returns out [n,B,1,Hq,D] and updates the caches in place."""
+    h = np.asarray(hist_len, dtype=np.int64)
+    return np.stack([decode(shape, q[t], k[t], v[t], (h + t).astype(np.int32), k_cache, v_cache, lib=lib)
+                     for t in range(q.shape[0])])

@@ -6,6 +6,11 @@ Argument marshalling only -- every stage runs in the library's CUDA kernels:
   prefill_kv  (Section 4.3)  the same at positions hist..hist+S-1 over hist cached tokens
   decode      (Section 4.4)  q [B,1,Hq,D], k/v [B,1,Hkv,D], hist_len [B] int32 on the device
 
+and the stage driver of Sections 4.1 and 4.5:
+
+  prompt        a prompt of any length in segments: 1 prefill (or prefill_kv) + N prefill_kv
+  decode_steps  n decode steps in a row, step t at positions hist_len + t (step-major inputs)
+
 Caches are [B,Hkv,L,D] bf16 tensors owned by the caller and updated in place.
 All calls are asynchronous on the given (default: current) torch CUDA stream.
 """
@@ -112,6 +117,37 @@ class Attention:
                                   _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
                                   _stream(stream))
         self._check(rc, "attn_decode")
+        return out
+
+    def prompt(self, q, k, v, hist_len: int, seg_len: int, k_cache, v_cache, out=None,
+               stream=None) -> torch.Tensor:
+        """The whole prompt q [B,P,Hq,D], k/v [B,P,Hkv,D] at positions hist_len.. in segments of seg_len."""
+        P = q.shape[1]
+        qs = (self.batch, P, self.n_q_heads, self.head_dim)
+        ks = (self.batch, P, self.n_kv_heads, self.head_dim)
+        out = self._new_out(q, out)
+        rc = self.lib.attn_prompt(self._ctx, _ptr(q, "q", qs), _ptr(k, "k", ks), _ptr(v, "v", ks), int(hist_len), P,
+                                  int(seg_len), _ptr(k_cache, "k_cache", self._cache_shape()),
+                                  _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
+                                  _stream(stream))
+        self._check(rc, "attn_prompt")
+        return out
+
+    def decode_steps(self, q, k, v, hist_len: torch.Tensor, k_cache, v_cache, out=None,
+                     stream=None) -> torch.Tensor:
+        """n = q.shape[0] decode steps; q [n,B,1,Hq,D], k/v [n,B,1,Hkv,D]; step t at hist_len + t."""
+        n = q.shape[0]
+        qs = (n, self.batch, 1, self.n_q_heads, self.head_dim)
+        ks = (n, self.batch, 1, self.n_kv_heads, self.head_dim)
+        if not (isinstance(hist_len, torch.Tensor) and hist_len.is_cuda and hist_len.dtype == torch.int32
+                and hist_len.is_contiguous() and tuple(hist_len.shape) == (self.batch,)):
+            raise TypeError("hist_len must be a contiguous int32 CUDA tensor of shape [batch]")
+        out = self._new_out(q, out)
+        rc = self.lib.attn_decode_steps(self._ctx, _ptr(q, "q", qs), _ptr(k, "k", ks), _ptr(v, "v", ks),
+                                        hist_len.data_ptr(), n, _ptr(k_cache, "k_cache", self._cache_shape()),
+                                        _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
+                                        _stream(stream))
+        self._check(rc, "attn_decode_steps")
         return out
 
     def timing_enable(self, max_launches: int):

@@ -114,13 +114,16 @@ int encode_map(const attn_ctx* c, CUtensorMap* map, const void* gaddr, cuuint32_
     return ATTN_OK;
 }
 
-// The prefill stages: validate, K1, build the maps over [0, hist+chunk), K2.
+// The prefill stages: validate, K1, build the maps over [0, hist+chunk), K2.  q/k/v/out
+// hold `chunk` tokens of each sequence, sequence b starting at token b * seq_stride
+// (seq_stride = chunk for a dense chunk; the prompt length for a segment of a prompt).
 int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist, int chunk,
-                uint16_t* kc, uint16_t* vc, uint16_t* out, cudaStream_t st) {
+                int seq_stride, uint16_t* kc, uint16_t* vc, uint16_t* out, cudaStream_t st) {
     if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || kc == nullptr || vc == nullptr ||
         out == nullptr)
         return ATTN_EINVAL;
-    if (chunk < 1 || hist < 0 || static_cast<long>(hist) + chunk > c->cfg.max_len) return ATTN_EINVAL;
+    if (chunk < 1 || seq_stride < chunk || hist < 0 || static_cast<long>(hist) + chunk > c->cfg.max_len)
+        return ATTN_EINVAL;
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(kc) || !aligned16(vc) || !aligned16(out))
         return ATTN_EINVAL;
     const attn::Shape& s = c->shape;
@@ -129,7 +132,8 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     {
         const cuuint64_t dims[4] = {D, static_cast<cuuint64_t>(s.n_q_heads), static_cast<cuuint64_t>(chunk),
                                     static_cast<cuuint64_t>(s.batch)};
-        const cuuint64_t strides[3] = {D * 2, D * 2 * s.n_q_heads, D * 2 * s.n_q_heads * static_cast<cuuint64_t>(chunk)};
+        const cuuint64_t strides[3] = {D * 2, D * 2 * s.n_q_heads,
+                                       D * 2 * s.n_q_heads * static_cast<cuuint64_t>(seq_stride)};
         const cuuint32_t box[4] = {64, 1, 128, 1};
         const int rc = encode_map(c, &maps.q, q, 4, dims, strides, box);
         if (rc != ATTN_OK) return rc;
@@ -144,12 +148,13 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         if (rc != ATTN_OK) return rc;
     }
     cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&](int*) {
-        return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, c->d_cos, c->d_sin, kc, vc, c->d_err, st);
+        return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, seq_stride, c->d_cos, c->d_sin, kc, vc, c->d_err,
+                                        st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
     e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&](int* n) {
-        return attn::launch_flash_fwd(s, maps, hist, chunk, c->d_cos_t, c->d_sin_t, out, c->d_flash_o, c->d_flash_ml,
-                                      c->d_err, c->num_sms, st, n);
+        return attn::launch_flash_fwd(s, maps, hist, chunk, seq_stride, c->d_cos_t, c->d_sin_t, out, c->d_flash_o,
+                                      c->d_flash_ml, c->d_err, c->num_sms, st, n);
     });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
     return ATTN_OK;
@@ -262,24 +267,29 @@ void attn_destroy(attn_ctx* c) {
 
 int attn_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int chunk_len,
                  uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
-    return run_prefill(c, q, k, v, 0, chunk_len, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
+    return run_prefill(c, q, k, v, 0, chunk_len, chunk_len, k_cache, v_cache, out,
+                       reinterpret_cast<cudaStream_t>(stream));
 }
 
 int attn_prefill_kv(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len,
                     int chunk_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
-    return run_prefill(c, q, k, v, hist_len, chunk_len, k_cache, v_cache, out,
+    return run_prefill(c, q, k, v, hist_len, chunk_len, chunk_len, k_cache, v_cache, out,
                        reinterpret_cast<cudaStream_t>(stream));
 }
 
-int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
-                uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// One decode step at positions d_hist_len[b] + hist_add.
+int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
+               int hist_add, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st) {
     if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
         k_cache == nullptr || v_cache == nullptr || out == nullptr)
         return ATTN_EINVAL;
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_cache) || !aligned16(v_cache) ||
         !aligned16(out) || (reinterpret_cast<uintptr_t>(d_hist_len) & 3u))
         return ATTN_EINVAL;
-    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool tc = c->cfg.head_dim == 128;  // tensor-core decode; head_dim 64 on the CUDA cores
     if (k_cache != c->dec_k || v_cache != c->dec_v) {
         const cudaError_t me = tc ? attn::make_decode_tc_maps(c->encode, c->shape, k_cache, v_cache, &c->dec_maps)
@@ -296,18 +306,70 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
                           : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         if (tc)
-            return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
+            return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
                                           c->d_err, st);
-        return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, k_cache, v_cache, c->d_cos,
+        return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
     if (tc) return ATTN_OK;  // the tensor-core decode merges its splits itself
     e = timed(c, ATTN_KERNEL_DECODE_COMBINE, st, [&](int*) {
-        return attn::launch_decode_combine(c->shape, d_hist_len, c->d_part_o, c->d_part_ml, nsplit, out, st);
+        return attn::launch_decode_combine(c->shape, d_hist_len, hist_add, c->d_part_o, c->d_part_ml, nsplit, out, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_combine launch");
+    return ATTN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
+                uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    return run_decode(c, q, k, v, d_hist_len, 0, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int attn_prompt(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len, int prompt_len,
+                int seg_len, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    // Section 4.1, third scenario: a prompt longer than the stages' static chunk runs as
+    // one prefill (no history) or prefill_kv, then prefill_kv for every further segment,
+    // each over everything before it.  Checked whole before the first launch.
+    if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || k_cache == nullptr || v_cache == nullptr ||
+        out == nullptr)
+        return ATTN_EINVAL;
+    if (prompt_len < 1 || seg_len < 1 || hist_len < 0 || static_cast<long>(hist_len) + prompt_len > c->cfg.max_len)
+        return ATTN_EINVAL;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out))
+        return ATTN_EINVAL;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t q_tok = static_cast<size_t>(c->cfg.n_q_heads) * c->cfg.head_dim;   // elements per token
+    const size_t kv_tok = static_cast<size_t>(c->cfg.n_kv_heads) * c->cfg.head_dim;
+    for (int s0 = 0; s0 < prompt_len; s0 += seg_len) {
+        const int n = std::min(seg_len, prompt_len - s0);
+        const int rc = run_prefill(c, q + s0 * q_tok, k + s0 * kv_tok, v + s0 * kv_tok, hist_len + s0, n, prompt_len,
+                                   k_cache, v_cache, out + s0 * q_tok, st);
+        if (rc != ATTN_OK) return rc;
+    }
+    return ATTN_OK;
+}
+
+int attn_decode_steps(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
+                      int n_steps, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
+    // Section 4.5, steps 3-5 restricted to attention: n_steps decode steps back to back,
+    // step t at positions d_hist_len[b] + t (the lengths array is read, never written).
+    if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
+        k_cache == nullptr || v_cache == nullptr || out == nullptr || n_steps < 1 || n_steps > c->cfg.max_len)
+        return ATTN_EINVAL;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t q_step = static_cast<size_t>(c->cfg.batch) * c->cfg.n_q_heads * c->cfg.head_dim;
+    const size_t kv_step = static_cast<size_t>(c->cfg.batch) * c->cfg.n_kv_heads * c->cfg.head_dim;
+    for (int t = 0; t < n_steps; ++t) {
+        const int rc = run_decode(c, q + t * q_step, k + t * kv_step, v + t * kv_step, d_hist_len, t, k_cache, v_cache,
+                                  out + t * q_step, st);
+        if (rc != ATTN_OK) return rc;
+    }
     return ATTN_OK;
 }
 

@@ -95,7 +95,7 @@ template <int D, int GM>
 __global__ void __launch_bounds__(NTHREADS, 2) decode_split_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
-    const int32_t* __restrict__ d_hist, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
+    const int32_t* __restrict__ d_hist, int hist_add, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
     const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv, int G, int passes,
     int max_len, int nsplit, float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml,
     int* __restrict__ err) {
@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) decode_split_kernel(
     const int warp = tid >> 5;
     const int lane = tid & 31;
 
-    const int hist = d_hist[b];
+    const int hist = decode_hist(d_hist, b, hist_add);
     if (hist < 0 || hist >= max_len) {
         if (s == 0 && blockIdx.y == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
         return;  // sequence skipped: nothing written
@@ -354,7 +354,8 @@ __global__ void __launch_bounds__(NTHREADS, 2) decode_split_kernel(
 template <int D>
 __global__ void __launch_bounds__(256) decode_combine_kernel(const float* __restrict__ part_o,
                                                              const float* __restrict__ part_ml,
-                                                             const int32_t* __restrict__ d_hist, int Hq, int nsplit,
+                                                             const int32_t* __restrict__ d_hist, int hist_add, int Hq,
+                                                             int nsplit,
                                                              int max_len, uint16_t* __restrict__ out) {
     constexpr int PER_LANE = D / 32;
     __shared__ float sm_w[256];
@@ -363,7 +364,7 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(const float* __rest
     asm volatile("griddepcontrol.wait;" ::: "memory");  // K3's partials are complete and visible
     const int h = blockIdx.x;
     const int b = blockIdx.y;
-    const int hist = d_hist[b];
+    const int hist = decode_hist(d_hist, b, hist_add);
     if (hist < 0 || hist >= max_len) return;
     const size_t row0 = (static_cast<size_t>(b) * Hq + h) * nsplit;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -409,18 +410,20 @@ __global__ void __launch_bounds__(256) decode_combine_kernel(const float* __rest
 
 template <int D, int GM>
 cudaError_t launch_split_t(const Shape& s, const DecodeMaps& maps, dim3 grid, const uint16_t* q,
-                           const uint16_t* k_new, const uint16_t* v_new, const int32_t* d_hist, uint16_t* kc,
-                           uint16_t* vc, const float* cos_tab, const float* sin_tab, int G, int passes, int nsplit,
+                           const uint16_t* k_new, const uint16_t* v_new, const int32_t* d_hist, int hist_add,
+                           uint16_t* kc, uint16_t* vc, const float* cos_tab, const float* sin_tab, int G, int passes,
+                           int nsplit,
                            float scale_log2, float* part_o, float* part_ml, int* err, cudaStream_t st) {
     decode_split_kernel<D, GM><<<grid, NTHREADS, DecLayout<D, GM>::ALLOC, st>>>(
-        maps.k, maps.v, q, k_new, v_new, d_hist, kc, vc, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads, G, passes,
+        maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, kc, vc, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads, G,
+        passes,
         s.max_len, nsplit, scale_log2, part_o, part_ml, err);
     return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_split_d(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
-                           const uint16_t* v_new, const int32_t* d_hist, uint16_t* kc, uint16_t* vc,
+                           const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* kc, uint16_t* vc,
                            const float* cos_tab, const float* sin_tab, int nsplit, float* part_o, float* part_ml,
                            int* err, cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
@@ -432,8 +435,8 @@ cudaError_t launch_split_d(const Shape& s, const DecodeMaps& maps, const uint16_
     switch (gm) {
 #define ATTN_SPLIT_CASE(N)                                                                                     \
     case N:                                                                                                    \
-        return launch_split_t<D, N>(s, maps, grid, q, k_new, v_new, d_hist, kc, vc, cos_tab, sin_tab, G, passes, \
-                                    nsplit, scale_log2, part_o, part_ml, err, st);
+        return launch_split_t<D, N>(s, maps, grid, q, k_new, v_new, d_hist, hist_add, kc, vc, cos_tab, sin_tab, G, \
+                                    passes, nsplit, scale_log2, part_o, part_ml, err, st);
         ATTN_SPLIT_CASE(1) ATTN_SPLIT_CASE(2) ATTN_SPLIT_CASE(3) ATTN_SPLIT_CASE(4)
         ATTN_SPLIT_CASE(5) ATTN_SPLIT_CASE(6) ATTN_SPLIT_CASE(7) ATTN_SPLIT_CASE(8)
 #undef ATTN_SPLIT_CASE
@@ -502,18 +505,18 @@ cudaError_t make_decode_maps(PFN_encodeTiled encode, const Shape& s, const uint1
 }
 
 cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
-                                const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
-                                const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
-                                int nsplit, int* err, cudaStream_t st) {
+                                const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
+                                uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
+                                float* part_ml, int nsplit, int* err, cudaStream_t st) {
     if (s.head_dim == 128)
-        return launch_split_d<128>(s, maps, q, k_new, v_new, d_hist, k_cache, v_cache, cos_tab, sin_tab, nsplit,
-                                   part_o, part_ml, err, st);
-    return launch_split_d<64>(s, maps, q, k_new, v_new, d_hist, k_cache, v_cache, cos_tab, sin_tab, nsplit, part_o,
-                              part_ml, err, st);
+        return launch_split_d<128>(s, maps, q, k_new, v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab,
+                                   nsplit, part_o, part_ml, err, st);
+    return launch_split_d<64>(s, maps, q, k_new, v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab, nsplit,
+                              part_o, part_ml, err, st);
 }
 
-cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
-                                  int nsplit, uint16_t* out, cudaStream_t st) {
+cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
+                                  const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(s.n_q_heads), static_cast<unsigned>(s.batch));
     cfg.blockDim = dim3(256);
@@ -525,9 +528,9 @@ cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const f
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     if (s.head_dim == 128)
-        return cudaLaunchKernelEx(&cfg, decode_combine_kernel<128>, part_o, part_ml, d_hist, s.n_q_heads, nsplit,
+        return cudaLaunchKernelEx(&cfg, decode_combine_kernel<128>, part_o, part_ml, d_hist, hist_add, s.n_q_heads, nsplit,
                                   s.max_len, out);
-    return cudaLaunchKernelEx(&cfg, decode_combine_kernel<64>, part_o, part_ml, d_hist, s.n_q_heads, nsplit,
+    return cudaLaunchKernelEx(&cfg, decode_combine_kernel<64>, part_o, part_ml, d_hist, hist_add, s.n_q_heads, nsplit,
                               s.max_len, out);
 }
 

@@ -188,7 +188,7 @@ template <int NHP>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
-    const int32_t* __restrict__ d_hist, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
+    const int32_t* __restrict__ d_hist, int hist_add, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
     const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv, int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
     uint16_t* __restrict__ out, int* __restrict__ err) {
@@ -210,7 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-    const int hist = d_hist[b];  // in flight while the barriers and TMEM are set up
+    const int hist = decode_hist(d_hist, b, hist_add);  // in flight while the barriers and TMEM are set up
     if (warp == kWarpTma && lane == 0) {
         tma_prefetch_desc(&map_k);
         tma_prefetch_desc(&map_v);
@@ -736,19 +736,19 @@ cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const ui
 }
 
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
-                             const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
-                             const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
-                             int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st) {
+                             const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
+                             uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
+                             float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
     if (G <= 8)
-        decode_tc_kernel<8><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, k_cache,
+        decode_tc_kernel<8><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, k_cache,
                                                               v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
                                                               s.max_len, nsplit, scale_log2, part_o, part_ml,
                                                               counters, out, err);
     else
-        decode_tc_kernel<16><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, k_cache,
+        decode_tc_kernel<16><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, k_cache,
                                                                v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
                                                                s.max_len, nsplit, scale_log2, part_o, part_ml,
                                                                counters, out, err);

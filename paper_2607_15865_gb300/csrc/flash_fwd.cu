@@ -253,7 +253,7 @@ __device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint3
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                     const __grid_constant__ CUtensorMap map_v, int S, int H, int Hq, int Hkv, int batch,
+                     const __grid_constant__ CUtensorMap map_v, int S, int s_stride, int H, int Hq, int Hkv, int batch,
                      int n_pairs, int head, int nsplit, float scale_log2, const float* __restrict__ cos_t,
                      const float* __restrict__ sin_t, int tab_stride, uint16_t* __restrict__ out, float* __restrict__ ws_o,
                      float* __restrict__ ws_ml, int* __restrict__ err) {
@@ -612,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float inv_l = 1.f / l_run;
                     const int lane = threadIdx.x & 31, r0 = row & ~31;
                     uint8_t* stage = gbase + L::OFF_STAGE + warp * L::STAGE_WARP;
-                    uint16_t* obase = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + r0) * Hq + it.h) * D;
+                    uint16_t* obase = out + ((static_cast<size_t>(it.b) * s_stride + it.q0(t) + r0) * Hq + it.h) * D;
 #pragma unroll
                     for (int c2 = 0; c2 < D / 64; ++c2) {
                         uint32_t o[2][32];
@@ -640,7 +640,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // O_T / l -> bf16 -> out straight from each thread's row, or for a piece the
                     // unnormalised O_T
                     const float inv_l = un.piece < 0 ? 1.f / l_run : 1.f;
-                    uint16_t* orow = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D;
+                    uint16_t* orow = out + ((static_cast<size_t>(it.b) * s_stride + it.q0(t) + row) * Hq + it.h) * D;
                     float* prow_o = ws_o + prow * D;
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
@@ -699,7 +699,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Block (tail item, query tile, group of 8 rows); one warp per row.
 template <int D>
 __global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restrict__ ws_o,
-                                                            const float* __restrict__ ws_ml, int S, int H, int Hq,
+                                                            const float* __restrict__ ws_ml, int S, int s_stride, int H,
+                                                            int Hq,
                                                             int G, int hq_b, int n_pairs, int head, int nsplit,
                                                             uint16_t* __restrict__ out) {
     constexpr int PER_LANE = D / 32;
@@ -735,7 +736,7 @@ __global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restr
             for (int e = 0; e < PER_LANE; ++e) acc[e] = fmaf(ws, src[e], acc[e]);
         }
         const float inv = 1.f / lw;
-        uint16_t* dst = out + ((static_cast<size_t>(it.b) * S + it.q0(t) + row) * Hq + it.h) * D + lane * PER_LANE;
+        uint16_t* dst = out + ((static_cast<size_t>(it.b) * s_stride + it.q0(t) + row) * Hq + it.h) * D + lane * PER_LANE;
 #pragma unroll
         for (int e = 0; e < PER_LANE; e += 2)
             *reinterpret_cast<uint32_t*>(dst + e) = pack_bf16x2(acc[e] * inv, acc[e + 1] * inv);
@@ -773,14 +774,14 @@ Schedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
 }
 
 template <int D>
-cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
+cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride, const float* cos_t,
                      const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                      cudaStream_t st, int* n_launched) {
     const Schedule sc = make_schedule(s, hist, chunk, num_sms);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     flash_fwd_kernel<D><<<sc.grid, kThreads, Layout<D>::ALLOC, st>>>(
-        maps.q, maps.k, maps.v, chunk, hist, s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head, sc.nsplit,
-        scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
+        maps.q, maps.k, maps.v, chunk, s_stride, hist, s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head,
+        sc.nsplit, scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
     cudaError_t e = cudaGetLastError();
     *n_launched = 1;
     if (e != cudaSuccess || sc.nsplit == 1) return e;
@@ -794,7 +795,7 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     const int G = s.n_q_heads / s.n_kv_heads;
-    e = cudaLaunchKernelEx(&cfg, flash_combine_kernel<D>, ws_o, ws_ml, chunk, hist, s.n_q_heads, G,
+    e = cudaLaunchKernelEx(&cfg, flash_combine_kernel<D>, ws_o, ws_ml, chunk, s_stride, hist, s.n_q_heads, G,
                            s.n_q_heads * s.batch, sc.n_pairs, sc.head, sc.nsplit, out);
     *n_launched = 2;
     return e;
@@ -818,12 +819,13 @@ cudaError_t configure_flash_fwd() {
     return e != cudaSuccess ? e : configure_d<64>();
 }
 
-cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
-                             const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
-                             cudaStream_t st, int* n_launched) {
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride,
+                             const float* cos_t, const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
+                             int num_sms, cudaStream_t st, int* n_launched) {
     if (s.head_dim == 128)
-        return launch_d<128>(s, maps, hist, chunk, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
-    return launch_d<64>(s, maps, hist, chunk, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
+        return launch_d<128>(s, maps, hist, chunk, s_stride, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st,
+                             n_launched);
+    return launch_d<64>(s, maps, hist, chunk, s_stride, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
 }
 
 }  // namespace attn

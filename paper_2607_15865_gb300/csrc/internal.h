@@ -19,10 +19,11 @@ struct Shape {
 
 // K1: RoPE of the new k (table gather, Section 4.6.2) and the in-place append of
 // k and v into cache slots hist+i (Listing 2 "Concat"; Section 4.6.3).
-// hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.
+// hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.  k and v
+// hold `chunk` tokens of each sequence, sequence b starting at token b * seq_stride.
 cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
-                               const int32_t* d_hist, int chunk, const float* cos_tab, const float* sin_tab,
-                               uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st);
+                               const int32_t* d_hist, int chunk, int seq_stride, const float* cos_tab,
+                               const float* sin_tab, uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st);
 
 // K2: causal flash attention of `chunk` new queries at positions hist.. over cache
 // slots [0, hist+chunk) (prefill: hist=0).  RoPE of q is applied in the kernel.
@@ -37,9 +38,11 @@ cudaError_t configure_flash_fwd();
 // cut into KV pieces whose partials go to ws_o [num_sms*256, D] / ws_ml [num_sms*256, 2]
 // and are merged by a second kernel (then *n_launched = 2).
 // cos_t / sin_t: the RoPE tables pair-major, [D/2][max_len] (entry (j, p) at j * max_len + p).
-cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, const float* cos_t,
-                             const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
-                             cudaStream_t st, int* n_launched);
+// out holds `chunk` tokens of each sequence, sequence b starting at token b * s_stride (the
+// q map carries the same stride).
+cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride,
+                             const float* cos_t, const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
+                             int num_sms, cudaStream_t st, int* n_launched);
 
 // K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
 // with 64-key boxes (built once per cache pair).  K3 also rotates the new key and
@@ -53,8 +56,11 @@ cudaError_t configure_decode();  // dynamic shared-memory limits of K3 (once per
 int decode_num_splits(const Shape& s, int num_sms, int max_splits);
 cudaError_t make_decode_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                              const uint16_t* v_cache, DecodeMaps* maps);
+// Decode lengths: sequence b's new token takes position d_hist[b] + hist_add (hist_add >= 0
+// lets a run of decode steps share one length array); see decode_hist().
 cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
-                                const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
+                                const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
+                                uint16_t* v_cache,
                                 const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                                 int nsplit, int* err, cudaStream_t st);
 // K3 for head_dim 128 on the tensor cores (decode_tc.cu): one CTA per SM, maps with
@@ -68,10 +74,20 @@ int decode_tc_num_splits(const Shape& s, int num_sms);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                                 const uint16_t* v_cache, DecodeMaps* maps);
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
-                             const uint16_t* v_new, const int32_t* d_hist, uint16_t* k_cache, uint16_t* v_cache,
+                             const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
+                             uint16_t* v_cache,
                              const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                              int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st);
-cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, const float* part_o, const float* part_ml,
-                                  int nsplit, uint16_t* out, cudaStream_t st);
+cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
+                                  const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
+
+#ifdef __CUDACC__
+// Position of sequence b's decode token: d_hist[b] + hist_add, or -1 (out of range, so
+// the caller flags and skips the sequence) when the sum leaves int.
+__device__ __forceinline__ int decode_hist(const int32_t* d_hist, int b, int hist_add) {
+    const long long h = static_cast<long long>(d_hist[b]) + hist_add;
+    return h > 0x7FFFFFFFLL ? -1 : static_cast<int>(h);
+}
+#endif
 
 }  // namespace attn

@@ -30,7 +30,8 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 template <int D>
 __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __restrict__ k,
                                                           const uint16_t* __restrict__ v, int hist,
-                                                          const int32_t* __restrict__ d_hist, int chunk, int Hkv,
+                                                          const int32_t* __restrict__ d_hist, int chunk,
+                                                          int seq_stride, int Hkv,
                                                           int max_len, const float* __restrict__ cos_tab,
                                                           const float* __restrict__ sin_tab,
                                                           uint16_t* __restrict__ k_cache,
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
         if (u < n_rope) {
             const int g = u / ROPE_UNITS;
             const int j0 = (u % ROPE_UNITS) * 8;
-            const size_t src = ((static_cast<size_t>(b) * chunk + i) * Hkv + g) * D;
+            const size_t src = ((static_cast<size_t>(b) * seq_stride + i) * Hkv + g) * D;
             const size_t dst = ((static_cast<size_t>(b) * Hkv + g) * max_len + p) * D;
             const uint4 xa = *reinterpret_cast<const uint4*>(k + src + j0);
             const uint4 xb = *reinterpret_cast<const uint4*>(k + src + j0 + HALF);
@@ -87,7 +88,7 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
             const int w = u - n_rope;
             const int g = w / COPY_UNITS;
             const int off = (w % COPY_UNITS) * 8;
-            const size_t src = ((static_cast<size_t>(b) * chunk + i) * Hkv + g) * D + off;
+            const size_t src = ((static_cast<size_t>(b) * seq_stride + i) * Hkv + g) * D + off;
             const size_t dst = ((static_cast<size_t>(b) * Hkv + g) * max_len + p) * D + off;
             *reinterpret_cast<uint4*>(v_cache + dst) = *reinterpret_cast<const uint4*>(v + src);
         }
@@ -97,14 +98,14 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
 }  // namespace
 
 cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
-                               const int32_t* d_hist, int chunk, const float* cos_tab, const float* sin_tab,
-                               uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st) {
+                               const int32_t* d_hist, int chunk, int seq_stride, const float* cos_tab,
+                               const float* sin_tab, uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st) {
     const dim3 grid(static_cast<unsigned>(chunk), static_cast<unsigned>(s.batch));
     if (s.head_dim == 128)
-        rope_append_kernel<128><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, s.n_kv_heads, s.max_len, cos_tab,
+        rope_append_kernel<128><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, seq_stride, s.n_kv_heads, s.max_len, cos_tab,
                                                       sin_tab, k_cache, v_cache, err);
     else
-        rope_append_kernel<64><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, s.n_kv_heads, s.max_len, cos_tab,
+        rope_append_kernel<64><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, seq_stride, s.n_kv_heads, s.max_len, cos_tab,
                                                      sin_tab, k_cache, v_cache, err);
     return cudaGetLastError();
 }
