@@ -580,6 +580,49 @@ def run_sweep(args):
     ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), args.sweep_reps)
     gbs = DECODE_BYTES / (ms * 1e-3) / 1e9
     rows.append({"config": "long decode hist 32767", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+    attn.close()
+    del kc, vc
+    # The stage driver (Sections 4.1 and 4.5).  A 32768-token prompt as 1 prefill + 7
+    # prefill_kv of 4096 tokens (the paper's 80K-prompt example scaled to this cache),
+    # beside the same prompt in one prefill call.
+    attn = Attention.for_shape(S)
+    P, seg = S.max_len, w.LONG_PREFILL
+    q = rnd((1, P, S.n_q_heads, S.head_dim), gen)
+    k, v = rnd((1, P, S.n_kv_heads, S.head_dim), gen), rnd((1, P, S.n_kv_heads, S.head_dim), gen)
+    kc, vc = torch.empty_like(k).view(1, S.n_kv_heads, P, S.head_dim), torch.empty_like(v).view(1, S.n_kv_heads, P, S.head_dim)
+    out = torch.empty_like(q)
+    flop = attn_flops(S, prefill_pairs(0, P))
+    for name, sg in ((f"long prompt {P} as {P // seg} segments of {seg}", seg), (f"long prompt {P} in one prefill", P)):
+        ms = time_calls(lambda: attn.prompt(q, k, v, 0, sg, kc, vc, out), max(3, args.sweep_reps // 4))
+        tf = flop / (ms * 1e-3) / 1e12
+        rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
+    attn.close()
+    del q, k, v, kc, vc, out
+    # A decode loop of 32 steps per call from 4096 valid tokens, B16, replayed from one
+    # CUDA graph: bytes = the 32 steps' decode bytes.
+    sh = w.decode_shape(16)
+    attn = Attention.for_shape(sh)
+    n, hist = 32, 4096
+    kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    q = rnd((n, sh.batch, 1, sh.n_q_heads, sh.head_dim), gen)
+    k = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+    v = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+    out = torch.empty_like(q)
+    hl = torch.full((sh.batch,), hist, dtype=torch.int32, device=dev)
+    attn.decode_steps(q, k, v, hl, kc, vc, out)
+    gr = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+        attn.decode_steps(q, k, v, hl, kc, vc, out)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    ms = time_calls(gr.replay, args.sweep_reps)
+    gbs = sum(decode_bytes(sh, hist + t) for t in range(n)) / (ms * 1e-3) / 1e9
+    rows.append({"config": f"decode loop {n} steps B16 from hist {hist} (CUDA graph)", "ms": ms, "GB/s": gbs,
+                 "frac_hbm": gbs / hbm})
+    attn.close()
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)
