@@ -598,31 +598,34 @@ def run_sweep(args):
         rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
     attn.close()
     del q, k, v, kc, vc, out
-    # A decode loop of 32 steps per call from 4096 valid tokens, B16, replayed from one
-    # CUDA graph: bytes = the 32 steps' decode bytes.
-    sh = w.decode_shape(16)
-    attn = Attention.for_shape(sh)
-    n, hist = 32, 4096
-    kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
-    vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
-    q = rnd((n, sh.batch, 1, sh.n_q_heads, sh.head_dim), gen)
-    k = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
-    v = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
-    out = torch.empty_like(q)
-    hl = torch.full((sh.batch,), hist, dtype=torch.int32, device=dev)
-    attn.decode_steps(q, k, v, hl, kc, vc, out)
-    gr = torch.cuda.CUDAGraph()
-    side = torch.cuda.Stream()
-    side.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+    # Decode loops of 32 steps per call from 4096 valid tokens (B16: bandwidth; B1: the
+    # latency-bound case), each replayed from one CUDA graph: bytes = the 32 steps'
+    # decode bytes.  Consecutive steps start as dependent launches.
+    for bsz in (16, 1):
+        sh = w.decode_shape(bsz)
+        attn = Attention.for_shape(sh)
+        n, hist = 32, 4096
+        kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        q = rnd((n, sh.batch, 1, sh.n_q_heads, sh.head_dim), gen)
+        k = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+        v = rnd((n, sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+        out = torch.empty_like(q)
+        hl = torch.full((sh.batch,), hist, dtype=torch.int32, device=dev)
         attn.decode_steps(q, k, v, hl, kc, vc, out)
-    torch.cuda.current_stream().wait_stream(side)
-    torch.cuda.synchronize()
-    ms = time_calls(gr.replay, args.sweep_reps)
-    gbs = sum(decode_bytes(sh, hist + t) for t in range(n)) / (ms * 1e-3) / 1e9
-    rows.append({"config": f"decode loop {n} steps B16 from hist {hist} (CUDA graph)", "ms": ms, "GB/s": gbs,
-                 "frac_hbm": gbs / hbm})
-    attn.close()
+        gr = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+            attn.decode_steps(q, k, v, hl, kc, vc, out)
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        ms = time_calls(gr.replay, args.sweep_reps)
+        gbs = sum(decode_bytes(sh, hist + t) for t in range(n)) / (ms * 1e-3) / 1e9
+        rows.append({"config": f"decode loop {n} steps B{bsz} from hist {hist} (CUDA graph)", "ms": ms,
+                     "GB/s": gbs, "frac_hbm": gbs / hbm})
+        attn.close()
+        del kc, vc, q, k, v, out, gr
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)

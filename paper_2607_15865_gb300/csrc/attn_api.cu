@@ -281,9 +281,10 @@ int attn_prefill_kv(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uin
 
 namespace {
 
-// One decode step at positions d_hist_len[b] + hist_add.
+// One decode step at positions d_hist_len[b] + hist_add.  after_decode: the previous
+// launch on `st` was this context's decode of the same caches (a decode loop).
 int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
-               int hist_add, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st) {
+               int hist_add, bool after_decode, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st) {
     if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
         k_cache == nullptr || v_cache == nullptr || out == nullptr)
         return ATTN_EINVAL;
@@ -308,7 +309,7 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
-                                          c->d_err, st);
+                                          c->d_err, after_decode, st);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
@@ -327,7 +328,7 @@ extern "C" {
 
 int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
                 uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
-    return run_decode(c, q, k, v, d_hist_len, 0, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
+    return run_decode(c, q, k, v, d_hist_len, 0, false, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int attn_prompt(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len, int prompt_len,
@@ -366,8 +367,8 @@ int attn_decode_steps(attn_ctx* c, const uint16_t* q, const uint16_t* k, const u
     const size_t q_step = static_cast<size_t>(c->cfg.batch) * c->cfg.n_q_heads * c->cfg.head_dim;
     const size_t kv_step = static_cast<size_t>(c->cfg.batch) * c->cfg.n_kv_heads * c->cfg.head_dim;
     for (int t = 0; t < n_steps; ++t) {
-        const int rc = run_decode(c, q + t * q_step, k + t * kv_step, v + t * kv_step, d_hist_len, t, k_cache, v_cache,
-                                  out + t * q_step, st);
+        const int rc = run_decode(c, q + t * q_step, k + t * kv_step, v + t * kv_step, d_hist_len, t, t > 0, k_cache,
+                                  v_cache, out + t * q_step, st);
         if (rc != ATTN_OK) return rc;
     }
     return ATTN_OK;

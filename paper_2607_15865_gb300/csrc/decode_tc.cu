@@ -210,6 +210,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
+    // The lengths, q and the new k/v are the caller's inputs: complete when this grid
+    // starts (it is a dependent launch only after another decode step, which lets its
+    // dependents start only once its own predecessors are complete).
     const int hist = decode_hist(d_hist, b, hist_add);  // in flight while the barriers and TMEM are set up
     if (warp == kWarpTma && lane == 0) {
         tma_prefetch_desc(&map_k);
@@ -244,6 +247,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<const uint32_t*>(gb + L::OFF_TMEM);
+    // Dependent launch after the previous decode step: the setup above overlaps that step's
+    // tail; its cache append, merge counters and partials are read or reused only after
+    // this wait.  The next step may start only after it.
+    griddep_wait();
+    griddep_launch_dependents();
 
     const bool hist_ok = hist >= 0 && hist < max_len;
     if (!hist_ok && s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
@@ -738,21 +746,24 @@ cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const ui
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
-                             float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, cudaStream_t st) {
+                             float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
+                             cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
-    if (G <= 8)
-        decode_tc_kernel<8><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, k_cache,
-                                                              v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
-                                                              s.max_len, nsplit, scale_log2, part_o, part_ml,
-                                                              counters, out, err);
-    else
-        decode_tc_kernel<16><<<grid, kThreads, L::ALLOC, st>>>(maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, k_cache,
-                                                               v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
-                                                               s.max_len, nsplit, scale_log2, part_o, part_ml,
-                                                               counters, out, err);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = L::ALLOC;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = after_decode ? 1 : 0;  // dependent launch only right after another decode step
+    return cudaLaunchKernelEx(&cfg, G <= 8 ? decode_tc_kernel<8> : decode_tc_kernel<16>, maps.k, maps.v, q, k_new,
+                              v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
+                              s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err);
 }
 
 }  // namespace attn

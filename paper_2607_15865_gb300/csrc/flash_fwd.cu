@@ -299,6 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
+    griddep_launch_dependents();  // the merge kernel waits for this whole grid before reading
 
     if (warp >= 8) {
         warpgroup_reg_dec<kRegsLow>();
@@ -312,6 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t gc = 0;  // groups issued
             int items = 0;
             bool ok = true;
+            bool kv_visible = false;  // K1's cache writes complete (dependent launch)
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
                 const Unit un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
                 const Item& it = un.it;
@@ -328,6 +330,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     it.b, bar(B_QFULL));
                 ++items;
                 const int kv_row = it.b * Hkv + it.g;
+                if (!kv_visible) {
+                    // This grid may start while K1 still appends the chunk's k and v: the q
+                    // copy and its RoPE (inputs of the caller, complete before K1 began) overlap
+                    // K1's tail; the first cache read waits for K1.
+                    griddep_wait();
+                    kv_visible = true;
+                }
                 for (int j = un.kv_lo; j <= un.kv_hi; ++j, ++gc) {
                     const int st = static_cast<int>(gc % GS);
                     if (gc >= GS && !mbar_wait(bar(B_GEMPTY0 + st), (gc / GS - 1u) & 1u, abort_flag)) {
@@ -779,10 +788,21 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
                      cudaStream_t st, int* n_launched) {
     const Schedule sc = make_schedule(s, hist, chunk, num_sms);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
-    flash_fwd_kernel<D><<<sc.grid, kThreads, Layout<D>::ALLOC, st>>>(
-        maps.q, maps.k, maps.v, chunk, s_stride, hist, s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head,
-        sc.nsplit, scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
-    cudaError_t e = cudaGetLastError();
+    // Dependent launch after K1 (programmatic stream serialization): only the producer's
+    // first K/V copy waits for K1 (griddep_wait).
+    cudaLaunchConfig_t kcfg = {};
+    kcfg.gridDim = dim3(static_cast<unsigned>(sc.grid));
+    kcfg.blockDim = dim3(kThreads);
+    kcfg.dynamicSmemBytes = Layout<D>::ALLOC;
+    kcfg.stream = st;
+    cudaLaunchAttribute kattr[1];
+    kattr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    kattr[0].val.programmaticStreamSerializationAllowed = 1;
+    kcfg.attrs = kattr;
+    kcfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&kcfg, flash_fwd_kernel<D>, maps.q, maps.k, maps.v, chunk, s_stride, hist,
+                                       s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head, sc.nsplit, scale_log2,
+                                       cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
     *n_launched = 1;
     if (e != cudaSuccess || sc.nsplit == 1) return e;
     cudaLaunchConfig_t cfg = {};

@@ -39,6 +39,9 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
     constexpr int HALF = D / 2;
     constexpr int ROPE_UNITS = D / 16;  // 8 pairs per unit
     constexpr int COPY_UNITS = D / 8;   // 8 elements per unit
+    // K1 is launched in stream order (its inputs are complete when it starts); the K2
+    // launch that follows it may begin its q-side prologue as soon as every K1 CTA runs.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int i = blockIdx.x;
     const int b = blockIdx.y;
     int h0 = hist;

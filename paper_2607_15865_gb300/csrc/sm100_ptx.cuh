@@ -70,6 +70,18 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const v
     }
 }
 
+// ------------------------------------------------------------------ programmatic dependent launch
+
+// Wait until the stream's preceding grid has completed and its writes are visible
+// (a no-op unless this grid was launched with programmatic stream serialization).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Allow the stream's next grid, if launched with programmatic stream serialization, to
+// begin once every CTA of this grid has executed this or exited.
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ TMA
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
