@@ -626,6 +626,30 @@ def run_sweep(args):
                      "GB/s": gbs, "frac_hbm": gbs / hbm})
         attn.close()
         del kc, vc, q, k, v, out, gr
+    # Multi-token decode (a speculative draft of n tokens verified in one call) against the
+    # same n tokens as one prefill_kv chunk: bytes = the history's K/V read once plus the
+    # new tokens' q, k, v and out.
+    for sh, hist, n in ((w.decode_shape(1), 8188, 4), (S, w.LONG_DECODE_HIST - 2, 3)):
+        attn = Attention.for_shape(sh)
+        kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+        q = rnd((sh.batch, n, sh.n_q_heads, sh.head_dim), gen)
+        k = rnd((sh.batch, n, sh.n_kv_heads, sh.head_dim), gen)
+        v = rnd((sh.batch, n, sh.n_kv_heads, sh.head_dim), gen)
+        out = torch.empty_like(q)
+        hl = torch.full((sh.batch,), hist, dtype=torch.int32, device=dev)
+        byts = sh.batch * (hist * sh.n_kv_heads * sh.head_dim * 4 +
+                           n * (sh.n_q_heads * sh.head_dim * 4 + sh.n_kv_heads * sh.head_dim * 8))
+        tag = f"Hq{sh.n_q_heads} Hkv{sh.n_kv_heads} B{sh.batch} hist {hist}"
+        for label, fn in ((f"verify {n} tokens, {tag}: multi-token decode",
+                           lambda: attn.decode_multi(q, k, v, hl, kc, vc, out)),
+                          (f"verify {n} tokens, {tag}: as a prefill_kv chunk",
+                           lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out))):
+            ms = time_calls(fn, args.sweep_reps)
+            gbs = byts / (ms * 1e-3) / 1e9
+            rows.append({"config": label, "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+        attn.close()
+        del kc, vc
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)

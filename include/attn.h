@@ -131,6 +131,21 @@ int attn_decode(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint1
                 attn_stream_t stream);
 
 /*
+ * Multi-token decode: n_new tokens per sequence in one call (Section 4.4 with more than
+ * one new token, e.g. to verify a speculative draft; the paper names speculative
+ * decoding as future work, Section 6).  Sequence b's token i takes position
+ * hist_len[b] + i, is written to that slot and attends to slots [0, hist_len[b] + i]
+ * (causal among the new tokens); lengths are per sequence, read on the device.
+ *   q [batch, n_new, Hq, D], k/v [batch, n_new, Hkv, D], out [batch, n_new, Hq, D].
+ * head_dim 128, 1 <= n_new and n_new * (Hq / Hkv) <= 16 (ATTN_EINVAL otherwise).  A
+ * sequence whose hist_len[b] + n_new exceeds max_len is skipped and flagged as in
+ * attn_decode.  n_new = 1 is attn_decode.
+ */
+int attn_decode_multi(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                      const int32_t* d_hist_len, int n_new, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
+                      attn_stream_t stream);
+
+/*
  * Stage driver, long prompts (Section 4.1, the third scenario: a prompt longer than
  * the stages' static chunk length runs as 1 prefill + N prefill_kv).  The prompt's
  * prompt_len tokens take positions hist_len .. hist_len+prompt_len-1.  They are

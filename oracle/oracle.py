@@ -203,3 +203,18 @@ def decode_steps(shape, q, k, v, hist_len, k_cache, v_cache, lib=None):
     h = np.asarray(hist_len, dtype=np.int64)
     return np.stack([decode(shape, q[t], k[t], v[t], (h + t).astype(np.int32), k_cache, v_cache, lib=lib)
                      for t in range(q.shape[0])])
+
+
+def decode_multi(shape, q, k, v, hist_len, k_cache, v_cache, lib=None):
+    """Decode of n new tokens per sequence (Section 4.4 with n > 1): sequence b's token i
+    takes position hist_len[b] + i and attends causally to slots [0, hist_len[b] + i] --
+    for each sequence exactly prefill_kv of its n tokens over its own history length.
+    q [B,n,Hq,D], k/v [B,n,Hkv,D]; returns out [B,n,Hq,D] and updates the caches in place."""
+    import dataclasses
+    one = dataclasses.replace(shape, batch=1)
+    h = np.asarray(hist_len, dtype=np.int64).reshape(-1)
+    out = np.zeros_like(_u16(q))
+    for b in range(shape.batch):
+        out[b:b + 1] = prefill_kv(one, q[b:b + 1], k[b:b + 1], v[b:b + 1], int(h[b]), k_cache[b:b + 1],
+                                  v_cache[b:b + 1], lib=lib)
+    return out

@@ -17,7 +17,7 @@ ATTN_OK, ATTN_EINVAL, ATTN_EARCH, ATTN_ECUDA, ATTN_ENOMEM, ATTN_EDEVICE = 0, -1,
 DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
-            "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_timing_enable", "attn_timing_read",
+            "attn_decode_multi", "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_timing_enable", "attn_timing_read",
             "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc")
 NOALLOC_SCRATCH_FLOATS = 1 << 20
 KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
@@ -62,6 +62,8 @@ def load(path: str = LIB_PATH):
     lib.attn_prefill_kv.restype = i32
     lib.attn_decode.argtypes = [vp, u16p, u16p, u16p, vp, u16p, u16p, u16p, vp]
     lib.attn_decode.restype = i32
+    lib.attn_decode_multi.argtypes = [vp, u16p, u16p, u16p, vp, i32, u16p, u16p, u16p, vp]
+    lib.attn_decode_multi.restype = i32
     lib.attn_prompt.argtypes = [vp, u16p, u16p, u16p, i32, i32, i32, u16p, u16p, u16p, vp]
     lib.attn_prompt.restype = i32
     lib.attn_decode_steps.argtypes = [vp, u16p, u16p, u16p, vp, i32, u16p, u16p, u16p, vp]

@@ -5,6 +5,7 @@ Argument marshalling only -- every stage runs in the library's CUDA kernels:
   prefill     (Section 4.2)  q [B,S,Hq,D], k/v [B,S,Hkv,D] at positions 0..S-1
   prefill_kv  (Section 4.3)  the same at positions hist..hist+S-1 over hist cached tokens
   decode      (Section 4.4)  q [B,1,Hq,D], k/v [B,1,Hkv,D], hist_len [B] int32 on the device
+              (decode_multi: q [B,n,Hq,D], k/v [B,n,Hkv,D], n new tokens per sequence)
 
 and the stage driver of Sections 4.1 and 4.5:
 
@@ -117,6 +118,23 @@ class Attention:
                                   _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
                                   _stream(stream))
         self._check(rc, "attn_decode")
+        return out
+
+    def decode_multi(self, q, k, v, hist_len: torch.Tensor, k_cache, v_cache, out=None,
+                     stream=None) -> torch.Tensor:
+        """n = q.shape[1] new tokens per sequence at positions hist_len[b] + i (causal among them)."""
+        n = q.shape[1]
+        qs = (self.batch, n, self.n_q_heads, self.head_dim)
+        ks = (self.batch, n, self.n_kv_heads, self.head_dim)
+        if not (isinstance(hist_len, torch.Tensor) and hist_len.is_cuda and hist_len.dtype == torch.int32
+                and hist_len.is_contiguous() and tuple(hist_len.shape) == (self.batch,)):
+            raise TypeError("hist_len must be a contiguous int32 CUDA tensor of shape [batch]")
+        out = self._new_out(q, out)
+        rc = self.lib.attn_decode_multi(self._ctx, _ptr(q, "q", qs), _ptr(k, "k", ks), _ptr(v, "v", ks),
+                                        hist_len.data_ptr(), n, _ptr(k_cache, "k_cache", self._cache_shape()),
+                                        _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", qs),
+                                        _stream(stream))
+        self._check(rc, "attn_decode_multi")
         return out
 
     def prompt(self, q, k, v, hist_len: int, seg_len: int, k_cache, v_cache, out=None,

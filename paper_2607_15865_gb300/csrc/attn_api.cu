@@ -281,10 +281,12 @@ int attn_prefill_kv(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uin
 
 namespace {
 
-// One decode step at positions d_hist_len[b] + hist_add.  after_decode: the previous
-// launch on `st` was this context's decode of the same caches (a decode loop).
+// One decode step of ntok new tokens per sequence at positions d_hist_len[b] + hist_add + i.
+// after_decode: the previous launch on `st` was this context's decode of the same caches
+// (a decode loop).
 int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
-               int hist_add, bool after_decode, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st) {
+               int hist_add, bool after_decode, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st,
+               int ntok = 1) {
     if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
         k_cache == nullptr || v_cache == nullptr || out == nullptr)
         return ATTN_EINVAL;
@@ -303,13 +305,15 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         c->dec_k = k_cache;
         c->dec_v = v_cache;
     }
-    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms), c->nsplit_max)
+    if (ntok < 1 || (ntok > 1 && (!tc || (c->cfg.n_q_heads / c->cfg.n_kv_heads) * ntok > 16))) return ATTN_EINVAL;
+    // the partials hold batch * Hq * nsplit_max rows: ntok tokens share them
+    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms), c->nsplit_max / ntok)
                           : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
-                                          c->d_err, after_decode, st);
+                                          c->d_err, after_decode, ntok, st);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
@@ -329,6 +333,13 @@ extern "C" {
 int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
                 uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, attn_stream_t stream) {
     return run_decode(c, q, k, v, d_hist_len, 0, false, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+int attn_decode_multi(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v,
+                      const int32_t* d_hist_len, int n_new, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
+                      attn_stream_t stream) {
+    return run_decode(c, q, k, v, d_hist_len, 0, false, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream),
+                      n_new);
 }
 
 int attn_prompt(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len, int prompt_len,

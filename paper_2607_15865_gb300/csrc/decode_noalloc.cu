@@ -127,7 +127,7 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (tc && static_cast<long long>(cfg->batch) * cfg->n_kv_heads > kNoallocCounters) return ATTN_EINVAL;
     cudaError_t e = tc ? attn::launch_decode_tc(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin, part_o,
-                                                part_ml, counters, nsplit, out, d_err, false, st)
+                                                part_ml, counters, nsplit, out, d_err, false, 1, st)
                        : attn::launch_decode_split(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin,
                                                    part_o, part_ml, nsplit, d_err, st);
     if (e == cudaSuccess && !tc) e = attn::launch_decode_combine(s, d_hist_len, 0, part_o, part_ml, nsplit, out, st);

@@ -3,34 +3,38 @@
 //
 // Decode (Section 4.4): one new query per sequence b at position p = hist_len[b]
 // attends to cache slots [0, p] of its kv head; its own k/v go to slot p (the
-// in-place "Concat" of Listing 2, Section 4.6.3).
+// in-place "Concat" of Listing 2, Section 4.6.3).  The same kernel takes ntok new
+// tokens per sequence (multi-token decode, e.g. verifying a speculative draft): token
+// i at position p + i attends to slots [0, p + i], causally among the new tokens.
 //
 // With grouped-query attention the G query heads of a kv head read the same keys,
-// so a CTA's work is a contraction [G x D] x [D x keys] -- done here with tcgen05
-// in swapped form so that the 128 keys of a tile fill the MMA's M dimension:
-//   S^T [128 keys x 16] = K_tile [128 x D] . Q^T       (Q: G heads, zero-padded to 16)
+// so a CTA's work is a contraction [C x D] x [D x keys], C = G x ntok columns (query
+// head, new token) -- done here with tcgen05 in swapped form so that the 128 keys of
+// a tile fill the MMA's M dimension:
+//   S^T [128 keys x 16] = K_tile [128 x D] . Q^T       (Q: C columns, zero-padded to 16)
 //   O^T [D x 16]      += V_tile^T [D x 128] . P^T [128 x 16]
-// Both accumulate in TMEM.  The T = ceil((p+1)/128) key tiles of a sequence are dealt
-// to the nsplit CTAs of (b, kv head) in contiguous, balanced runs (split s owns tiles
-// [s*T/nsplit, (s+1)*T/nsplit)), so no CTA loads keys that another one owns.
+// Both accumulate in TMEM.  The T = ceil((p+ntok)/128) key tiles of a sequence are
+// claimed by the nsplit CTAs of (b, kv head): split s starts with tile s, then takes
+// tickets from a per-(b, kv head) counter, so CTAs that stream faster take more tiles
+// and no CTA loads keys that another one owns.
 // 192 threads:
 //   warps 0-3  one thread per key of the tile: scores from TMEM, masking, P^T (bf16)
 //              into shared memory, per-thread partial row sums.  The running max m
 //              moves lazily: a tile whose scores all stay within 2^8 of m (checked
 //              with one OR-barrier) is exponentiated against m as it is; otherwise
-//              the per-head tile maxima are reduced (a halving butterfly: 16
-//              shuffles for 16 heads) and O^T is rescaled.  Epilogue: one thread
+//              the per-column tile maxima are reduced (a halving butterfly: 16
+//              shuffles for 16 columns) and O^T is rescaled.  Epilogue: one thread
 //              per output dimension d;
 //   warp 4     TMA producer: K and V tiles of 128 keys (128-byte swizzle) into
 //              rings of 2 (K) and 4 (V) stages of 32 KB;
-//   warp 5     tcgen05 issuer; it also owns the new token: it rotates k (RoPE from
-//              the table, the same float arithmetic and bf16 rounding as K1), writes
-//              k and v to slot p of the cache and into the shared-memory copies of
-//              the tile that holds slot p (whose later rows it zeroes in V: slots
-//              past p may hold anything, and 0 * NaN would poison O), so the MMA
-//              itself produces the new key's score.
+//   warp 5     tcgen05 issuer; it also owns the new tokens: it rotates their k (RoPE
+//              from the table, the same float arithmetic and bf16 rounding as K1),
+//              writes k and v to their slots of the cache and into the shared-memory
+//              copies of the tiles that hold those slots (zeroing the V rows past the
+//              last new slot: slots past it may hold anything, and 0 * NaN would poison
+//              O), so the MMA itself produces the new keys' scores.
 // Merge: with one split the CTA writes the normalised output.  Otherwise each CTA
-// writes its partial (m, l, acc[D]) per head; the last CTA of (b, kv head) to finish
+// writes its partial (m, l, acc[D]) per column; the last CTA of (b, kv head) to finish
 // (a device counter, reset by that CTA) merges them:
 //   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its copies
@@ -48,7 +52,8 @@ namespace {
 
 constexpr int D = 128;
 constexpr int KT = 128;     // keys per tile (MMA M)
-constexpr int NH = 16;      // padded query heads (MMA N)
+constexpr int NH = 16;      // padded columns of Q^T (MMA N): query heads x new tokens
+constexpr int kMaxTok = 16;  // new tokens per sequence in one launch (heads x tokens <= NH)
 constexpr int KST = 2;      // K ring stages (a K tile is free once S^T of it completes)
 constexpr int VST = 4;      // V ring stages (a V tile is held until its PV completes)
 constexpr int kThreads = 192;
@@ -182,14 +187,15 @@ __device__ __forceinline__ bool halving_leader(int lane) {
     return N == 16 ? (lane & 1) == 0 : (lane & 3) == 0;
 }
 
-// NHP: query heads the softmax processes (8 when G <= 8, else 16); the MMA always
-// runs N = 16 with the rows of Q^T past G zero.
+// NHP: columns the softmax processes (8 when G * ntok <= 8, else 16); the MMA always
+// runs N = 16 with the rows of Q^T past C = G * ntok zero.
 template <int NHP>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
-    const int32_t* __restrict__ d_hist, int hist_add, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
-    const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv, int max_len, int nsplit,
+    const int32_t* __restrict__ d_hist, int hist_add, int ntok, uint16_t* __restrict__ k_cache,
+    uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
+    int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
     uint16_t* __restrict__ out, int* __restrict__ err) {
     constexpr int HALF = D / 2;
@@ -203,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     auto bar = [&](int i) -> uint32_t { return base + L::OFF_BAR + 8u * static_cast<uint32_t>(i); };
 
     const int G = Hq / Hkv;
+    const int C = G * ntok;  // columns of Q^T: column c = token c / G, head h0 + c % G
     const int s = blockIdx.x;
     const int g = blockIdx.y;
     const int b = blockIdx.z;
@@ -253,12 +260,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     griddep_wait();
     griddep_launch_dependents();
 
-    const bool hist_ok = hist >= 0 && hist < max_len;
+    const bool hist_ok = hist >= 0 && hist <= max_len - ntok;
     if (!hist_ok && s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
-    const int nkeys = hist + 1;
-    const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds slot p
+    const int nkeys = hist + ntok;        // slots [0, hist) and the new tokens' [hist, hist + ntok)
+    const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds the last new slot
     const int kv_row = b * Hkv + g;
-    const size_t row0 = (static_cast<size_t>(b) * Hq + h0) * nsplit + s;  // head h adds h * nsplit
+    // partial row of column c and split sp: ((b * ntok + c / G) * Hq + h0 + c % G) * nsplit + sp
+    auto col_row = [&](int c) -> size_t {
+        return ((static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G) * nsplit;
+    };
+    auto out_row = [&](int c) -> size_t { return (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G; };
     int* meta = reinterpret_cast<int*>(gb + L::OFF_META);  // tile index of local tile j at [j % 8]; -1 ends
 
     if (!hist_ok) {
@@ -321,19 +332,23 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             }
         }
     } else if (warp == kWarpMma) {
-        // ------------------------------------------------------------ tcgen05 issuer (+ the new token)
-        // Lane l handles dimensions 4l .. 4l+3 of the new token (rotated by every CTA;
-        // written by the one that gets tile T-1).
-        const int hrow = hist - (T - 1) * KT;  // row of slot p in tile T-1
-        uint2 k_rot, v_val;
-        {
+        // ------------------------------------------------------------ tcgen05 issuer (+ the new tokens)
+        // Lane l handles dimensions 4l .. 4l+3 of each new token tt (slot hist + tt, rotated
+        // at that position by every CTA; written by the CTA that gets the slot's tile).
+        const int last_row = (hist + ntok - 1) - (T - 1) * KT;  // row of the last new slot in tile T-1
+        uint2 k_rot[kMaxTok], v_val[kMaxTok];
+#pragma unroll
+        for (int tt = 0; tt < kMaxTok; ++tt) {
+            if (tt >= ntok) break;
             const int d0 = 4 * lane;
             const int dp = d0 < HALF ? d0 + HALF : d0 - HALF;  // RoPE partner dimensions
-            const uint2 kx = *reinterpret_cast<const uint2*>(k_new + static_cast<size_t>(kv_row) * D + d0);
-            const uint2 ky = *reinterpret_cast<const uint2*>(k_new + static_cast<size_t>(kv_row) * D + dp);
-            v_val = *reinterpret_cast<const uint2*>(v_new + static_cast<size_t>(kv_row) * D + d0);
-            const float4 c4 = *reinterpret_cast<const float4*>(cos_tab + static_cast<size_t>(hist) * HALF + d0 % HALF);
-            const float4 s4 = *reinterpret_cast<const float4*>(sin_tab + static_cast<size_t>(hist) * HALF + d0 % HALF);
+            const size_t src = (static_cast<size_t>(b * ntok + tt) * Hkv + g) * D;
+            const uint2 kx = *reinterpret_cast<const uint2*>(k_new + src + d0);
+            const uint2 ky = *reinterpret_cast<const uint2*>(k_new + src + dp);
+            v_val[tt] = *reinterpret_cast<const uint2*>(v_new + src + d0);
+            const size_t pos = static_cast<size_t>(hist + tt);
+            const float4 c4 = *reinterpret_cast<const float4*>(cos_tab + pos * HALF + d0 % HALF);
+            const float4 s4 = *reinterpret_cast<const float4*>(sin_tab + pos * HALF + d0 % HALF);
             const float xs[4] = {__uint_as_float(kx.x << 16), __uint_as_float(kx.x & 0xFFFF0000u),
                                  __uint_as_float(kx.y << 16), __uint_as_float(kx.y & 0xFFFF0000u)};
             const float ys[4] = {__uint_as_float(ky.x << 16), __uint_as_float(ky.x & 0xFFFF0000u),
@@ -346,7 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                                           : __fadd_rn(__fmul_rn(xs[e], cs[e]), __fmul_rn(ys[e], ss[e]));
                 kb[e] = to_bf16(r);
             }
-            k_rot = make_uint2(kb[0] | (kb[1] << 16), kb[2] | (kb[3] << 16));
+            k_rot[tt] = make_uint2(kb[0] | (kb[1] << 16), kb[2] | (kb[3] << 16));
         }
         constexpr uint32_t kIdQK = idesc_bf16_f32(KT, NH, false, false);
         constexpr uint32_t kIdPV = idesc_bf16_f32(D, NH, true, false);
@@ -358,12 +373,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             if (!wait_all(B_PFULL0 + (jj & 1), static_cast<uint32_t>(jj >> 1) & 1u)) return false;
             if (!wait_all(B_VFULL0 + jj % VST, static_cast<uint32_t>(jj / VST) & 1u)) return false;
             const uint32_t sV = base + L::OFF_V + (jj % VST) * L::TILE;
-            if (meta[jj % 8] == T - 1) {
-                // v_new into row hrow; the rows past it (slots past p) zeroed
+            const int vtile = meta[jj % 8];
+            if (vtile * KT + KT > hist) {
+                // the new tokens' v into their rows of this tile; in tile T-1 the rows past the
+                // last new slot zeroed (those slots may hold anything, and 0 * NaN would poison O)
                 uint8_t* vt = gb + L::OFF_V + (jj % VST) * L::TILE;
-                *reinterpret_cast<uint2*>(vt + sw_elem(hrow, 4 * lane, KT)) = v_val;
-                for (int i = (hrow + 1) * 16 + lane; i < KT * 16; i += 32)
-                    *reinterpret_cast<uint4*>(vt + sw_elem(i >> 4, 8 * (i & 15), KT)) = make_uint4(0, 0, 0, 0);
+#pragma unroll
+                for (int tt = 0; tt < kMaxTok; ++tt)
+                    if (tt < ntok && (hist + tt) / KT == vtile)
+                        *reinterpret_cast<uint2*>(vt + sw_elem(hist + tt - vtile * KT, 4 * lane, KT)) = v_val[tt];
+                if (vtile == T - 1)
+                    for (int i = (last_row + 1) * 16 + lane; i < KT * 16; i += 32)
+                        *reinterpret_cast<uint4*>(vt + sw_elem(i >> 4, 8 * (i & 15), KT)) = make_uint4(0, 0, 0, 0);
                 fence_proxy_async_smem();
             }
             __syncwarp();
@@ -396,11 +417,17 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     break;
                 }
                 const uint32_t sK = base + L::OFF_K + ks * L::TILE;
-                if (tile == T - 1) {  // the new token: to the cache, and its rotated k into row hrow
-                    const size_t dst = (static_cast<size_t>(kv_row) * max_len + hist) * D + 4 * lane;
-                    *reinterpret_cast<uint2*>(k_cache + dst) = k_rot;
-                    *reinterpret_cast<uint2*>(v_cache + dst) = v_val;
-                    *reinterpret_cast<uint2*>(gb + L::OFF_K + ks * L::TILE + sw_elem(hrow, 4 * lane, KT)) = k_rot;
+                if (tile * KT + KT > hist) {  // new tokens in this tile: to the cache, rotated k into their rows
+#pragma unroll
+                    for (int tt = 0; tt < kMaxTok; ++tt) {
+                        if (tt < ntok && (hist + tt) / KT == tile) {
+                            const size_t dst = (static_cast<size_t>(kv_row) * max_len + hist + tt) * D + 4 * lane;
+                            *reinterpret_cast<uint2*>(k_cache + dst) = k_rot[tt];
+                            *reinterpret_cast<uint2*>(v_cache + dst) = v_val[tt];
+                            *reinterpret_cast<uint2*>(gb + L::OFF_K + ks * L::TILE +
+                                                      sw_elem(hist + tt - tile * KT, 4 * lane, KT)) = k_rot[tt];
+                        }
+                    }
                     fence_proxy_async_smem();
                 }
                 __syncwarp();
@@ -444,29 +471,31 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         const int t = tid;  // key row of a tile; output dimension in the epilogue
         const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
         {
-            // Q^T: row h = rotated q of head h0 + h (bf16), zero rows past G; P^T buffers zeroed.
-            // Each thread owns dimension t of every head: all loads first, then the math.
+            // Q^T: row c = rotated q of token c / G, head h0 + c % G (bf16) at position
+            // hist + c / G; zero rows past C; P^T buffers zeroed.  Each thread owns dimension t
+            // of every column: all loads first, then the math.
             uint8_t* qs = gb + L::OFF_Q;
-            const float* cos_row = cos_tab + static_cast<size_t>(hist) * HALF;
-            const float* sin_row = sin_tab + static_cast<size_t>(hist) * HALF;
             const int tp = t < HALF ? t + HALF : t - HALF;  // RoPE partner dimension
-            const float c_t = cos_row[t % HALF], s_t = sin_row[t % HALF];
-            float qx[NHP], qy[NHP];
+            float qx[NHP], qy[NHP], c_t[NHP], s_t[NHP];
 #pragma unroll
-            for (int h = 0; h < NHP; ++h) {
-                const uint16_t* qrow = q + (static_cast<size_t>(b) * Hq + h0 + min(h, G - 1)) * D;
-                qx[h] = bf16_at(qrow + t);
-                qy[h] = bf16_at(qrow + tp);
+            for (int c = 0; c < NHP; ++c) {
+                const int cc = min(c, C - 1);
+                const uint16_t* qrow = q + out_row(cc) * D;
+                qx[c] = bf16_at(qrow + t);
+                qy[c] = bf16_at(qrow + tp);
+                const size_t pos = static_cast<size_t>(hist + cc / G);
+                c_t[c] = cos_tab[pos * HALF + t % HALF];
+                s_t[c] = sin_tab[pos * HALF + t % HALF];
             }
 #pragma unroll
-            for (int h = 0; h < NH; ++h) {
+            for (int c = 0; c < NH; ++c) {
                 uint16_t qb = 0;
-                if (h < NHP && h < G) {
-                    const float r = t < HALF ? __fsub_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t))
-                                             : __fadd_rn(__fmul_rn(qx[h], c_t), __fmul_rn(qy[h], s_t));
+                if (c < NHP && c < C) {
+                    const float r = t < HALF ? __fsub_rn(__fmul_rn(qx[c], c_t[c]), __fmul_rn(qy[c], s_t[c]))
+                                             : __fadd_rn(__fmul_rn(qx[c], c_t[c]), __fmul_rn(qy[c], s_t[c]));
                     qb = to_bf16(r);
                 }
-                *reinterpret_cast<uint16_t*>(qs + sw_elem(h, t, NH)) = qb;
+                *reinterpret_cast<uint16_t*>(qs + sw_elem(c, t, NH)) = qb;
             }
             for (int i = t; i < 2 * NH * 128 / 16; i += 128)
                 reinterpret_cast<uint4*>(gb + L::OFF_P)[i] = make_uint4(0, 0, 0, 0);
@@ -494,12 +523,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             uint32_t r[NHP];
             tmem_ld_cols<NHP>(tmem + lane_base + (j & 1) * NH, r);
             tmem_wait_ld();
-            const bool valid = tile * KT + t < nkeys;
+            // key tile * KT + t is visible to column c (token c / G) iff it is <= hist + c / G
+            const int kpos = tile * KT + t - hist;  // >= 0 for the new tokens' slots
             float sc[NHP];
             bool exceed = false;
 #pragma unroll
             for (int h = 0; h < NHP; ++h) {
-                sc[h] = (valid && h < G) ? __uint_as_float(r[h]) * scale_log2 : -INFINITY;
+                sc[h] = (h < C && kpos <= h / G) ? __uint_as_float(r[h]) * scale_log2 : -INFINITY;
                 exceed |= sc[h] > m_run[h] + 8.f;  // lazy: P stays <= 2^8 otherwise
             }
             if (named_or_128(exceed)) {
@@ -543,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             uint8_t* pbuf = gb + L::OFF_P + (j & 1) * (2 * NH * 128);
 #pragma unroll
             for (int h = 0; h < NHP; ++h) {
-                if (h < G) {
+                if (h < C) {
                     const float m_ref = m_run[h] == -INFINITY ? 0.f : m_run[h];
                     const float p = fast_exp2(sc[h] - m_ref);
                     l_run[h] += p;
@@ -555,9 +585,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             mbar_arrive(bar(B_PFULL0 + (j & 1)));
         }
         if (ok && n == 0) {
-            if (t < G) {  // no tile came to this CTA: weight 0 in the merge
-                part_ml[(row0 + static_cast<size_t>(t) * nsplit) * 2 + 0] = -INFINITY;
-                part_ml[(row0 + static_cast<size_t>(t) * nsplit) * 2 + 1] = 0.f;
+            if (t < C) {  // no tile came to this CTA: weight 0 in the merge
+                part_ml[(col_row(t) + s) * 2 + 0] = -INFINITY;
+                part_ml[(col_row(t) + s) * 2 + 1] = 0.f;
             }
         } else if (ok) {
             // (PVDONE could be two phases behind here -- PV(n-2) may still run -- so the
@@ -575,13 +605,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             named_sync_128();
 #pragma unroll
             for (int h = 0; h < NHP; ++h) {
-                if (h < G) {
+                if (h < C) {
                     const float4 l4 = reinterpret_cast<const float4*>(ls)[h];
                     const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
                     if (nsplit == 1) {
-                        out[(static_cast<size_t>(b) * Hq + h0 + h) * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
+                        out[out_row(h) * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
                     } else {
-                        const size_t row = row0 + static_cast<size_t>(h) * nsplit;
+                        const size_t row = col_row(h) + s;
                         part_o[row * D + t] = __uint_as_float(o[h]);
                         if (t == 0) {
                             part_ml[row * 2 + 0] = m_run[h];
@@ -624,12 +654,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             float2* wml = reinterpret_cast<float2*>(gb + L::OFF_K);
             float* winv = reinterpret_cast<float*>(gb + L::OFF_K + NH * 256 * 8);
             float* racc = winv + NH;
-            const size_t hrow0 = (static_cast<size_t>(b) * Hq + h0) * nsplit;  // row of (head 0, split 0)
-            const int npair = G * nsplit;
-            for (int p = tid; p < npair; p += kThreads)  // pair p = (head p / nsplit, split p % nsplit)
-                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + hrow0 + p);
+            const int npair = C * nsplit;
+            for (int p = tid; p < npair; p += kThreads)  // pair p = (column p / nsplit, split p % nsplit)
+                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + col_row(p / nsplit) + p % nsplit);
             __syncthreads();
-            for (int h = warp; h < G; h += kThreads / 32) {  // per head: M, weights, 1/L
+            for (int h = warp; h < C; h += kThreads / 32) {  // per column: M, weights, 1/L
                 float mm = -INFINITY;
                 for (int sp = lane; sp < nsplit; sp += 32) {
                     const float2 ml = wml[h * nsplit + sp];
@@ -662,10 +691,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 float wgt[NHP];
 #pragma unroll
                 for (int h = 0; h < NHP; ++h) {
-                    const int hh = min(h, G - 1);
-                    wgt[h] = h < G ? wml[hh * nsplit + sp].x : 0.f;
-                    o4[h] = __ldcg(reinterpret_cast<const float4*>(
-                                       part_o + (hrow0 + static_cast<size_t>(hh) * nsplit + sp) * D) + lane);
+                    const int hh = min(h, C - 1);
+                    wgt[h] = h < C ? wml[hh * nsplit + sp].x : 0.f;
+                    o4[h] = __ldcg(reinterpret_cast<const float4*>(part_o + (col_row(hh) + sp) * D) + lane);
                 }
 #pragma unroll
                 for (int h = 0; h < NHP; ++h) {
@@ -678,9 +706,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             }
 #pragma unroll
             for (int h = 0; h < NHP; ++h)
-                if (h < G) reinterpret_cast<float4*>(racc + (warp * NH + h) * D)[lane] = acc[h];
+                if (h < C) reinterpret_cast<float4*>(racc + (warp * NH + h) * D)[lane] = acc[h];
             __syncthreads();
-            for (int p = tid; p < G * (D / 4); p += kThreads) {  // (head, 4 dimensions)
+            for (int p = tid; p < C * (D / 4); p += kThreads) {  // (column, 4 dimensions)
                 const int h = p / (D / 4), c = p % (D / 4);
                 float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -695,7 +723,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 const uint2 packed = make_uint2(
                     to_bf16(sum.x * inv) | (static_cast<uint32_t>(to_bf16(sum.y * inv)) << 16),
                     to_bf16(sum.z * inv) | (static_cast<uint32_t>(to_bf16(sum.w * inv)) << 16));
-                *reinterpret_cast<uint2*>(out + (static_cast<size_t>(b) * Hq + h0 + h) * D + 4 * c) = packed;
+                *reinterpret_cast<uint2*>(out + out_row(h) * D + 4 * c) = packed;
             }
         }
     }
@@ -747,7 +775,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
                              float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
-                             cudaStream_t st) {
+                             int ntok, cudaStream_t st) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
@@ -761,9 +789,10 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = after_decode ? 1 : 0;  // dependent launch only right after another decode step
-    return cudaLaunchKernelEx(&cfg, G <= 8 ? decode_tc_kernel<8> : decode_tc_kernel<16>, maps.k, maps.v, q, k_new,
-                              v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads,
-                              s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err);
+    if (ntok < 1 || ntok > kMaxTok || G * ntok > NH) return cudaErrorInvalidValue;
+    return cudaLaunchKernelEx(&cfg, G * ntok <= 8 ? decode_tc_kernel<8> : decode_tc_kernel<16>, maps.k, maps.v, q,
+                              k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
+                              s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err);
 }
 
 }  // namespace attn

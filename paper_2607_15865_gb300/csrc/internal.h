@@ -68,7 +68,10 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
 // in (the last CTA of each (b, kv head) merges and writes `out`), so no K4 follows.
 // Splits claim key tiles from a per-(b, kv head) counter.  `counters`: 2*B*Hkv ints
 // (merge counts, then tile claims), zero before the first launch; every launch leaves
-// them zero.  after_decode: the stream's previous kernel is a decode_tc launch (the
+// them zero.  ntok >= 1 new tokens per sequence (q/k/v/out [B, ntok, H, D]) at positions
+// d_hist[b] + hist_add + i, token i attending causally to slots [0, that position];
+// (Hq / Hkv) * ntok <= 16, and the partials need B * ntok * Hq * nsplit rows.
+// after_decode: the stream's previous kernel is a decode_tc launch (the
 // previous step of a decode loop); this one then starts as a dependent launch whose
 // setup overlaps that step's tail.  Never set it after any other kernel: the inputs
 // are read before the grid waits on its predecessor.
@@ -80,7 +83,8 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache,
                              const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
-                             int* counters, int nsplit, uint16_t* out, int* err, bool after_decode, cudaStream_t st);
+                             int* counters, int nsplit, uint16_t* out, int* err, bool after_decode, int ntok,
+                             cudaStream_t st);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
                                   const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
 

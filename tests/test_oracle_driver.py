@@ -56,3 +56,31 @@ def test_decode_steps_follow_each_sequence_own_length():
         ref = O.decode(shape, step(q)[t], step(k)[t], step(v)[t], hist + t, rk, rv)
         assert (got[t] == ref).all()
     assert (kc == rk).all() and (vc == rv).all()
+
+
+def test_multi_token_decode_one_token_is_decode():
+    shape = SHAPES[0]
+    q, k, v = w.tokens(shape, "mtd1", 1)
+    hist = np.array([12, 99], np.int32)
+    kc, vc = w.cache(shape, "mtd1", int(hist.max()), fill="random")
+    rk, rv = kc.copy(), vc.copy()
+    got = O.decode_multi(shape, q, k, v, hist, kc, vc)
+    ref = O.decode(shape, q, k, v, hist, rk, rv)
+    assert (got == ref).all()
+    assert (kc == rk).all() and (vc == rv).all()
+
+
+def test_multi_token_decode_equals_decode_steps():
+    """n new tokens at once = n single-token decode steps (each token sees the earlier new
+    tokens, as they were appended by the earlier steps)."""
+    shape = SHAPES[0]
+    n = 5
+    q, k, v = w.tokens(shape, "mtd2", n)
+    hist = np.array([3, 70], np.int32)
+    kc, vc = w.cache(shape, "mtd2", int(hist.max()), fill="random")
+    rk, rv = kc.copy(), vc.copy()
+    got = O.decode_multi(shape, q, k, v, hist, kc, vc)
+    step = lambda a: np.ascontiguousarray(a.transpose(1, 0, 2, 3)[:, :, None])
+    ref = O.decode_steps(shape, step(q), step(k), step(v), hist, rk, rv)
+    assert (got == ref[:, :, 0].transpose(1, 0, 2, 3)).all()
+    assert (kc == rk).all() and (vc == rv).all()
