@@ -54,6 +54,9 @@ constexpr int D = 128;
 constexpr int KT = 128;     // keys per tile (MMA M)
 constexpr int NH = 16;      // padded columns of Q^T (MMA N): query heads x new tokens
 constexpr int kMaxTok = 16;  // new tokens per sequence in one launch (heads x tokens <= NH)
+// The kernel is built for MAXTOK = 1 (plain decode) and kMaxTok (multi-token decode): the
+// issuer keeps the new tokens' rotated k and v in registers, unrolled over MAXTOK, and
+// sixteen unrolled slots cost a single-token decode about 2 us.
 constexpr int KST = 2;      // K ring stages (a K tile is free once S^T of it completes)
 constexpr int VST = 4;      // V ring stages (a V tile is held until its PV completes)
 constexpr int kThreads = 192;
@@ -80,7 +83,9 @@ struct L {
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
     static constexpr int OFF_ABORT = OFF_TMEM + 4;
     static constexpr int OFF_LAST = OFF_ABORT + 4;
-    static constexpr int BYTES = OFF_LAST + 8;
+    static constexpr int OFF_CROW = OFF_LAST + 8;  // size_t [16]: partial row (split 0) of column c
+    static constexpr int OFF_OROW = OFF_CROW + NH * 8;  // size_t [16]: q / out row of column c
+    static constexpr int BYTES = OFF_OROW + NH * 8;
     static constexpr int ALLOC = BYTES + 1024;
 };
 static_assert(L::ALLOC <= 232448, "shared memory of one CTA");
@@ -189,7 +194,7 @@ __device__ __forceinline__ bool halving_leader(int lane) {
 
 // NHP: columns the softmax processes (8 when G * ntok <= 8, else 16); the MMA always
 // runs N = 16 with the rows of Q^T past C = G * ntok zero.
-template <int NHP>
+template <int NHP, int MAXTOK>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
@@ -226,6 +231,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         tma_prefetch_desc(&map_v);
     }
 
+    if (tid < NH) {
+        const int c = min(tid, G * ntok - 1);
+        const size_t r = (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G;
+        reinterpret_cast<size_t*>(gb + L::OFF_OROW)[tid] = r;
+        reinterpret_cast<size_t*>(gb + L::OFF_CROW)[tid] = r * nsplit;
+    }
     if (tid == 0) {
         *abort_flag = 0;
         mbar_init(bar(B_QREADY), 128);
@@ -265,11 +276,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const int nkeys = hist + ntok;        // slots [0, hist) and the new tokens' [hist, hist + ntok)
     const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds the last new slot
     const int kv_row = b * Hkv + g;
-    // partial row of column c and split sp: ((b * ntok + c / G) * Hq + h0 + c % G) * nsplit + sp
-    auto col_row = [&](int c) -> size_t {
-        return ((static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G) * nsplit;
-    };
-    auto out_row = [&](int c) -> size_t { return (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G; };
+    // Rows of column c (token c / G, head h0 + c % G), tabulated once in the prologue:
+    // q / out row (b * ntok + c / G) * Hq + h0 + c % G, and partial row of split 0 that
+    // times nsplit (split sp adds sp).  Columns past C repeat column C - 1.
+    const size_t* crow = reinterpret_cast<const size_t*>(gb + L::OFF_CROW);
+    const size_t* orow = reinterpret_cast<const size_t*>(gb + L::OFF_OROW);
     int* meta = reinterpret_cast<int*>(gb + L::OFF_META);  // tile index of local tile j at [j % 8]; -1 ends
 
     if (!hist_ok) {
@@ -336,9 +347,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         // Lane l handles dimensions 4l .. 4l+3 of each new token tt (slot hist + tt, rotated
         // at that position by every CTA; written by the CTA that gets the slot's tile).
         const int last_row = (hist + ntok - 1) - (T - 1) * KT;  // row of the last new slot in tile T-1
-        uint2 k_rot[kMaxTok], v_val[kMaxTok];
+        uint2 k_rot[MAXTOK], v_val[MAXTOK];
 #pragma unroll
-        for (int tt = 0; tt < kMaxTok; ++tt) {
+        for (int tt = 0; tt < MAXTOK; ++tt) {
             if (tt >= ntok) break;
             const int d0 = 4 * lane;
             const int dp = d0 < HALF ? d0 + HALF : d0 - HALF;  // RoPE partner dimensions
@@ -379,7 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 // last new slot zeroed (those slots may hold anything, and 0 * NaN would poison O)
                 uint8_t* vt = gb + L::OFF_V + (jj % VST) * L::TILE;
 #pragma unroll
-                for (int tt = 0; tt < kMaxTok; ++tt)
+                for (int tt = 0; tt < MAXTOK; ++tt)
                     if (tt < ntok && (hist + tt) / KT == vtile)
                         *reinterpret_cast<uint2*>(vt + sw_elem(hist + tt - vtile * KT, 4 * lane, KT)) = v_val[tt];
                 if (vtile == T - 1)
@@ -419,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 const uint32_t sK = base + L::OFF_K + ks * L::TILE;
                 if (tile * KT + KT > hist) {  // new tokens in this tile: to the cache, rotated k into their rows
 #pragma unroll
-                    for (int tt = 0; tt < kMaxTok; ++tt) {
+                    for (int tt = 0; tt < MAXTOK; ++tt) {
                         if (tt < ntok && (hist + tt) / KT == tile) {
                             const size_t dst = (static_cast<size_t>(kv_row) * max_len + hist + tt) * D + 4 * lane;
                             *reinterpret_cast<uint2*>(k_cache + dst) = k_rot[tt];
@@ -480,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
 #pragma unroll
             for (int c = 0; c < NHP; ++c) {
                 const int cc = min(c, C - 1);
-                const uint16_t* qrow = q + out_row(cc) * D;
+                const uint16_t* qrow = q + orow[cc] * D;
                 qx[c] = bf16_at(qrow + t);
                 qy[c] = bf16_at(qrow + tp);
                 const size_t pos = static_cast<size_t>(hist + cc / G);
@@ -523,13 +534,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             uint32_t r[NHP];
             tmem_ld_cols<NHP>(tmem + lane_base + (j & 1) * NH, r);
             tmem_wait_ld();
-            // key tile * KT + t is visible to column c (token c / G) iff it is <= hist + c / G
-            const int kpos = tile * KT + t - hist;  // >= 0 for the new tokens' slots
+            // key tile * KT + t is visible to column c (token c / G) iff it is <= hist + c / G,
+            // i.e. iff c >= (key - hist) * G (always for a history key: key - hist < 0)
+            const int kg = (tile * KT + t - hist) * G;
             float sc[NHP];
             bool exceed = false;
 #pragma unroll
             for (int h = 0; h < NHP; ++h) {
-                sc[h] = (h < C && kpos <= h / G) ? __uint_as_float(r[h]) * scale_log2 : -INFINITY;
+                sc[h] = (h < C && h >= kg) ? __uint_as_float(r[h]) * scale_log2 : -INFINITY;
                 exceed |= sc[h] > m_run[h] + 8.f;  // lazy: P stays <= 2^8 otherwise
             }
             if (named_or_128(exceed)) {
@@ -586,8 +598,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         }
         if (ok && n == 0) {
             if (t < C) {  // no tile came to this CTA: weight 0 in the merge
-                part_ml[(col_row(t) + s) * 2 + 0] = -INFINITY;
-                part_ml[(col_row(t) + s) * 2 + 1] = 0.f;
+                part_ml[(crow[t] + s) * 2 + 0] = -INFINITY;
+                part_ml[(crow[t] + s) * 2 + 1] = 0.f;
             }
         } else if (ok) {
             // (PVDONE could be two phases behind here -- PV(n-2) may still run -- so the
@@ -609,9 +621,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     const float4 l4 = reinterpret_cast<const float4*>(ls)[h];
                     const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
                     if (nsplit == 1) {
-                        out[out_row(h) * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
+                        out[orow[h] * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
                     } else {
-                        const size_t row = col_row(h) + s;
+                        const size_t row = crow[h] + s;
                         part_o[row * D + t] = __uint_as_float(o[h]);
                         if (t == 0) {
                             part_ml[row * 2 + 0] = m_run[h];
@@ -654,9 +666,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             float2* wml = reinterpret_cast<float2*>(gb + L::OFF_K);
             float* winv = reinterpret_cast<float*>(gb + L::OFF_K + NH * 256 * 8);
             float* racc = winv + NH;
-            const int npair = C * nsplit;
-            for (int p = tid; p < npair; p += kThreads)  // pair p = (column p / nsplit, split p % nsplit)
-                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + col_row(p / nsplit) + p % nsplit);
+            for (int p = tid; p < C * nsplit; p += kThreads) {  // pair p = (column p / nsplit, split p % nsplit)
+                const int c = p / nsplit;
+                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + crow[c] + (p - c * nsplit));
+            }
             __syncthreads();
             for (int h = warp; h < C; h += kThreads / 32) {  // per column: M, weights, 1/L
                 float mm = -INFINITY;
@@ -693,7 +706,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 for (int h = 0; h < NHP; ++h) {
                     const int hh = min(h, C - 1);
                     wgt[h] = h < C ? wml[hh * nsplit + sp].x : 0.f;
-                    o4[h] = __ldcg(reinterpret_cast<const float4*>(part_o + (col_row(hh) + sp) * D) + lane);
+                    o4[h] = __ldcg(reinterpret_cast<const float4*>(part_o + (crow[hh] + sp) * D) + lane);
                 }
 #pragma unroll
                 for (int h = 0; h < NHP; ++h) {
@@ -723,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 const uint2 packed = make_uint2(
                     to_bf16(sum.x * inv) | (static_cast<uint32_t>(to_bf16(sum.y * inv)) << 16),
                     to_bf16(sum.z * inv) | (static_cast<uint32_t>(to_bf16(sum.w * inv)) << 16));
-                *reinterpret_cast<uint2*>(out + out_row(h) * D + 4 * c) = packed;
+                *reinterpret_cast<uint2*>(out + orow[h] * D + 4 * c) = packed;
             }
         }
     }
@@ -738,9 +751,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
 }  // namespace
 
 cudaError_t configure_decode_tc() {
-    cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(decode_tc_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
+    cudaError_t e = cudaSuccess;
+    for (auto fn : {decode_tc_kernel<8, 1>, decode_tc_kernel<16, 1>, decode_tc_kernel<8, kMaxTok>,
+                    decode_tc_kernel<16, kMaxTok>})
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
     return e;
 }
 
@@ -790,7 +804,9 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     cfg.attrs = attr;
     cfg.numAttrs = after_decode ? 1 : 0;  // dependent launch only right after another decode step
     if (ntok < 1 || ntok > kMaxTok || G * ntok > NH) return cudaErrorInvalidValue;
-    return cudaLaunchKernelEx(&cfg, G * ntok <= 8 ? decode_tc_kernel<8> : decode_tc_kernel<16>, maps.k, maps.v, q,
+    const auto kernel = ntok == 1 ? (G <= 8 ? decode_tc_kernel<8, 1> : decode_tc_kernel<16, 1>)
+                                  : (G * ntok <= 8 ? decode_tc_kernel<8, kMaxTok> : decode_tc_kernel<16, kMaxTok>);
+    return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err);
 }
