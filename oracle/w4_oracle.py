@@ -1,0 +1,84 @@
+"""CPU oracle of the W4BF16 weight-only GEMV -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the bench's CPU-baseline leg use it.
+
+The paper deploys every model with W4BF16 quantization: 4-bit weights, bf16
+activations (Section 5.1), and its decode throughput is set by streaming those
+weights (Section 5.2).  The paper fixes no group size, zero-point convention or
+storage layout; the reading taken here is the common grouped asymmetric form
+(GPTQ/AWQ style): weight row n, input index k, group g = k // 128 along k, code
+q[n,k] in 0..15, zero point z[n,g] in 0..15 and bf16 scale s[n,g]:
+
+    W[n,k] = (q[n,k] - z[n,g]) * s[n,g]
+    y[m,n] = sum_k x[m,k] * W[n,k]
+
+computed here exactly in float64 from the bf16 inputs (``gemv``).
+
+Storage read by ``unpack_tiles`` (this module's own reader of the documented format):
+the matrix is cut into tiles of 16 rows x 128 inputs; tile (T, G) -- rows 16T..16T+15,
+group G -- is the (T * K/128 + G)-th record of 1072 bytes:
+  bytes    0..1023  codes: row r of the tile holds 16 little-endian uint32 words at
+                    byte 64 r; word i carries k = 128 G + 8 i + j (j = 0..7) with the
+                    nibble of j at bit offset (0, 16, 4, 20, 8, 24, 12, 28)[j]
+  bytes 1024..1055  the 16 rows' scales, bf16 bits, row r at byte 1024 + 2 r
+  bytes 1056..1071  the 16 rows' zero points, one byte each, row r at byte 1056 + r
+Rows past N in the last row-tile are padding and ignored.
+
+No arithmetic in this module is pinned by a value the paper prints: the paper gives
+no worked example of the quantized product.  The pins are the definition's own
+closed forms and brute force (tests/test_w4_oracle.py).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GROUP = 128
+TILE_ROWS = 16
+TILE_BYTES = 1072
+CODE_BYTES = 1024
+SCALE_OFFSET = 1024
+ZERO_OFFSET = 1056
+NIBBLE_SHIFT = (0, 16, 4, 20, 8, 24, 12, 28)
+
+
+def unpack_row_words(words: np.ndarray) -> np.ndarray:
+    """uint32 [..., K/8] -> codes uint8 [..., K] (the nibble order within a word)."""
+    w = np.asarray(words, dtype=np.uint32)
+    out = np.empty(w.shape[:-1] + (w.shape[-1] * 8,), dtype=np.uint8)
+    for j, sh in enumerate(NIBBLE_SHIFT):
+        out[..., j::8] = ((w >> np.uint32(sh)) & np.uint32(15)).astype(np.uint8)
+    return out
+
+
+def unpack_tiles(buf: np.ndarray, N: int, K: int):
+    """Tile stream (uint8, ceil(N/16) * K/128 * 1072 bytes) -> (codes uint8 [N, K],
+    scales bf16 bits uint16 [N, K/128], zeros uint8 [N, K/128])."""
+    ng, nt = K // GROUP, (N + TILE_ROWS - 1) // TILE_ROWS
+    b = np.asarray(buf, dtype=np.uint8)
+    assert b.size == nt * ng * TILE_BYTES
+    rec = b.reshape(nt, ng, TILE_BYTES)
+    words = rec[:, :, :CODE_BYTES].copy().view("<u4").reshape(nt, ng, TILE_ROWS, 16)
+    # [tile, group, row, word] -> [tile, row, group, word] -> rows x (K/8) words
+    words = words.transpose(0, 2, 1, 3).reshape(nt * TILE_ROWS, ng * 16)
+    scales = rec[:, :, SCALE_OFFSET:ZERO_OFFSET].copy().view("<u2").reshape(nt, ng, TILE_ROWS)
+    zeros = rec[:, :, ZERO_OFFSET:TILE_BYTES].reshape(nt, ng, TILE_ROWS)
+    scales = scales.transpose(0, 2, 1).reshape(nt * TILE_ROWS, ng)
+    zeros = zeros.transpose(0, 2, 1).reshape(nt * TILE_ROWS, ng)
+    return unpack_row_words(words)[:N], scales[:N].copy(), zeros[:N].copy()
+
+
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+def dequant(codes, scales_bf16, zeros) -> np.ndarray:
+    """W [N, K] float64 = (q - z) * s, groups of 128 along k."""
+    q = np.asarray(codes, dtype=np.float64)
+    z = np.repeat(np.asarray(zeros, dtype=np.float64), GROUP, axis=-1)
+    s = np.repeat(bf16_to_f64(scales_bf16), GROUP, axis=-1)
+    return (q - z) * s
+
+
+def gemv(codes, scales_bf16, zeros, x_bf16) -> np.ndarray:
+    """y [M, N] float64 = x [M, K] . W[N, K]^T, exactly in float64."""
+    return bf16_to_f64(x_bf16) @ dequant(codes, scales_bf16, zeros).T

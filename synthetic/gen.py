@@ -146,3 +146,17 @@ def normal_bf16(workload: str, tensor: str, shape, scale: float, seed: int = 0) 
 
 
 BF16_NAN = np.uint16(0x7FC0)
+
+
+def uint4_codes(workload: str, tensor: str, shape, seed: int = 0) -> np.ndarray:
+    """4-bit codes (0..15, uint8) of the given shape: the low four bits of the stream's outputs."""
+    n = int(np.prod(shape)) if len(shape) else 1
+    return (splitmix64_stream(tensor_key(workload, tensor, seed), 0, n) & np.uint64(15)).astype(np.uint8).reshape(shape)
+
+
+def uint32_words(workload: str, tensor: str, shape, seed: int = 0) -> np.ndarray:
+    """Uniform 32-bit words (uint32) of the given shape: the low half of the stream's outputs.
+    Read as eight 4-bit fields each, they are eight independent uniform codes."""
+    n = int(np.prod(shape)) if len(shape) else 1
+    return (splitmix64_stream(tensor_key(workload, tensor, seed), 0, n) & np.uint64(0xFFFFFFFF)).astype(
+        np.uint32).reshape(shape)
