@@ -253,6 +253,37 @@ int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_
                         const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len, uint16_t* k_cache,
                         uint16_t* v_cache, uint16_t* out, int32_t* d_err, attn_stream_t stream);
 
+/* W4BF16 weight-only matrix-vector product of the decode stage (Section 5.1: the
+ * models run with 4-bit weights and bf16 activations; Section 5.2: decode speed is
+ * the rate at which the weights stream from memory).  For m < M, n < N:
+ *   y[m][n] = bf16( sum_{k<K} x[m][k] * (q[n][k] - z[n][k/128]) * s[n][k/128] )
+ * with the sum formed in float (products exact, sums rounded), y rounded to nearest.
+ *   w_tiles device, 16-byte aligned: the [N, K] weight matrix as ceil(N/16) * (K/128)
+ *           records of ATTN_W4_TILE_BYTES (1072) bytes, record T * (K/128) + G holding
+ *           rows 16T..16T+15 of input group G (k = 128G .. 128G+127):
+ *             bytes    0..1023  codes, tile row r at byte 64 r as 16 little-endian uint32
+ *                               words; word i holds k = 128G + 8i + j (j = 0..7), the
+ *                               4-bit code of j at bit (0,16,4,20,8,24,12,28)[j];
+ *             bytes 1024..1055  the 16 rows' scales s, bf16, row r at byte 1024 + 2r;
+ *             bytes 1056..1071  the 16 rows' zero points z (0..15), row r at 1056 + r.
+ *           Rows past N in the last row-tile are ignored.
+ *   x       device, bf16 [M][K], 16-byte aligned.   y: device, bf16 [M][N].
+ *   d_err   device int32 or NULL: a wait of the kernel that runs out (a copy that never
+ *           lands) sets ATTN_DEVERR_TIMEOUT in it and leaves y undefined.
+ * K a positive multiple of 128 with attn_w4bf16_rows_per_launch(K) >= 1; any M >= 1,
+ * N >= 1.  One launch serves attn_w4bf16_rows_per_launch(K) rows of x (x is staged in
+ * shared memory); further rows take further passes over the weights.  Enqueued on
+ * `stream`; nothing is allocated or synchronised; buffers stay the caller's.
+ * Returns ATTN_OK, ATTN_EINVAL (null pointer, bad size or alignment), ATTN_EARCH
+ * or ATTN_ECUDA. */
+#define ATTN_W4_TILE_BYTES 1072
+int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
+                     attn_stream_t stream);
+
+/* Rows of x one attn_w4bf16_gemv launch serves for inner size K: 8, 4, 2 or 1, or 0
+ * when K is not a positive multiple of 128 or too large to stage (host only). */
+int attn_w4bf16_rows_per_launch(int K);
+
 /* Static text for an ATTN_* code. */
 const char* attn_strerror(int code);
 

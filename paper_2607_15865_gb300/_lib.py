@@ -18,7 +18,8 @@ DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
             "attn_decode_multi", "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_timing_enable", "attn_timing_read",
-            "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc")
+            "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc", "attn_w4bf16_gemv",
+            "attn_w4bf16_rows_per_launch")
 NOALLOC_SCRATCH_FLOATS = 1 << 20
 KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
 
@@ -77,6 +78,10 @@ def load(path: str = LIB_PATH):
     lib.attn_decode_noalloc.argtypes = [ctypes.POINTER(AttnCfg), vp, vp, u16p, u16p, u16p, vp, u16p, u16p, u16p,
                                         vp, vp]
     lib.attn_decode_noalloc.restype = i32
+    lib.attn_w4bf16_gemv.argtypes = [vp, u16p, i32, i32, i32, u16p, vp, vp]
+    lib.attn_w4bf16_gemv.restype = i32
+    lib.attn_w4bf16_rows_per_launch.argtypes = [i32]
+    lib.attn_w4bf16_rows_per_launch.restype = i32
     lib.attn_strerror.argtypes = [i32]
     lib.attn_strerror.restype = ctypes.c_char_p
     lib.attn_last_cuda_error_string.argtypes = []

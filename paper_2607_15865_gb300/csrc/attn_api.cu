@@ -14,6 +14,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -54,6 +55,10 @@ struct attn_ctx {
 namespace {
 
 thread_local char g_cuda_msg[256] = "no error";
+
+// Per device: whether it is an sm_103 part (attn_w4bf16_gemv checks once per device).
+constexpr int kArchCacheDevices = 64;
+std::atomic<int> g_arch_ok[kArchCacheDevices];
 
 int cuda_fail(cudaError_t e, const char* where) {
     std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
@@ -434,6 +439,42 @@ int attn_timing_read(attn_ctx* c, double* ms, long long* launches) {
         c->launches[k] = 0;
     }
     c->ev_used = 0;
+    return ATTN_OK;
+}
+
+int attn_w4bf16_rows_per_launch(int K) { return K >= 128 && K % 128 == 0 ? attn::w4_gemv_max_rows(K) : 0; }
+
+int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
+                     attn_stream_t stream) {
+    if (w_tiles == nullptr || x == nullptr || y == nullptr) return ATTN_EINVAL;
+    if (M < 1 || N < 1 || K < 128 || K % 128 != 0) return ATTN_EINVAL;
+    const int rows = attn::w4_gemv_max_rows(K);
+    if (rows < 1) return ATTN_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(w_tiles) & 15u) || (reinterpret_cast<uintptr_t>(x) & 15u) ||
+        (reinterpret_cast<uintptr_t>(y) & 1u) || (reinterpret_cast<uintptr_t>(d_err) & 3u))
+        return ATTN_EINVAL;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "attn_w4bf16_gemv device query");
+    if (dev < 0 || dev >= kArchCacheDevices) return ATTN_EINVAL;
+    int arch = g_arch_ok[dev].load(std::memory_order_relaxed);  // 0 unknown, 1 sm_103, 2 other
+    if (arch == 0) {
+        int major = 0, minor = 0;
+        e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "attn_w4bf16_gemv device query");
+        arch = major == 10 && minor == 3 ? 1 : 2;
+        g_arch_ok[dev].store(arch, std::memory_order_relaxed);
+    }
+    if (arch != 1) return ATTN_EARCH;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // Rows of x past what one launch stages take further passes over the weights.
+    for (int m0 = 0; m0 < M; m0 += rows) {
+        const int mc = std::min(rows, M - m0);
+        e = attn::launch_w4_gemv(static_cast<const uint8_t*>(w_tiles), x + static_cast<size_t>(m0) * K, mc, N, K,
+                                 y + static_cast<size_t>(m0) * N, d_err, st);
+        if (e != cudaSuccess) return cuda_fail(e, "w4_gemv");
+    }
     return ATTN_OK;
 }
 

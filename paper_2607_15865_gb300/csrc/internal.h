@@ -88,6 +88,16 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
                                   const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
 
+// W4BF16 GEMV (w4_gemv.cu): y[m, n] = sum_k x[m, k] (q[n, k] - z[n, k/128]) s[n, k/128] for
+// the 1 <= M <= w4_gemv_max_rows(K) activation rows of one launch.  tiles: the tile
+// stream of attn_w4bf16_gemv (16-byte aligned); x: bf16 [M][K] (16-byte aligned);
+// y: bf16 [M][N].  K a multiple of 128.  A launch stages x and its group sums in the
+// shared memory its rings leave free.  A bounded wait that runs out sets
+// kDevErrTimeout in *err (when err is not null).
+int w4_gemv_max_rows(int K);  // 8, 4, 2, 1 or 0 (K too large)
+cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
+                           cudaStream_t st);
+
 #ifdef __CUDACC__
 // Position of sequence b's decode token: d_hist[b] + hist_add, or -1 (out of range, so
 // the caller flags and skips the sequence) when the sum leaves int.
