@@ -21,6 +21,9 @@ stages    per-stage times; prefill stages in TFLOP/s, decode in HBM GB/s.
 cpu_baseline  the CPU oracle on a bounded row sample of the same step.
 
 --impl reference times the CPU oracle (the reference arm of this path) instead.
+--sweep times every configuration's stages, the stage driver, decode loops, the
+multi-token decode and the W4BF16 decode GEMV; --stage / --w4 M,N,K only run one
+stage or one GEMV shape (the launch pattern of a profiler capture).
 Multi-GPU (torchrun): every rank runs its own replica of the workload (weak
 scaling, no collective on the data path); value is the whole-job aggregate.
 """
@@ -650,6 +653,49 @@ def run_sweep(args):
             rows.append({"config": label, "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
         attn.close()
         del kc, vc
+    # W4BF16 decode GEMV (the weight stream of the paper's W4BF16 decode): one large matrix
+    # (268 MB of tiles, beyond L2) at 1 and 8 rows of x, and the 128 GEMVs of a 7B-class
+    # decode step (32 layers x qkv, o, gate_up, down; 3.4 GB of tiles) replayed from one
+    # CUDA graph.  Bytes = tiles + x + y.
+    from paper_2607_15865_gb300.w4 import TILE_BYTES, w4bf16_gemv
+
+    def w4_inputs(M, N, K):
+        nrec = (N + 15) // 16 * (K // 128)
+        tiles = torch.randint(0, 256, (nrec, TILE_BYTES), dtype=torch.uint8, device=dev, generator=gen)
+        tiles[:, 1024:1056].view(torch.int16).fill_(0x3C00)  # scales 2^-7
+        tiles[:, 1056:] &= 15
+        x = rnd((M, K), gen)
+        return tiles.view(-1), x, torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+
+    def w4_bytes(M, N, K):
+        return (N + 15) // 16 * (K // 128) * TILE_BYTES + 2 * M * K + 2 * M * N
+
+    for M in (1, 8):
+        N, K = 65536, 8192
+        tiles, x, y = w4_inputs(M, N, K)
+        ms = time_calls(lambda: w4bf16_gemv(tiles, x, N, out=y), args.sweep_reps)
+        gbs = w4_bytes(M, N, K) / (ms * 1e-3) / 1e9
+        rows.append({"config": f"W4BF16 GEMV M={M} N={N} K={K}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+        del tiles, x, y
+    layer = [(12288, 4096), (4096, 4096), (22016, 4096), (4096, 11008)]
+    for M in (1, 4):
+        mats = [w4_inputs(M, N, K) + (N,) for N, K in layer * 32]
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            for tiles, x, y, N in mats:
+                w4bf16_gemv(tiles, x, N, out=y, stream=side)
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+            for tiles, x, y, N in mats:
+                w4bf16_gemv(tiles, x, N, out=y, stream=side)
+        torch.cuda.synchronize()
+        ms = time_calls(gr.replay, args.sweep_reps)
+        gbs = sum(w4_bytes(M, N, K) for N, K in layer * 32) / (ms * 1e-3) / 1e9
+        rows.append({"config": f"W4BF16 7B-class decode step M={M}: 128 GEMVs (CUDA graph)", "ms": ms, "GB/s": gbs,
+                     "frac_hbm": gbs / hbm})
+        del mats, gr
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)
@@ -704,6 +750,33 @@ def run_stage(args):
     return 0 if flags == 0 else 1
 
 
+def run_w4_stage(args):
+    """Runs the W4BF16 GEMV of --w4 M,N,K --warmup + --reps times on random tiles (no
+    timing, no JSON line): the launch pattern of a profiler capture of that kernel."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.w4 import TILE_BYTES, w4bf16_gemv
+    M, N, K = (int(v) for v in args.w4.split(","))
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    g = torch.Generator(device=dev).manual_seed(3)
+    tiles = torch.randint(0, 256, ((N + 15) // 16 * (K // 128), TILE_BYTES), dtype=torch.uint8, device=dev,
+                          generator=g)
+    tiles[:, 1024:1056].view(torch.int16).fill_(0x3C00)
+    tiles[:, 1056:] &= 15
+    x = (torch.randn(M, K, device=dev, generator=g)).to(torch.bfloat16)
+    y = torch.empty((M, N), dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    for _ in range(args.warmup + args.reps):
+        w4bf16_gemv(tiles.view(-1), x, N, out=y, err=err)
+    torch.cuda.synchronize()
+    flags = int(err.item())
+    print(f"w4 GEMV M={M} N={N} K={K}: {args.warmup} + {args.reps} calls, device error word {flags}")
+    return 0 if flags == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -720,9 +793,12 @@ def main():
     ap.add_argument("--reps", type=int, default=2)
     ap.add_argument("--hist", type=int)
     ap.add_argument("--chunk", type=int)
+    ap.add_argument("--w4", help="M,N,K: run only the W4BF16 GEMV of that shape (for profiler captures)")
     args = ap.parse_args()
     if args.stage:  # no timing in this mode
         return run_stage(args)
+    if args.w4:
+        return run_w4_stage(args)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
