@@ -270,15 +270,23 @@ int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_
  *   x       device, bf16 [M][K], 16-byte aligned.   y: device, bf16 [M][N].
  *   d_err   device int32 or NULL: a wait of the kernel that runs out (a copy that never
  *           lands) sets ATTN_DEVERR_TIMEOUT in it and leaves y undefined.
+ *   flags   0 or ATTN_W4_WEIGHTS_STATIC.  The kernel is launched as a programmatic
+ *           dependent of the kernel before it on `stream`: it reads x and writes y only
+ *           after that kernel has finished, and lets the kernel after it begin early.
+ *           With ATTN_W4_WEIGHTS_STATIC it also starts reading w_tiles before the
+ *           previous kernel has finished, so a chain of calls streams the next matrix
+ *           during the previous call's last CTAs: set it only when the kernel right
+ *           before this call on the stream does not write w_tiles.
  * K a positive multiple of 128 with attn_w4bf16_rows_per_launch(K) >= 1; any M >= 1,
  * N >= 1.  One launch serves attn_w4bf16_rows_per_launch(K) rows of x (x is staged in
  * shared memory); further rows take further passes over the weights.  Enqueued on
  * `stream`; nothing is allocated or synchronised; buffers stay the caller's.
- * Returns ATTN_OK, ATTN_EINVAL (null pointer, bad size or alignment), ATTN_EARCH
+ * Returns ATTN_OK, ATTN_EINVAL (null pointer, bad size, alignment or flag), ATTN_EARCH
  * or ATTN_ECUDA. */
 #define ATTN_W4_TILE_BYTES 1072
+#define ATTN_W4_WEIGHTS_STATIC 1
 int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
-                     attn_stream_t stream);
+                     int flags, attn_stream_t stream);
 
 /* Rows of x one attn_w4bf16_gemv launch serves for inner size K: 8, 4, 2 or 1, or 0
  * when K is not a positive multiple of 128 or too large to stage (host only). */

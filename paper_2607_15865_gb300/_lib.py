@@ -14,6 +14,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libattn_gb300.so")
 
 ATTN_OK, ATTN_EINVAL, ATTN_EARCH, ATTN_ECUDA, ATTN_ENOMEM, ATTN_EDEVICE = 0, -1, -2, -3, -4, -5
+W4_WEIGHTS_STATIC = 1
 DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
@@ -78,7 +79,7 @@ def load(path: str = LIB_PATH):
     lib.attn_decode_noalloc.argtypes = [ctypes.POINTER(AttnCfg), vp, vp, u16p, u16p, u16p, vp, u16p, u16p, u16p,
                                         vp, vp]
     lib.attn_decode_noalloc.restype = i32
-    lib.attn_w4bf16_gemv.argtypes = [vp, u16p, i32, i32, i32, u16p, vp, vp]
+    lib.attn_w4bf16_gemv.argtypes = [vp, u16p, i32, i32, i32, u16p, vp, i32, vp]
     lib.attn_w4bf16_gemv.restype = i32
     lib.attn_w4bf16_rows_per_launch.argtypes = [i32]
     lib.attn_w4bf16_rows_per_launch.restype = i32

@@ -445,8 +445,9 @@ int attn_timing_read(attn_ctx* c, double* ms, long long* launches) {
 int attn_w4bf16_rows_per_launch(int K) { return K >= 128 && K % 128 == 0 ? attn::w4_gemv_max_rows(K) : 0; }
 
 int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
-                     attn_stream_t stream) {
+                     int flags, attn_stream_t stream) {
     if (w_tiles == nullptr || x == nullptr || y == nullptr) return ATTN_EINVAL;
+    if (flags & ~ATTN_W4_WEIGHTS_STATIC) return ATTN_EINVAL;
     if (M < 1 || N < 1 || K < 128 || K % 128 != 0) return ATTN_EINVAL;
     const int rows = attn::w4_gemv_max_rows(K);
     if (rows < 1) return ATTN_EINVAL;
@@ -472,7 +473,8 @@ int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K
     for (int m0 = 0; m0 < M; m0 += rows) {
         const int mc = std::min(rows, M - m0);
         e = attn::launch_w4_gemv(static_cast<const uint8_t*>(w_tiles), x + static_cast<size_t>(m0) * K, mc, N, K,
-                                 y + static_cast<size_t>(m0) * N, d_err, st);
+                                 y + static_cast<size_t>(m0) * N, d_err, (flags & ATTN_W4_WEIGHTS_STATIC) != 0,
+                                 st);
         if (e != cudaSuccess) return cuda_fail(e, "w4_gemv");
     }
     return ATTN_OK;

@@ -31,7 +31,13 @@
 //     8 / KS units, KS warps per unit on a KS-th of its groups each, and the partial
 //     sums meet in shared memory;
 //   * a warp's first copies are issued before x is staged, so the prologue overlaps the
-//     weight stream.
+//     weight stream;
+//   * launched as a programmatic dependent of the previous kernel on the stream: every
+//     read of data that kernel may write (x) and every write (y) comes after
+//     griddepcontrol.wait, and each CTA lets the next kernel start once it has begun.  With
+//     early_weights the first weight copies are issued before the wait too (the caller
+//     promises the previous kernel does not write the tiles), so a chain of GEMVs streams
+//     the next matrix while the last CTAs of the previous one finish.
 // Every wait is bounded: a tile that never lands sets ATTN_DEVERR_TIMEOUT in *err (when
 // err is not null) and the warp stops decoding.
 #include <cuda_bf16.h>
@@ -145,7 +151,8 @@ __device__ __forceinline__ void decode_tile(const uint8_t* st, const uint2* xb, 
 template <int MT>
 __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __restrict__ tiles,
                                                            const uint16_t* __restrict__ x, int M, int N, int K,
-                                                           int KS, uint16_t* __restrict__ y, int* err) {
+                                                           int KS, uint16_t* __restrict__ y, int* err,
+                                                           int early_weights) {
     extern __shared__ __align__(1024) uint8_t smem[];
     const int ngroup = K / 128;
     const uint32_t ring = smem_u32(smem);
@@ -156,6 +163,7 @@ __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __rest
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, t = lane & 3;
 
+    if (!early_weights) griddep_wait();
     // each warp's ring: barriers, then its first kStages - 1 copies, in flight while x is staged
     if (lane == 0) {
         for (int s = 0; s < kStages; ++s) mbar_init(bars + 8 * (warp * kStages + s), 1);
@@ -196,6 +204,8 @@ __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __rest
         }
     };
     for (int s = 0; s < kStages - 1 && ivalid; ++s) issue();
+    if (early_weights) griddep_wait();  // x and y belong to the stream order from here on
+    griddep_launch_dependents();
 
     // x in fragment order (asynchronous 8-byte copies, rows past M zero)
     const uint32_t xfrag_s = smem_u32(xfrag);
@@ -306,7 +316,7 @@ int g_occ[kMaxDevices][4] = {};
 
 template <int MT>
 cudaError_t launch_t(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
-                     cudaStream_t st) {
+                     bool early_weights, cudaStream_t st) {
     constexpr int mi = MT == 1 ? 0 : MT == 2 ? 1 : MT == 4 ? 2 : 3;
     auto kern = w4_gemv_kernel<MT>;
     const size_t smem = smem_bytes(MT, K);
@@ -361,8 +371,17 @@ cudaError_t launch_t(const uint8_t* tiles, const uint16_t* x, int M, int N, int 
         }
     }
     const unsigned grid = static_cast<unsigned>(best_blocks < grid_max ? best_blocks : grid_max);
-    kern<<<grid, kThreads, smem, st>>>(tiles, x, M, N, K, best_ks, y, err);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, tiles, x, M, N, K, best_ks, y, err, early_weights ? 1 : 0);
 }
 
 }  // namespace
@@ -376,11 +395,11 @@ int w4_gemv_max_rows(int K) {
 }
 
 cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
-                           cudaStream_t st) {
-    if (M <= 1) return launch_t<1>(tiles, x, M, N, K, y, err, st);
-    if (M <= 2) return launch_t<2>(tiles, x, M, N, K, y, err, st);
-    if (M <= 4) return launch_t<4>(tiles, x, M, N, K, y, err, st);
-    return launch_t<8>(tiles, x, M, N, K, y, err, st);
+                           bool early_weights, cudaStream_t st) {
+    if (M <= 1) return launch_t<1>(tiles, x, M, N, K, y, err, early_weights, st);
+    if (M <= 2) return launch_t<2>(tiles, x, M, N, K, y, err, early_weights, st);
+    if (M <= 4) return launch_t<4>(tiles, x, M, N, K, y, err, early_weights, st);
+    return launch_t<8>(tiles, x, M, N, K, y, err, early_weights, st);
 }
 
 }  // namespace attn

@@ -63,10 +63,13 @@ def pack_tiles(words: np.ndarray, scales: np.ndarray, zeros: np.ndarray) -> np.n
     return out.reshape(-1)
 
 
-def w4bf16_gemv(tiles: torch.Tensor, x: torch.Tensor, N: int, out=None, stream=None, err=None) -> torch.Tensor:
+def w4bf16_gemv(tiles: torch.Tensor, x: torch.Tensor, N: int, out=None, stream=None, err=None,
+                weights_static: bool = False) -> torch.Tensor:
     """y [M, N] (bf16) = x [M, K] . W^T for the tile stream of an [N, K] matrix (a uint8
     CUDA tensor from pack_tiles) and x bf16 [M, K] on the same device.  err: optional
-    int32 CUDA tensor whose bit ATTN_DEVERR_TIMEOUT the kernel sets when a wait runs out."""
+    int32 CUDA tensor whose bit ATTN_DEVERR_TIMEOUT the kernel sets when a wait runs out.
+    weights_static: the kernel right before this call on the stream does not write the
+    tiles, so the call may start streaming them before that kernel has finished."""
     lib = _lib.load()
     M, K = x.shape
     for t, name in ((tiles, "tiles"), (x, "x")):
@@ -83,7 +86,8 @@ def w4bf16_gemv(tiles: torch.Tensor, x: torch.Tensor, N: int, out=None, stream=N
     if err is not None and not (isinstance(err, torch.Tensor) and err.is_cuda and err.dtype == torch.int32):
         raise TypeError("err must be an int32 CUDA tensor")
     rc = lib.attn_w4bf16_gemv(tiles.data_ptr(), x.data_ptr(), M, N, K, out.data_ptr(),
-                              None if err is None else err.data_ptr(), _stream(stream))
+                              None if err is None else err.data_ptr(),
+                              _lib.W4_WEIGHTS_STATIC if weights_static else 0, _stream(stream))
     if rc != _lib.ATTN_OK:
         raise _lib.AttnError(rc, "attn_w4bf16_gemv", lib)
     return out

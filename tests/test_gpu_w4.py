@@ -158,12 +158,58 @@ def test_w4_gemv_rejects_bad_arguments(torch):
     lib = _lib.load()
     buf = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
     p = buf.data_ptr()
-    ok = lib.attn_w4bf16_gemv(p, p, 1, 8, 128, p + 65536, p + 131072, None)
+    ok = lib.attn_w4bf16_gemv(p, p, 1, 8, 128, p + 65536, p + 131072, 0, None)
     assert ok == _lib.ATTN_OK
-    for args in [(None, p, 1, 8, 128, p, None), (p, None, 1, 8, 128, p, None), (p, p, 1, 8, 128, None, None),
-                 (p, p, 0, 8, 128, p, None), (p, p, 1, 0, 128, p, None), (p, p, 1, 8, 64, p, None),
-                 (p, p, 1, 8, 200, p, None), (p, p, 1, 8, k_max() + 128, p, None), (p + 8, p, 1, 8, 128, p, None),
-                 (p, p + 8, 1, 8, 128, p, None), (p, p, 1, 8, 128, p + 1, None), (p, p, 1, 8, 128, p, p + 2)]:
+    for args in [(None, p, 1, 8, 128, p, None, 0), (p, None, 1, 8, 128, p, None, 0), (p, p, 1, 8, 128, None, None, 0),
+                 (p, p, 0, 8, 128, p, None, 0), (p, p, 1, 0, 128, p, None, 0), (p, p, 1, 8, 64, p, None, 0),
+                 (p, p, 1, 8, 200, p, None, 0), (p, p, 1, 8, k_max() + 128, p, None, 0),
+                 (p + 8, p, 1, 8, 128, p, None, 0), (p, p + 8, 1, 8, 128, p, None, 0),
+                 (p, p, 1, 8, 128, p + 1, None, 0), (p, p, 1, 8, 128, p, p + 2, 0), (p, p, 1, 8, 128, p, None, 2)]:
         assert lib.attn_w4bf16_gemv(*args, None) == _lib.ATTN_EINVAL, args
     torch.cuda.synchronize()
     assert int(buf[131072:131076].view(torch.int32).item()) == 0
+
+
+@pytest.mark.parametrize("weights_static", [False, True])
+def test_w4_gemv_chain_feeds_each_output_forward(torch, weights_static):
+    """A chain of GEMVs where each call's x is the previous call's y (dependent launches,
+    in a CUDA graph and eagerly): every output against the oracle applied to the input the
+    GPU actually fed it.  With weights_static the next matrix is streamed before the
+    previous call finishes; x and y must still follow the stream order."""
+    from paper_2607_15865_gb300.w4 import pack_codes, pack_tiles, w4bf16_gemv
+    M, dims = 2, [1024, 3072, 512, 2048, 1024]
+    layers = []
+    for i in range(len(dims) - 1):
+        K, N = dims[i], dims[i + 1]
+        codes, zeros, scales, _ = make(f"chain{i}", 1, N, K)
+        tiles = torch.from_numpy(pack_tiles(pack_codes(codes), scales, zeros)).cuda()
+        layers.append((codes, zeros, scales, tiles, N))
+    x0 = make("chain_x", M, 8, dims[0])[3]
+    xs = [torch.from_numpy(x0.view(np.int16)).cuda().view(torch.bfloat16)]
+    xs += [torch.empty((M, n), dtype=torch.bfloat16, device="cuda") for n in dims[1:]]
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+    def chain(stream):
+        for i, (_, _, _, tiles, N) in enumerate(layers):
+            w4bf16_gemv(tiles, xs[i], N, out=xs[i + 1], stream=stream, err=err, weights_static=weights_static)
+
+    def check_all():
+        torch.cuda.synchronize()
+        assert int(err.item()) == 0
+        for i, (codes, zeros, scales, _, _) in enumerate(layers):
+            xin = xs[i].view(torch.int16).cpu().numpy().view(np.uint16)
+            yout = xs[i + 1].view(torch.int16).cpu().numpy().view(np.uint16)
+            check(codes, zeros, scales, xin, yout)
+
+    chain(None)
+    check_all()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+        chain(side)
+    torch.cuda.current_stream().wait_stream(side)
+    for t in xs[1:]:
+        t.fill_(float("nan"))
+    gr.replay()
+    check_all()
