@@ -697,6 +697,50 @@ def run_sweep(args):
         rows.append({"config": f"W4BF16 7B-class decode step M={M}: 128 GEMVs (CUDA graph, {tag})", "ms": ms,
                      "GB/s": gbs, "frac_hbm": gbs / hbm})
         del mats, gr
+    # The attention half of a decoder block with W4BF16 weights (attn_decode_layer: RMSNorm ->
+    # stacked QKV GEMV -> decode attention -> o_proj + residual), 32 layers of an 8B-class
+    # model (hidden 4096, Hq 32, Hkv 8, D 128) at 4096 valid tokens, one CUDA graph.  Bytes =
+    # the weights' tile streams + the K/V history read + the new K/V and the activations.
+    lsh = w.decode_shape(1)
+    for bsz in (1, 4):
+        sh = Shape(f"layer_b{bsz}", bsz, lsh.n_q_heads, lsh.n_kv_heads, lsh.head_dim, lsh.max_len, lsh.rope_theta)
+        hidden, hist, nl = 4096, 4096, 32
+        qd, kd = sh.n_q_heads * sh.head_dim, sh.n_kv_heads * sh.head_dim
+        attn = Attention.for_shape(sh)
+        gamma = (1.0 + 0.1 * torch.randn(hidden, device=dev, generator=gen)).to(torch.bfloat16)
+        x = torch.randn(bsz, hidden, device=dev, generator=gen).to(torch.bfloat16)
+        hl = torch.full((bsz,), hist, dtype=torch.int32, device=dev)
+        layers_ = []
+        for _ in range(nl):
+            tq = w4_inputs(1, qd + 2 * kd, hidden)[0]
+            to = w4_inputs(1, hidden, qd)[0]
+            kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+            vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+            layers_.append((tq, to, kc, vc))
+
+        def block_step(stream=None):
+            h = x
+            for tq, to, kc, vc in layers_:
+                h = attn.decode_layer(h, gamma, 1e-6, tq, to, hl, kc, vc, weights_static=True, stream=stream)
+            return h
+
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            block_step(side)
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+            block_step(side)
+        torch.cuda.synchronize()
+        ms = time_calls(gr.replay, args.sweep_reps)
+        byts = nl * (w4_bytes(bsz, qd + 2 * kd, hidden) + w4_bytes(bsz, hidden, qd) +
+                     decode_bytes(sh, hist) + 2 * bsz * hidden * 2)
+        gbs = byts / (ms * 1e-3) / 1e9
+        rows.append({"config": f"W4BF16 attention half of 32 decoder blocks B{bsz} hist {hist} (CUDA graph)",
+                     "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+        attn.close()
+        del layers_, gr
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)

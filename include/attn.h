@@ -288,6 +288,42 @@ int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_
 int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
                      int flags, attn_stream_t stream);
 
+/* attn_w4bf16_gemv with the parts of Listing 1's block around the product fused in (each
+ * optional):
+ *   rms_gamma  NULL, or device bf16 [K], 8-byte aligned: x is replaced by RMSNorm(x):
+ *              x * r * gamma rounded to bf16, r = 1 / sqrt(mean over k of x^2 + rms_eps),
+ *              in float, per row of x (0 <= rms_eps < 1);
+ *   residual   NULL, or device bf16 [M][N]: added to the product in float before the
+ *              rounding of y (it may be y itself: each element is read before it is written);
+ *   y1, y2     NULL (y is [M][N]), or both set with 0 < n_split0 < n_split1 < N: columns
+ *              [0, n_split0) go to y as [M][n_split0], [n_split0, n_split1) to y1 as
+ *              [M][n_split1 - n_split0] and [n_split1, N) to y2 as [M][N - n_split1] (q, k
+ *              and v of a stacked QKV projection).
+ * The other arguments and the errors are those of attn_w4bf16_gemv. */
+int attn_w4bf16_gemv_fused(const void* w_tiles, const uint16_t* x, int M, int N, int K, const uint16_t* rms_gamma,
+                           float rms_eps, const uint16_t* residual, uint16_t* y, int n_split0, uint16_t* y1,
+                           int n_split1, uint16_t* y2, int32_t* d_err, int flags, attn_stream_t stream);
+
+/* One decode step of the attention half of a decoder block (Listing 1: input_layernorm,
+ * q/k/v projections, RoPE, attention, o_proj + residual) with W4BF16 weights, for the
+ * context's shape (B = batch sequences, one new token each):
+ *   x           device bf16 [B][hidden], 16-byte aligned: the block's input (residual stream);
+ *   rms_gamma   device bf16 [hidden], 8-byte aligned; rms_eps: see attn_w4bf16_gemv_fused;
+ *   wqkv_tiles  the tile stream (attn_w4bf16_gemv) of the stacked [(Hq + 2 Hkv) D, hidden]
+ *               matrix: rows of q_proj, then k_proj, then v_proj;
+ *   wo_tiles    the tile stream of o_proj, [hidden, Hq D];
+ *   hidden      a multiple of 128 (as is Hq D);
+ *   d_hist_len, k_cache, v_cache: as in attn_decode (the new k and v are appended);
+ *   h_out       device bf16 [B][hidden]: x + o_proj(attention); may be x itself.
+ * q, k, v and the attention output live in buffers of the context; the step enqueues the
+ * fused QKV GEMV, the decode kernels and the o_proj GEMV on `stream` (flags applies to the
+ * QKV GEMV, as in attn_w4bf16_gemv; the o_proj GEMV always streams its weights early).  A
+ * GEMV wait that runs out sets ATTN_DEVERR_TIMEOUT in the context's error word
+ * (attn_device_error).  Returns ATTN_OK, ATTN_EINVAL, ATTN_EARCH or ATTN_ECUDA. */
+int attn_decode_layer(attn_ctx* ctx, const uint16_t* x, const uint16_t* rms_gamma, float rms_eps,
+                      const void* wqkv_tiles, const void* wo_tiles, int hidden, const int32_t* d_hist_len,
+                      uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, int flags, attn_stream_t stream);
+
 /* Rows of x one attn_w4bf16_gemv launch serves for inner size K: 8, 4, 2 or 1, or 0
  * when K is not a positive multiple of 128 or too large to stage (host only). */
 int attn_w4bf16_rows_per_launch(int K);

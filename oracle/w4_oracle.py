@@ -25,8 +25,8 @@ group G -- is the (T * K/128 + G)-th record of 1072 bytes:
 Rows past N in the last row-tile are padding and ignored.
 
 No arithmetic in this module is pinned by a value the paper prints: the paper gives
-no worked example of the quantized product.  The pins are the definition's own
-closed forms and brute force (tests/test_w4_oracle.py).
+no worked example of the quantized product or of the block around attention.  The pins
+are the definitions' own closed forms and brute force (tests/test_w4_oracle.py).
 """
 from __future__ import annotations
 
@@ -82,3 +82,47 @@ def dequant(codes, scales_bf16, zeros) -> np.ndarray:
 def gemv(codes, scales_bf16, zeros, x_bf16) -> np.ndarray:
     """y [M, N] float64 = x [M, K] . W[N, K]^T, exactly in float64."""
     return bf16_to_f64(x_bf16) @ dequant(codes, scales_bf16, zeros).T
+
+
+# ----------------------------------------------------------------------------- the block around attention
+# Listing 1's attention half of a decoder block, for one decode step with W4BF16 weights:
+#   xn = RMSNorm(x) * gamma                    (input_layernorm)
+#   q | k | v = xn . Wqkv^T                    (q_proj, k_proj, v_proj stacked by rows)
+#   o = attention(RoPE(q), RoPE(k) -> cache, v -> cache)   (the decode stage)
+#   h = x + o . Wo^T                           (o_proj + residual)
+# Readings (the paper gives the dataflow only): RMSNorm r = 1 / sqrt(mean(x^2) + eps) per row
+# and x * r * gamma rounded once to bf16; q, k, v and o are bf16 (the stage's inputs and
+# output); the residual is added before h is rounded to bf16.
+
+
+def to_bf16_bits(v) -> np.ndarray:
+    """float64 -> bf16 bits, round to nearest, ties to even (finite values in the normal range)."""
+    a = np.asarray(v, dtype=np.float64)
+    assert np.isfinite(a).all()
+    m, e = np.frexp(a)                     # a = m * 2^e, 0.5 <= |m| < 1
+    r = np.ldexp(np.rint(np.ldexp(m, 8)), e - 8)  # 8 significant bits, ties to even
+    return (r.astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+def rmsnorm(x_bf16, gamma_bf16, eps: float) -> np.ndarray:
+    """bf16 bits [M, K] -> bf16 bits of x * r * gamma, r = 1 / sqrt(mean_k x^2 + eps) per row."""
+    x = bf16_to_f64(x_bf16)
+    r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)
+    return to_bf16_bits(x * r * bf16_to_f64(gamma_bf16))
+
+
+def decode_layer(shape, x_bf16, gamma_bf16, eps, wqkv, wo, hist, k_cache, v_cache, attn_oracle=None):
+    """h (bf16 bits [B, hidden]) of one decode step; wqkv / wo are (codes, scales, zeros) of the
+    stacked [(Hq + 2 Hkv) D, hidden] and the [hidden, Hq D] matrices.  The caches get the new k
+    (rotated) and v at slot hist[b], as the decode stage does."""
+    if attn_oracle is None:
+        from oracle import oracle as attn_oracle
+    B, D = shape.batch, shape.head_dim
+    qd, kd = shape.n_q_heads * D, shape.n_kv_heads * D
+    xn = rmsnorm(x_bf16, gamma_bf16, eps)
+    qkv = to_bf16_bits(gemv(*wqkv, xn))
+    q = qkv[:, :qd].reshape(B, 1, shape.n_q_heads, D)
+    k = qkv[:, qd:qd + kd].reshape(B, 1, shape.n_kv_heads, D)
+    v = qkv[:, qd + kd:].reshape(B, 1, shape.n_kv_heads, D)
+    o = attn_oracle.decode(shape, q, k, v, hist, k_cache, v_cache).reshape(B, qd)
+    return to_bf16_bits(bf16_to_f64(x_bf16) + gemv(*wo, o))

@@ -137,6 +137,31 @@ class Attention:
         self._check(rc, "attn_decode_multi")
         return out
 
+    def decode_layer(self, x, rms_gamma, rms_eps: float, wqkv_tiles, wo_tiles, hist_len: torch.Tensor, k_cache,
+                     v_cache, out=None, weights_static: bool = False, stream=None) -> torch.Tensor:
+        """One decode step of the attention half of a decoder block with W4BF16 weights
+        (attn_decode_layer): x [B, hidden] -> x + o_proj(attention(qkv_proj(RMSNorm(x))))."""
+        hidden = x.shape[-1]
+        if not (isinstance(hist_len, torch.Tensor) and hist_len.is_cuda and hist_len.dtype == torch.int32
+                and hist_len.is_contiguous() and tuple(hist_len.shape) == (self.batch,)):
+            raise TypeError("hist_len must be a contiguous int32 CUDA tensor of shape [batch]")
+        for t, name in ((wqkv_tiles, "wqkv_tiles"), (wo_tiles, "wo_tiles")):
+            if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous() and t.dtype == torch.uint8):
+                raise TypeError(f"{name} must be a contiguous uint8 CUDA tensor (a W4BF16 tile stream)")
+        qd, kd = self.n_q_heads * self.head_dim, self.n_kv_heads * self.head_dim
+        if wqkv_tiles.numel() != (qd + 2 * kd + 15) // 16 * (hidden // 128) * 1072 or \
+                wo_tiles.numel() != (hidden + 15) // 16 * (qd // 128) * 1072:
+            raise ValueError("tile streams must hold [(Hq + 2 Hkv) D, hidden] and [hidden, Hq D] matrices")
+        xs = (self.batch, hidden)
+        out = self._new_out(x, out)
+        rc = self.lib.attn_decode_layer(self._ctx, _ptr(x, "x", xs), _ptr(rms_gamma, "rms_gamma", (hidden,)),
+                                        float(rms_eps), wqkv_tiles.data_ptr(), wo_tiles.data_ptr(), hidden,
+                                        hist_len.data_ptr(), _ptr(k_cache, "k_cache", self._cache_shape()),
+                                        _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", xs),
+                                        _lib.W4_WEIGHTS_STATIC if weights_static else 0, _stream(stream))
+        self._check(rc, "attn_decode_layer")
+        return out
+
     def prompt(self, q, k, v, hist_len: int, seg_len: int, k_cache, v_cache, out=None,
                stream=None) -> torch.Tensor:
         """The whole prompt q [B,P,Hq,D], k/v [B,P,Hkv,D] at positions hist_len.. in segments of seg_len."""

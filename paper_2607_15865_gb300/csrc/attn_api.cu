@@ -37,6 +37,10 @@ struct attn_ctx {
     float* d_part_o;
     float* d_part_ml;
     int* d_counters;    // decode counters, [2][B * Hkv] (merge count, tile claims), zero between launches
+    uint16_t* d_lq;     // decode layer: q, k, v of the fused QKV projection and the attention
+    uint16_t* d_lk;     // output, bf16 [B][Hq*D], [B][Hkv*D], [B][Hkv*D], [B][Hq*D]
+    uint16_t* d_lv;
+    uint16_t* d_lo;
     float* d_flash_o;   // flash tail pieces: [num_sms * 256, D] partial O
     float* d_flash_ml;  // and [num_sms * 256, 2] (m, l)
     int* d_err;
@@ -231,6 +235,12 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     oom |= cudaMalloc(&c->d_flash_o, piece_rows * cfg->head_dim * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_flash_ml, piece_rows * 2 * sizeof(float)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_err, sizeof(int)) != cudaSuccess;
+    const size_t qd = static_cast<size_t>(cfg->batch) * cfg->n_q_heads * cfg->head_dim;
+    const size_t kd = static_cast<size_t>(cfg->batch) * cfg->n_kv_heads * cfg->head_dim;
+    oom |= cudaMalloc(&c->d_lq, qd * sizeof(uint16_t)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_lk, kd * sizeof(uint16_t)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_lv, kd * sizeof(uint16_t)) != cudaSuccess;
+    oom |= cudaMalloc(&c->d_lo, qd * sizeof(uint16_t)) != cudaSuccess;
     const size_t n_counters = 2 * static_cast<size_t>(cfg->batch) * cfg->n_kv_heads;  // merge + tile claims
     oom |= cudaMalloc(&c->d_counters, n_counters * sizeof(int)) != cudaSuccess;
     if (oom) {
@@ -267,6 +277,10 @@ void attn_destroy(attn_ctx* c) {
     cudaFree(c->d_flash_ml);
     cudaFree(c->d_err);
     cudaFree(c->d_counters);
+    cudaFree(c->d_lq);
+    cudaFree(c->d_lk);
+    cudaFree(c->d_lv);
+    cudaFree(c->d_lo);
     delete c;
 }
 
@@ -444,16 +458,29 @@ int attn_timing_read(attn_ctx* c, double* ms, long long* launches) {
 
 int attn_w4bf16_rows_per_launch(int K) { return K >= 128 && K % 128 == 0 ? attn::w4_gemv_max_rows(K) : 0; }
 
-int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
-                     int flags, attn_stream_t stream) {
+int attn_w4bf16_gemv_fused(const void* w_tiles, const uint16_t* x, int M, int N, int K, const uint16_t* rms_gamma,
+                           float rms_eps, const uint16_t* residual, uint16_t* y, int n_split0, uint16_t* y1,
+                           int n_split1, uint16_t* y2, int32_t* d_err, int flags, attn_stream_t stream) {
     if (w_tiles == nullptr || x == nullptr || y == nullptr) return ATTN_EINVAL;
     if (flags & ~ATTN_W4_WEIGHTS_STATIC) return ATTN_EINVAL;
     if (M < 1 || N < 1 || K < 128 || K % 128 != 0) return ATTN_EINVAL;
     const int rows = attn::w4_gemv_max_rows(K);
     if (rows < 1) return ATTN_EINVAL;
     if ((reinterpret_cast<uintptr_t>(w_tiles) & 15u) || (reinterpret_cast<uintptr_t>(x) & 15u) ||
-        (reinterpret_cast<uintptr_t>(y) & 1u) || (reinterpret_cast<uintptr_t>(d_err) & 3u))
+        (reinterpret_cast<uintptr_t>(y) & 1u) || (reinterpret_cast<uintptr_t>(d_err) & 3u) ||
+        (reinterpret_cast<uintptr_t>(rms_gamma) & 7u) || (reinterpret_cast<uintptr_t>(residual) & 1u) ||
+        (reinterpret_cast<uintptr_t>(y1) & 1u) || (reinterpret_cast<uintptr_t>(y2) & 1u))
         return ATTN_EINVAL;
+    if (rms_gamma != nullptr && !(rms_eps >= 0.f && rms_eps < 1.f)) return ATTN_EINVAL;
+    attn::W4Fused fz{rms_gamma, rms_eps, residual, N, N, nullptr, nullptr};
+    if (y1 != nullptr || y2 != nullptr) {
+        if (y1 == nullptr || y2 == nullptr || !(0 < n_split0 && n_split0 < n_split1 && n_split1 < N))
+            return ATTN_EINVAL;
+        fz.n0 = n_split0;
+        fz.n1 = n_split1;
+        fz.y1 = y1;
+        fz.y2 = y2;
+    }
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_fail(e, "attn_w4bf16_gemv device query");
@@ -472,12 +499,46 @@ int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K
     // Rows of x past what one launch stages take further passes over the weights.
     for (int m0 = 0; m0 < M; m0 += rows) {
         const int mc = std::min(rows, M - m0);
-        e = attn::launch_w4_gemv(static_cast<const uint8_t*>(w_tiles), x + static_cast<size_t>(m0) * K, mc, N, K,
-                                 y + static_cast<size_t>(m0) * N, d_err, (flags & ATTN_W4_WEIGHTS_STATIC) != 0,
-                                 st);
+        attn::W4Fused f = fz;
+        const size_t r0 = static_cast<size_t>(m0);
+        if (f.residual != nullptr) f.residual += r0 * N;
+        if (f.y1 != nullptr) {
+            f.y1 += r0 * (f.n1 - f.n0);
+            f.y2 += r0 * (N - f.n1);
+        }
+        e = attn::launch_w4_gemv(static_cast<const uint8_t*>(w_tiles), x + r0 * K, mc, N, K, y + r0 * fz.n0, d_err,
+                                 (flags & ATTN_W4_WEIGHTS_STATIC) != 0, f, st);
         if (e != cudaSuccess) return cuda_fail(e, "w4_gemv");
     }
     return ATTN_OK;
+}
+
+int attn_decode_layer(attn_ctx* c, const uint16_t* x, const uint16_t* rms_gamma, float rms_eps,
+                      const void* wqkv_tiles, const void* wo_tiles, int hidden, const int32_t* d_hist_len,
+                      uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, int flags, attn_stream_t stream) {
+    if (c == nullptr || x == nullptr || rms_gamma == nullptr || wqkv_tiles == nullptr || wo_tiles == nullptr ||
+        h_out == nullptr)
+        return ATTN_EINVAL;
+    const int B = c->cfg.batch;
+    const int qd = c->cfg.n_q_heads * c->cfg.head_dim, kd = c->cfg.n_kv_heads * c->cfg.head_dim;
+    if (hidden < 128 || hidden % 128 != 0 || qd % 128 != 0) return ATTN_EINVAL;
+    // input_layernorm + q/k/v projections (one GEMV over the stacked rows, split three ways)
+    int rc = attn_w4bf16_gemv_fused(wqkv_tiles, x, B, qd + 2 * kd, hidden, rms_gamma, rms_eps, nullptr, c->d_lq, qd,
+                                    c->d_lk, qd + kd, c->d_lv, c->d_err, flags, stream);
+    if (rc != ATTN_OK) return rc;
+    // RoPE of q and k, cache append, attention over the history (the decode stage)
+    rc = run_decode(c, c->d_lq, c->d_lk, c->d_lv, d_hist_len, 0, false, k_cache, v_cache, c->d_lo,
+                    reinterpret_cast<cudaStream_t>(stream));
+    if (rc != ATTN_OK) return rc;
+    // o_proj + residual; the decode kernels never write the weights, so they may stream early
+    return attn_w4bf16_gemv_fused(wo_tiles, c->d_lo, B, hidden, qd, nullptr, 0.f, x, h_out, 0, nullptr, 0, nullptr,
+                                  c->d_err, ATTN_W4_WEIGHTS_STATIC, stream);
+}
+
+int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
+                     int flags, attn_stream_t stream) {
+    return attn_w4bf16_gemv_fused(w_tiles, x, M, N, K, nullptr, 0.f, nullptr, y, 0, nullptr, 0, nullptr, d_err, flags,
+                                  stream);
 }
 
 const char* attn_strerror(int code) {

@@ -95,10 +95,22 @@ cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int his
 // shared memory its rings leave free.  A bounded wait that runs out sets
 // kDevErrTimeout in *err (when err is not null).
 int w4_gemv_max_rows(int K);  // 8, 4, 2, 1 or 0 (K too large)
+// Fused parts of a GEMV (all optional): RMSNorm of x before the product (gamma: bf16 [K],
+// 8-byte aligned), a residual added before rounding (bf16 [M][N]), and the output columns
+// split three ways: [0, n0) -> y (row stride n0), [n0, n1) -> y1, [n1, N) -> y2 (no split:
+// n0 = n1 = N).
+struct W4Fused {
+    const uint16_t* gamma;
+    float eps;
+    const uint16_t* residual;
+    int n0, n1;
+    uint16_t* y1;
+    uint16_t* y2;
+};
 // The launch is a programmatic dependent of the stream's previous kernel; early_weights lets
 // it read the tiles before that kernel has finished (see attn_w4bf16_gemv).
 cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
-                           bool early_weights, cudaStream_t st);
+                           bool early_weights, const W4Fused& fz, cudaStream_t st);
 
 #ifdef __CUDACC__
 // Position of sequence b's decode token: d_hist[b] + hist_add, or -1 (out of range, so

@@ -32,6 +32,10 @@
 //     sums meet in shared memory;
 //   * a warp's first copies are issued before x is staged, so the prologue overlaps the
 //     weight stream;
+//   * fused around the product (Listing 1's block): an optional RMSNorm of x, applied to
+//     the staged copy before the group sums; an optional residual added in f32 before the
+//     bf16 rounding; and an optional split of the output columns into three arrays (q, k
+//     and v of a fused QKV projection);
 //   * launched as a programmatic dependent of the previous kernel on the stream: every
 //     read of data that kernel may write (x) and every write (y) comes after
 //     griddepcontrol.wait, and each CTA lets the next kernel start once it has begun.  With
@@ -152,7 +156,7 @@ template <int MT>
 __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __restrict__ tiles,
                                                            const uint16_t* __restrict__ x, int M, int N, int K,
                                                            int KS, uint16_t* __restrict__ y, int* err,
-                                                           int early_weights) {
+                                                           int early_weights, W4Fused fz) {
     extern __shared__ __align__(1024) uint8_t smem[];
     const int ngroup = K / 128;
     const uint32_t ring = smem_u32(smem);
@@ -219,6 +223,41 @@ __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __rest
     }
     cp_async_wait_all();
     __syncthreads();
+    if (fz.gamma != nullptr) {
+        // RMSNorm of each row of x (Listing 1 "input_layernorm"): r = 1 / sqrt(mean(x^2) + eps),
+        // then x * r * gamma rounded to bf16 in place.  A thread's fragment slot, and so its row,
+        // is the same for all its elements (the stride divides by 4 * MT).
+        const int slot = tid % (4 * MT), m = slot >> 2;
+        float ss = 0.f;
+        for (int i = tid; i < ngroup * 8 * 4 * MT; i += kThreads) {
+            const uint2 v = xfrag[i];
+            const float a = bf16_lo(v.x), b = bf16_hi(v.x), c = bf16_lo(v.y), d = bf16_hi(v.y);
+            ss = fmaf(a, a, fmaf(b, b, fmaf(c, c, fmaf(d, d, ss))));
+        }
+        // lanes of one row: those that differ in the two low lane bits or in bits >= 4 * MT
+        ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 1);
+        ss += __shfl_xor_sync(0xFFFFFFFFu, ss, 2);
+        for (int off = 4 * MT; off < 32; off <<= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+        if ((lane & 3) == 0 && lane < 4 * MT) red[warp * 8 + m] = ss;
+        __syncthreads();
+        if (tid < MT) {
+            float tot = 0.f;
+            for (int w = 0; w < kWarps; ++w) tot += red[w * 8 + tid];
+            red[kWarps * 8 + tid] = 1.f / sqrtf(tot / static_cast<float>(K) + fz.eps);
+        }
+        __syncthreads();
+        const float r = red[kWarps * 8 + m];
+        for (int i = tid; i < ngroup * 8 * 4 * MT; i += kThreads) {
+            if (m >= M) break;
+            const int ge = i / (4 * MT), e = ge & 7, G = ge >> 3, tt = slot & 3;
+            const int k0 = 128 * G + 32 * tt + 8 * (e >> 1) + 4 * (e & 1);
+            const uint2 gm = *reinterpret_cast<const uint2*>(fz.gamma + k0);
+            const uint2 v = xfrag[i];
+            xfrag[i] = make_uint2(pack_bf16x2(bf16_lo(v.x) * r * bf16_lo(gm.x), bf16_hi(v.x) * r * bf16_hi(gm.x)),
+                                  pack_bf16x2(bf16_lo(v.y) * r * bf16_lo(gm.y), bf16_hi(v.y) * r * bf16_hi(gm.y)));
+        }
+        __syncthreads();
+    }
     // group sums of x, one (group, row) per thread
     for (int i = tid; i < ngroup * 8; i += kThreads) {
         const int G = i >> 3, m = i & 7;
@@ -287,9 +326,16 @@ __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __rest
             const int r0 = unit * kUnitRows + g, n0 = 2 * t;
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
+                // weight row `row` is output column `row` of x row `n`
                 const int row = r0 + ((v & 2) ? 8 : 0), n = n0 + (v & 1);
-                if (n < M && row < N)
-                    y[static_cast<size_t>(n) * N + row] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[v]));
+                if (n < M && row < N) {
+                    float o = acc[v];
+                    if (fz.residual != nullptr) o += bf16_lo(fz.residual[static_cast<size_t>(n) * N + row]);
+                    uint16_t* dst = row < fz.n0   ? y + static_cast<size_t>(n) * fz.n0 + row
+                                    : row < fz.n1 ? fz.y1 + static_cast<size_t>(n) * (fz.n1 - fz.n0) + (row - fz.n0)
+                                                  : fz.y2 + static_cast<size_t>(n) * (N - fz.n1) + (row - fz.n1);
+                    *dst = __bfloat16_as_ushort(__float2bfloat16_rn(o));
+                }
             }
         }
     }
@@ -316,7 +362,7 @@ int g_occ[kMaxDevices][4] = {};
 
 template <int MT>
 cudaError_t launch_t(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
-                     bool early_weights, cudaStream_t st) {
+                     bool early_weights, const W4Fused& fz, cudaStream_t st) {
     constexpr int mi = MT == 1 ? 0 : MT == 2 ? 1 : MT == 4 ? 2 : 3;
     auto kern = w4_gemv_kernel<MT>;
     const size_t smem = smem_bytes(MT, K);
@@ -381,7 +427,7 @@ cudaError_t launch_t(const uint8_t* tiles, const uint16_t* x, int M, int N, int 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, tiles, x, M, N, K, best_ks, y, err, early_weights ? 1 : 0);
+    return cudaLaunchKernelEx(&cfg, kern, tiles, x, M, N, K, best_ks, y, err, early_weights ? 1 : 0, fz);
 }
 
 }  // namespace
@@ -395,11 +441,11 @@ int w4_gemv_max_rows(int K) {
 }
 
 cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
-                           bool early_weights, cudaStream_t st) {
-    if (M <= 1) return launch_t<1>(tiles, x, M, N, K, y, err, early_weights, st);
-    if (M <= 2) return launch_t<2>(tiles, x, M, N, K, y, err, early_weights, st);
-    if (M <= 4) return launch_t<4>(tiles, x, M, N, K, y, err, early_weights, st);
-    return launch_t<8>(tiles, x, M, N, K, y, err, early_weights, st);
+                           bool early_weights, const W4Fused& fz, cudaStream_t st) {
+    if (M <= 1) return launch_t<1>(tiles, x, M, N, K, y, err, early_weights, fz, st);
+    if (M <= 2) return launch_t<2>(tiles, x, M, N, K, y, err, early_weights, fz, st);
+    if (M <= 4) return launch_t<4>(tiles, x, M, N, K, y, err, early_weights, fz, st);
+    return launch_t<8>(tiles, x, M, N, K, y, err, early_weights, fz, st);
 }
 
 }  // namespace attn

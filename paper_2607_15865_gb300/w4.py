@@ -91,3 +91,40 @@ def w4bf16_gemv(tiles: torch.Tensor, x: torch.Tensor, N: int, out=None, stream=N
     if rc != _lib.ATTN_OK:
         raise _lib.AttnError(rc, "attn_w4bf16_gemv", lib)
     return out
+
+
+def w4bf16_gemv_fused(tiles: torch.Tensor, x: torch.Tensor, N: int, rms_gamma=None, rms_eps: float = 0.0,
+                      residual=None, out=None, split=None, stream=None, err=None,
+                      weights_static: bool = False):
+    """w4bf16_gemv with the fused parts of attn_w4bf16_gemv_fused: RMSNorm of x by rms_gamma
+    (bf16 [K]), a residual (bf16 [M, N]) added before rounding, and split = (n0, n1) to return
+    the output columns as three tensors [M, n0], [M, n1 - n0], [M, N - n1]."""
+    lib = _lib.load()
+    M, K = x.shape
+    for t, name in ((tiles, "tiles"), (x, "x")):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()):
+            raise TypeError(f"{name} must be a contiguous CUDA tensor")
+    if x.dtype != torch.bfloat16 or tiles.dtype != torch.uint8:
+        raise TypeError("dtypes: tiles uint8, x bf16")
+    if K % 128 or tiles.numel() != (N + TILE_ROWS - 1) // TILE_ROWS * (K // 128) * TILE_BYTES:
+        raise ValueError("tiles must hold ceil(N/16) * (K/128) records of 1072 bytes, K a multiple of 128")
+    for t, name, shape in ((rms_gamma, "rms_gamma", (K,)), (residual, "residual", (M, N))):
+        if t is not None and not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()
+                                  and t.dtype == torch.bfloat16 and tuple(t.shape) == shape):
+            raise TypeError(f"{name} must be a contiguous CUDA bf16 tensor of shape {shape}")
+    if split is None:
+        outs = [torch.empty((M, N), dtype=x.dtype, device=x.device) if out is None else out]
+        n0 = n1 = 0
+    else:
+        n0, n1 = split
+        outs = [torch.empty((M, w), dtype=x.dtype, device=x.device) for w in (n0, n1 - n0, N - n1)]
+    if err is not None and not (isinstance(err, torch.Tensor) and err.is_cuda and err.dtype == torch.int32):
+        raise TypeError("err must be an int32 CUDA tensor")
+    ptr = (lambda t: None if t is None else t.data_ptr())
+    rc = lib.attn_w4bf16_gemv_fused(tiles.data_ptr(), x.data_ptr(), M, N, K, ptr(rms_gamma), float(rms_eps),
+                                    ptr(residual), outs[0].data_ptr(), n0, ptr(outs[1]) if split else None, n1,
+                                    ptr(outs[2]) if split else None, ptr(err),
+                                    _lib.W4_WEIGHTS_STATIC if weights_static else 0, _stream(stream))
+    if rc != _lib.ATTN_OK:
+        raise _lib.AttnError(rc, "attn_w4bf16_gemv_fused", lib)
+    return outs[0] if split is None else tuple(outs)

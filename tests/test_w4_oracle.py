@@ -80,3 +80,92 @@ def test_gemv_closed_forms():
     four = gen.f32_to_bf16_bits(np.full((N, K // 128), 4.0, np.float32))
     rnd = gen.uint4_codes("w4pin", "cf_codes", (N, K))
     assert (W.gemv(rnd, four, zeros, x) == 4 * W.gemv(rnd, one, zeros, x)).all()
+
+
+# ----------------------------------------------------------------------------- the block around attention
+
+
+def test_bf16_rounding_is_nearest_even():
+    one = 1.0
+    cases = {one: 0x3F80, one + 2.0 ** -8: 0x3F80, one + 3 * 2.0 ** -8: 0x3F82, one + 2.0 ** -8 + 2.0 ** -30: 0x3F81,
+             -2.5: 0xC020, 0.0: 0x0000, 3.0e-30: None}
+    for v, want in cases.items():
+        got = int(W.to_bf16_bits(np.array([v]))[0])
+        if want is not None:
+            assert got == want, (v, hex(got))
+    # values exactly representable in float32: the input generator's own float32 -> bf16 rounding
+    f = (gen.normal_bf16("w4pin", "rnd_hi", (4096,), 1.0).astype(np.uint32) << np.uint32(16)).view(np.float32)
+    f = f + (gen.uint4_codes("w4pin", "rnd_lo", (4096,)).astype(np.float32) - 7.5) * np.abs(f) * 2.0 ** -10
+    assert (W.to_bf16_bits(f.astype(np.float64)) == gen.f32_to_bf16_bits(f)).all()
+
+
+def test_rmsnorm_brute_force_and_closed_forms():
+    M, K = 2, 256
+    x = gen.normal_bf16("w4pin", "rms_x", (M, K), 1.0)
+    g = gen.normal_bf16("w4pin", "rms_g", (K,), 0.3)
+    xf, gf = W.bf16_to_f64(x), W.bf16_to_f64(g)
+    got = W.rmsnorm(x, g, 1e-6)
+    for m in range(M):
+        ss = 0.0
+        for k in range(K):
+            ss += float(xf[m, k]) ** 2
+        r = 1.0 / (ss / K + 1e-6) ** 0.5
+        want = W.to_bf16_bits(np.array([float(xf[m, k]) * r * float(gf[k]) for k in range(K)]))
+        assert (got[m] == want).all()
+    # a constant row c: x * r = sign(c) exactly (eps = 0), so the output is +-gamma
+    c = gen.f32_to_bf16_bits(np.array([[-3.0] * K, [0.375] * K], np.float32))
+    out = W.rmsnorm(c, g, 0.0)
+    assert (out[0] == (g ^ np.uint16(0x8000))).all() and (out[1] == g).all()
+    # scaling x by a power of two changes nothing (eps = 0)
+    x4 = gen.f32_to_bf16_bits((W.bf16_to_f64(x) * 4.0).astype(np.float32))
+    assert (W.rmsnorm(x4, g, 0.0) == W.rmsnorm(x, g, 0.0)).all()
+
+
+def _layer_case(shape, tag, q_zero=False, wo_kind="random"):
+    """Inputs of one decode-layer step for the pins: (x, gamma, wqkv, wo, hist, caches)."""
+    from synthetic import workloads as w
+    D, hq, hkv = shape.head_dim, shape.n_q_heads, shape.n_kv_heads
+    qd, kd, hidden = hq * D, hkv * D, hq * D
+    B = shape.batch
+    x = gen.normal_bf16("w4pin", f"{tag}_x", (B, hidden), 1.0)
+    gamma = gen.normal_bf16("w4pin", f"{tag}_g", (hidden,), 1.0)
+    zq = gen.uint4_codes("w4pin", f"{tag}_zq", (qd + 2 * kd, hidden // 128)) % 15
+    cq = gen.uint4_codes("w4pin", f"{tag}_cq", (qd + 2 * kd, hidden))
+    if q_zero:
+        cq[:qd] = np.repeat(zq[:qd], 128, axis=1)
+    sq = gen.normal_bf16("w4pin", f"{tag}_sq", (qd + 2 * kd, hidden // 128), 0.02) & np.uint16(0x7FFF)
+    zo = gen.uint4_codes("w4pin", f"{tag}_zo", (hidden, qd // 128)) % 15
+    so = gen.normal_bf16("w4pin", f"{tag}_so", (hidden, qd // 128), 0.02) & np.uint16(0x7FFF)
+    if wo_kind == "zero":
+        co = np.repeat(zo, 128, axis=1)
+    elif wo_kind == "identity":
+        co = np.repeat(zo, 128, axis=1)
+        co[np.arange(hidden), np.arange(hidden)] += 1
+        so = gen.f32_to_bf16_bits(np.ones((hidden, qd // 128), np.float32))
+    else:
+        co = gen.uint4_codes("w4pin", f"{tag}_co", (hidden, qd))
+    hist = np.array([37 + 50 * b for b in range(B)], np.int32)
+    kc, vc = w.cache(shape, f"{tag}_cache", int(hist.max()), fill="random")
+    return x, gamma, (cq, sq, zq), (co, so, zo), hist, kc, vc
+
+
+def test_decode_layer_residual_only_when_o_proj_is_zero():
+    from synthetic.workloads import Shape
+    shape = Shape("w4layer_a", 2, 4, 2, 64, 256, 1.0e4)
+    x, gamma, wqkv, wo, hist, kc, vc = _layer_case(shape, "lz", wo_kind="zero")
+    h = W.decode_layer(shape, x, gamma, 1e-6, wqkv, wo, hist, kc, vc)
+    assert (h == x).all()
+
+
+def test_decode_layer_with_q_zero_and_identity_o_proj_averages_v():
+    """q = 0 makes every score equal, so attention returns the plain mean of the visible v rows
+    (the new one included); with o_proj = I the block returns x + that mean."""
+    from synthetic.workloads import Shape
+    shape = Shape("w4layer_b", 2, 4, 2, 64, 256, 1.0e4)
+    x, gamma, wqkv, wo, hist, kc, vc = _layer_case(shape, "lq", q_zero=True, wo_kind="identity")
+    h = W.decode_layer(shape, x, gamma, 1e-6, wqkv, wo, hist, kc, vc)
+    G, D = shape.n_q_heads // shape.n_kv_heads, shape.head_dim
+    for b in range(shape.batch):
+        o = np.concatenate([W.bf16_to_f64(vc[b, hq // G, :hist[b] + 1]).mean(axis=0) for hq in range(shape.n_q_heads)])
+        want = W.to_bf16_bits(W.bf16_to_f64(x[b]) + W.bf16_to_f64(W.to_bf16_bits(o)))
+        assert (h[b] == want).all()
