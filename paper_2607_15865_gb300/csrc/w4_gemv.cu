@@ -120,6 +120,8 @@ __host__ __device__ constexpr size_t smem_bytes(int MT, int K) {
 
 // One tile: D = sum over the group of (128 + q) x on the tensor cores, then
 // acc += s * (D - (128 + z) * sum of x) for rows (g, g + 8) x columns (2t, 2t + 1).
+// xb points at this lane's B fragments; lanes g >= MT read those of lane g mod MT, which
+// only fills output columns >= MT, never stored.
 template <int MT>
 __device__ __forceinline__ void decode_tile(const uint8_t* st, const uint2* xb, const float* xs_g, int g, int t,
                                             uint32_t mask, uint32_t magic, float (&acc)[4]) {
@@ -132,8 +134,8 @@ __device__ __forceinline__ void decode_tile(const uint8_t* st, const uint2* xb, 
     for (int i = 0; i < 4; ++i) {
         const uint32_t w0 = i == 0 ? c0.x : i == 1 ? c0.y : i == 2 ? c0.z : c0.w;
         const uint32_t w8 = i == 0 ? c8.x : i == 1 ? c8.y : i == 2 ? c8.z : c8.w;
-        const uint2 b0 = g < MT ? xb[(2 * i) * 4 * MT] : make_uint2(0u, 0u);
-        const uint2 b1 = g < MT ? xb[(2 * i + 1) * 4 * MT] : make_uint2(0u, 0u);
+        const uint2 b0 = xb[(2 * i) * 4 * MT];
+        const uint2 b1 = xb[(2 * i + 1) * 4 * MT];
         mma_bf16_16816(da, code_pair(w0, 0, mask, magic), code_pair(w8, 0, mask, magic), code_pair(w0, 1, mask, magic),
                        code_pair(w8, 1, mask, magic), b0.x, b0.y);
         mma_bf16_16816(db, code_pair(w0, 2, mask, magic), code_pair(w8, 2, mask, magic), code_pair(w0, 3, mask, magic),
@@ -297,11 +299,17 @@ __global__ void __launch_bounds__(kThreads) w4_gemv_kernel(const uint8_t* __rest
                     --outstanding;
                     const uint8_t* st = smem + (my_ring - ring) + cslot * kStageBytes;
                     const int nt = min(kTilesPerStage, g1 - G);
+                    const uint2* xb = xfrag + static_cast<size_t>(G) * 8 * 4 * MT + (lane & (4 * MT - 1));
+                    if (nt == kTilesPerStage) {
 #pragma unroll
-                    for (int tt = 0; tt < kTilesPerStage; ++tt)
-                        if (tt < nt)
-                            decode_tile<MT>(st + tt * kTileBytes, xfrag + static_cast<size_t>(G + tt) * 8 * 4 * MT + lane,
-                                            xsum + (G + tt) * 8, g, t, kPairMask, magic, acc);
+                        for (int tt = 0; tt < kTilesPerStage; ++tt)
+                            decode_tile<MT>(st + tt * kTileBytes, xb + tt * 8 * 4 * MT, xsum + (G + tt) * 8, g, t,
+                                            kPairMask, magic, acc);
+                    } else {
+                        for (int tt = 0; tt < nt; ++tt)
+                            decode_tile<MT>(st + tt * kTileBytes, xb + tt * 8 * 4 * MT, xsum + (G + tt) * 8, g, t,
+                                            kPairMask, magic, acc);
+                    }
                     cslot = cslot + 1 == kStages ? 0 : cslot + 1;
                     if (cslot == 0) cphase ^= 1u;
                 }
