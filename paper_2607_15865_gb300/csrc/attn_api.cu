@@ -303,9 +303,12 @@ namespace {
 // One decode step of ntok new tokens per sequence at positions d_hist_len[b] + hist_add + i.
 // after_decode: the previous launch on `st` was this context's decode of the same caches
 // (a decode loop).
+// producer_early: the previous launch wrote q, k and v and nothing the decode streams (the
+// fused QKV GEMV of attn_decode_layer); the head_dim 128 decode then starts its K/V stream as
+// a dependent launch before that kernel has finished.
 int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, const int32_t* d_hist_len,
                int hist_add, bool after_decode, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out, cudaStream_t st,
-               int ntok = 1) {
+               int ntok = 1, bool producer_early = false) {
     if (c == nullptr || q == nullptr || k == nullptr || v == nullptr || d_hist_len == nullptr ||
         k_cache == nullptr || v_cache == nullptr || out == nullptr)
         return ATTN_EINVAL;
@@ -332,7 +335,7 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
-                                          c->d_err, after_decode, ntok, st);
+                                          c->d_err, after_decode, ntok, st, producer_early);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
     });
@@ -528,7 +531,7 @@ int attn_decode_layer(attn_ctx* c, const uint16_t* x, const uint16_t* rms_gamma,
     if (rc != ATTN_OK) return rc;
     // RoPE of q and k, cache append, attention over the history (the decode stage)
     rc = run_decode(c, c->d_lq, c->d_lk, c->d_lv, d_hist_len, 0, false, k_cache, v_cache, c->d_lo,
-                    reinterpret_cast<cudaStream_t>(stream));
+                    reinterpret_cast<cudaStream_t>(stream), 1, true);
     if (rc != ATTN_OK) return rc;
     // o_proj + residual; the decode kernels never write the weights, so they may stream early
     return attn_w4bf16_gemv_fused(wo_tiles, c->d_lo, B, hidden, qd, nullptr, 0.f, x, h_out, 0, nullptr, 0, nullptr,

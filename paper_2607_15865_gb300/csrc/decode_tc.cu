@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
     int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
-    uint16_t* __restrict__ out, int* __restrict__ err) {
+    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -268,8 +268,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     // Dependent launch after the previous decode step: the setup above overlaps that step's
     // tail; its cache append, merge counters and partials are read or reused only after
     // this wait.  The next step may start only after it.
-    griddep_wait();
-    griddep_launch_dependents();
+    // With producer_early (a dependent launch after the kernel that writes q and the new k/v)
+    // the TMA warp skips this wait: it reads only the lengths, the tile counters and cache
+    // tiles, which that kernel does not write (the new tokens' rows are patched in shared
+    // memory), so the history streams in while that kernel finishes.  It waits before the
+    // merge, and the CTA releases its own dependents only from threads that have waited.
+    const bool early = producer_early != 0 && warp == kWarpTma;
+    if (!early) {
+        griddep_wait();
+        griddep_launch_dependents();
+    }
 
     const bool hist_ok = hist >= 0 && hist <= max_len - ntok;
     if (!hist_ok && s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
@@ -342,6 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     mbar_wait(bar(B_VFULL0 + t % VST), static_cast<uint32_t>(t / VST) & 1u, nullptr);
             }
         }
+        if (early) griddep_wait();
     } else if (warp == kWarpMma) {
         // ------------------------------------------------------------ tcgen05 issuer (+ the new tokens)
         // Lane l handles dimensions 4l .. 4l+3 of each new token tt (slot hist + tt, rotated
@@ -789,7 +798,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
                              float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
-                             int ntok, cudaStream_t st) {
+                             int ntok, cudaStream_t st, bool producer_early) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
@@ -802,13 +811,15 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = after_decode ? 1 : 0;  // dependent launch only right after another decode step
+    // dependent launch only right after another decode step, or with producer_early
+    cfg.numAttrs = (after_decode || producer_early) ? 1 : 0;
     if (ntok < 1 || ntok > kMaxTok || G * ntok > NH) return cudaErrorInvalidValue;
     const auto kernel = ntok == 1 ? (G <= 8 ? decode_tc_kernel<8, 1> : decode_tc_kernel<16, 1>)
                                   : (G * ntok <= 8 ? decode_tc_kernel<8, kMaxTok> : decode_tc_kernel<16, kMaxTok>);
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
-                              s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err);
+                              s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
+                              producer_early ? 1 : 0);
 }
 
 }  // namespace attn

@@ -75,6 +75,8 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
 // previous step of a decode loop); this one then starts as a dependent launch whose
 // setup overlaps that step's tail.  Never set it after any other kernel: the inputs
 // are read before the grid waits on its predecessor.
+// producer_early: a dependent launch after a kernel that writes q / the new k, v (and
+// neither the caches, the lengths nor the counters); the K/V stream starts before the wait.
 cudaError_t configure_decode_tc();
 int decode_tc_num_splits(const Shape& s, int num_sms);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
@@ -84,7 +86,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              uint16_t* v_cache,
                              const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                              int* counters, int nsplit, uint16_t* out, int* err, bool after_decode, int ntok,
-                             cudaStream_t st);
+                             cudaStream_t st, bool producer_early = false);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
                                   const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
 
