@@ -22,8 +22,9 @@ cpu_baseline  the CPU oracle on a bounded row sample of the same step.
 
 --impl reference times the CPU oracle (the reference arm of this path) instead.
 --sweep times every configuration's stages, the stage driver, decode loops, the
-multi-token decode and the W4BF16 decode GEMV; --stage / --w4 M,N,K only run one
-stage or one GEMV shape (the launch pattern of a profiler capture).
+multi-token decode, the W4BF16 decode GEMV and decode block; --stage / --w4 M,N,K /
+--layer B,HIST only run one stage, GEMV shape or decode block (the launch pattern of a
+profiler capture).
 Multi-GPU (torchrun): every rank runs its own replica of the workload (weak
 scaling, no collective on the data path); value is the whole-job aggregate.
 """
@@ -822,6 +823,50 @@ def run_w4_stage(args):
     return 0 if flags == 0 else 1
 
 
+def run_layer_stage(args):
+    """Runs --layer B,HIST: the attention half of one 8B-class decoder block (hidden 4096,
+    Hq 32, Hkv 8, D 128) at HIST valid tokens through attn_decode_layer, --warmup + --reps
+    times (no timing, no JSON line): the launch pattern of a profiler capture."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.attention import Attention
+    from paper_2607_15865_gb300.w4 import TILE_BYTES
+    from synthetic.workloads import Shape
+    bsz, hist = (int(v) for v in args.layer.split(","))
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    g = torch.Generator(device=dev).manual_seed(3)
+    base = w.decode_shape(1)
+    sh = Shape(f"layer_b{bsz}", bsz, base.n_q_heads, base.n_kv_heads, base.head_dim, base.max_len, base.rope_theta)
+    hidden, qd, kd = 4096, sh.n_q_heads * sh.head_dim, sh.n_kv_heads * sh.head_dim
+
+    def tiles(N, K):
+        t = torch.randint(0, 256, ((N + 15) // 16 * (K // 128), TILE_BYTES), dtype=torch.uint8, device=dev, generator=g)
+        t[:, 1024:1056].view(torch.int16).fill_(0x3C00)
+        t[:, 1056:] &= 15
+        return t.view(-1)
+
+    def rnd(*shape):
+        return (torch.randn(*shape, device=dev, generator=g) * 0.0884).to(torch.bfloat16)
+
+    attn = Attention.for_shape(sh)
+    tq, to = tiles(qd + 2 * kd, hidden), tiles(hidden, qd)
+    kc = rnd(sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim)
+    vc = rnd(sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim)
+    x = torch.randn(bsz, hidden, device=dev, generator=g).to(torch.bfloat16)
+    gamma = torch.ones(hidden, device=dev, dtype=torch.bfloat16)
+    hl = torch.full((bsz,), hist, dtype=torch.int32, device=dev)
+    for _ in range(args.warmup + args.reps):
+        attn.decode_layer(x, gamma, 1e-6, tq, to, hl, kc, vc, weights_static=True)
+    torch.cuda.synchronize()
+    flags = attn.device_error()
+    attn.close()
+    print(f"decode block B{bsz} hist {hist}: {args.warmup} + {args.reps} calls, device error word {flags}")
+    return 0 if flags == 0 else 1
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -839,11 +884,14 @@ def main():
     ap.add_argument("--hist", type=int)
     ap.add_argument("--chunk", type=int)
     ap.add_argument("--w4", help="M,N,K: run only the W4BF16 GEMV of that shape (for profiler captures)")
+    ap.add_argument("--layer", help="B,HIST: run only the W4BF16 decode block (for profiler captures)")
     args = ap.parse_args()
     if args.stage:  # no timing in this mode
         return run_stage(args)
     if args.w4:
         return run_w4_stage(args)
+    if args.layer:
+        return run_layer_stage(args)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
