@@ -294,7 +294,8 @@ int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K
  *              x * r * gamma rounded to bf16, r = 1 / sqrt(mean over k of x^2 + rms_eps),
  *              in float, per row of x (0 <= rms_eps < 1);
  *   residual   NULL, or device bf16 [M][N]: added to the product in float before the
- *              rounding of y (it may be y itself: each element is read before it is written);
+ *              rounding of y (when y is not split it may be y itself: each element is read
+ *              before it is written);
  *   y1, y2     NULL (y is [M][N]), or both set with 0 < n_split0 < n_split1 < N: columns
  *              [0, n_split0) go to y as [M][n_split0], [n_split0, n_split1) to y1 as
  *              [M][n_split1 - n_split0] and [n_split1, N) to y2 as [M][N - n_split1] (q, k
