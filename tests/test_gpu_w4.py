@@ -77,6 +77,9 @@ CASES = [
     ("m1_small", 1, 64, 1024),
     ("m1_ragged_rows_and_steps", 1, 131, 4096 + 384),
     ("m1_one_group", 1, 5, 128),
+    ("m1_single_row", 1, 1, 128),
+    ("m2_fifteen_rows_of_a_tile", 2, 15, 384),
+    ("m7_seventeen_rows", 7, 17, 640),
     ("m2", 2, 100, 2048),
     ("m3_in_the_4_row_kernel", 3, 77, 1152),
     ("m4", 4, 256, 4096),
