@@ -325,6 +325,19 @@ int attn_decode_layer(attn_ctx* ctx, const uint16_t* x, const uint16_t* rms_gamm
                       const void* wqkv_tiles, const void* wo_tiles, int hidden, const int32_t* d_hist_len,
                       uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, int flags, attn_stream_t stream);
 
+/* W4BF16 weight GEMM of the prefill-side projections (Listing 1's q/k/v/o_proj over a
+ * chunk of T tokens; Section 5.1 W4BF16), on the tensor cores:
+ *   y[t][n] = bf16( sum_{k<K} x[t][k] * W[n][k] ),  W[n][k] = bf16((q - z) * s)
+ * each weight rounded once to bf16 (the decode-then-multiply reading), f32 sums.
+ *   w_tiles  the tile stream of the [N, K] matrix (format of attn_w4bf16_gemv);
+ *   x        device bf16 [T][K], 16-byte aligned;  y: device bf16 [T][N], 16-byte aligned;
+ *   d_err    device int32 or NULL: a wait that runs out sets ATTN_DEVERR_TIMEOUT in it.
+ * 1 <= T <= 65535 * 128; N and K positive multiples of 128.  Enqueued on `stream`;
+ * nothing is allocated or synchronised.  Returns ATTN_OK, ATTN_EINVAL, ATTN_EARCH or
+ * ATTN_ECUDA. */
+int attn_w4bf16_gemm(const void* w_tiles, const uint16_t* x, int T, int N, int K, uint16_t* y, int32_t* d_err,
+                     attn_stream_t stream);
+
 /* Rows of x one attn_w4bf16_gemv launch serves for inner size K: 8, 4, 2 or 1, or 0
  * when K is not a positive multiple of 128 or too large to stage (host only). */
 int attn_w4bf16_rows_per_launch(int K);

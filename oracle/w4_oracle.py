@@ -126,3 +126,20 @@ def decode_layer(shape, x_bf16, gamma_bf16, eps, wqkv, wo, hist, k_cache, v_cach
     v = qkv[:, qd + kd:].reshape(B, 1, shape.n_kv_heads, D)
     o = attn_oracle.decode(shape, q, k, v, hist, k_cache, v_cache).reshape(B, qd)
     return to_bf16_bits(bf16_to_f64(x_bf16) + gemv(*wo, o))
+
+
+# ----------------------------------------------------------------------------- prefill-side GEMM
+# For a chunk of T tokens the projections are GEMMs; their kernel decodes each weight into the
+# tensor cores' bf16 operand, so the reading there is the usual dequantize-then-multiply one:
+#   W_bf16[n, k] = bf16((q[n, k] - z[n, g]) * s[n, g])   (one rounding of each weight)
+#   Y[t, n] = sum_k x[t, k] * W_bf16[n, k]               (exact here in float64)
+
+
+def dequant_bf16(codes, scales_bf16, zeros) -> np.ndarray:
+    """bf16 bits [N, K] of (q - z) * s, each rounded once to bf16."""
+    return to_bf16_bits(dequant(codes, scales_bf16, zeros))
+
+
+def gemm_bf16w(codes, scales_bf16, zeros, x_bf16) -> np.ndarray:
+    """Y [T, N] float64 = x [T, K] . W_bf16[N, K]^T."""
+    return bf16_to_f64(x_bf16) @ bf16_to_f64(dequant_bf16(codes, scales_bf16, zeros)).T

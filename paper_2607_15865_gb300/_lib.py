@@ -20,7 +20,8 @@ DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
             "attn_decode_multi", "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_timing_enable", "attn_timing_read",
             "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc", "attn_w4bf16_gemv",
-            "attn_w4bf16_rows_per_launch", "attn_w4bf16_gemv_fused", "attn_decode_layer")
+            "attn_w4bf16_rows_per_launch", "attn_w4bf16_gemv_fused", "attn_decode_layer",
+            "attn_w4bf16_gemm")
 NOALLOC_SCRATCH_FLOATS = 1 << 20
 KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
 
@@ -86,6 +87,8 @@ def load(path: str = LIB_PATH):
     lib.attn_w4bf16_gemv_fused.restype = i32
     lib.attn_decode_layer.argtypes = [vp, u16p, u16p, ctypes.c_float, vp, vp, i32, vp, u16p, u16p, u16p, i32, vp]
     lib.attn_decode_layer.restype = i32
+    lib.attn_w4bf16_gemm.argtypes = [vp, u16p, i32, i32, i32, u16p, vp, vp]
+    lib.attn_w4bf16_gemm.restype = i32
     lib.attn_w4bf16_rows_per_launch.argtypes = [i32]
     lib.attn_w4bf16_rows_per_launch.restype = i32
     lib.attn_strerror.argtypes = [i32]

@@ -20,7 +20,8 @@ LIB = os.path.join(PKG, "libattn_gb300.so")
 # (source, object name, extra nvcc flags)
 SOURCES = [("attn_api.cu", "attn_api", []), ("rope_append.cu", "rope_append", []), ("decode.cu", "decode", []),
            ("decode_tc.cu", "decode_tc", []), ("flash_fwd.cu", "flash_fwd", []),
-           ("decode_noalloc.cu", "decode_noalloc", []), ("w4_gemv.cu", "w4_gemv", [])]
+           ("decode_noalloc.cu", "decode_noalloc", []), ("w4_gemv.cu", "w4_gemv", []),
+           ("w4_gemm.cu", "w4_gemm", [])]
 HEADERS = ["internal.h", "sm100_ptx.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

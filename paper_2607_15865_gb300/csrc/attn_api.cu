@@ -538,6 +538,32 @@ int attn_decode_layer(attn_ctx* c, const uint16_t* x, const uint16_t* rms_gamma,
                                   c->d_err, ATTN_W4_WEIGHTS_STATIC, stream);
 }
 
+int attn_w4bf16_gemm(const void* w_tiles, const uint16_t* x, int T, int N, int K, uint16_t* y, int32_t* d_err,
+                     attn_stream_t stream) {
+    if (w_tiles == nullptr || x == nullptr || y == nullptr) return ATTN_EINVAL;
+    if (T < 1 || T > 65535 * 128 || N < 128 || N % 128 != 0 || K < 128 || K % 128 != 0) return ATTN_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(w_tiles) & 15u) || (reinterpret_cast<uintptr_t>(x) & 15u) ||
+        (reinterpret_cast<uintptr_t>(y) & 15u) || (reinterpret_cast<uintptr_t>(d_err) & 3u))
+        return ATTN_EINVAL;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "attn_w4bf16_gemm device query");
+    if (dev < 0 || dev >= kArchCacheDevices) return ATTN_EINVAL;
+    int arch = g_arch_ok[dev].load(std::memory_order_relaxed);  // 0 unknown, 1 sm_103, 2 other
+    if (arch == 0) {
+        int major = 0, minor = 0;
+        e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "attn_w4bf16_gemm device query");
+        arch = major == 10 && minor == 3 ? 1 : 2;
+        g_arch_ok[dev].store(arch, std::memory_order_relaxed);
+    }
+    if (arch != 1) return ATTN_EARCH;
+    e = attn::launch_w4_gemm(static_cast<const uint8_t*>(w_tiles), x, T, N, K, y, d_err,
+                             reinterpret_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ATTN_OK : cuda_fail(e, "w4_gemm");
+}
+
 int attn_w4bf16_gemv(const void* w_tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int32_t* d_err,
                      int flags, attn_stream_t stream) {
     return attn_w4bf16_gemv_fused(w_tiles, x, M, N, K, nullptr, 0.f, nullptr, y, 0, nullptr, 0, nullptr, d_err, flags,

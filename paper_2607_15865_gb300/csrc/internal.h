@@ -114,6 +114,12 @@ struct W4Fused {
 cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N, int K, uint16_t* y, int* err,
                            bool early_weights, const W4Fused& fz, cudaStream_t st);
 
+// W4BF16 GEMM (w4_gemm.cu): y[t, n] = sum_k x[t, k] bf16((q - z) s)[n, k] for T tokens;
+// N and K multiples of 128; x bf16 [T][K] and y bf16 [T][N] 16-byte aligned; tiles: the
+// tile stream of attn_w4bf16_gemv.
+cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N, int K, uint16_t* y, int* err,
+                           cudaStream_t st);
+
 #ifdef __CUDACC__
 // Position of sequence b's decode token: d_hist[b] + hist_add, or -1 (out of range, so
 // the caller flags and skips the sequence) when the sum leaves int.

@@ -128,3 +128,28 @@ def w4bf16_gemv_fused(tiles: torch.Tensor, x: torch.Tensor, N: int, rms_gamma=No
     if rc != _lib.ATTN_OK:
         raise _lib.AttnError(rc, "attn_w4bf16_gemv_fused", lib)
     return outs[0] if split is None else tuple(outs)
+
+
+def w4bf16_gemm(tiles: torch.Tensor, x: torch.Tensor, N: int, out=None, stream=None, err=None) -> torch.Tensor:
+    """Y [T, N] (bf16) = x [T, K] . W_bf16^T on the tensor cores (attn_w4bf16_gemm), for a chunk of
+    T tokens; W_bf16 = bf16((q - z) s) from the tile stream of an [N, K] matrix."""
+    lib = _lib.load()
+    T, K = x.shape
+    for t, name in ((tiles, "tiles"), (x, "x")):
+        if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous()):
+            raise TypeError(f"{name} must be a contiguous CUDA tensor")
+    if x.dtype != torch.bfloat16 or tiles.dtype != torch.uint8:
+        raise TypeError("dtypes: tiles uint8, x bf16")
+    if K % 128 or N % 128 or tiles.numel() != N // TILE_ROWS * (K // 128) * TILE_BYTES:
+        raise ValueError("N and K multiples of 128; tiles must hold N/16 * K/128 records of 1072 bytes")
+    if out is None:
+        out = torch.empty((T, N), dtype=x.dtype, device=x.device)
+    elif out.dtype != torch.bfloat16 or tuple(out.shape) != (T, N) or not out.is_contiguous() or not out.is_cuda:
+        raise ValueError("out must be a contiguous CUDA bf16 tensor [T, N]")
+    if err is not None and not (isinstance(err, torch.Tensor) and err.is_cuda and err.dtype == torch.int32):
+        raise TypeError("err must be an int32 CUDA tensor")
+    rc = lib.attn_w4bf16_gemm(tiles.data_ptr(), x.data_ptr(), T, N, K, out.data_ptr(),
+                              None if err is None else err.data_ptr(), _stream(stream))
+    if rc != _lib.ATTN_OK:
+        raise _lib.AttnError(rc, "attn_w4bf16_gemm", lib)
+    return out

@@ -4,8 +4,8 @@ oracle fails one of them.
 Each mutant is oracle/w4_oracle.py with one plausible mistake substituted in (a wrong
 nibble order or tile transpose, a dropped zero point, a wrong group, a wrong bf16 decode
 or rounding, RMSNorm without eps or gamma or with a sum for the mean, a block without its
-residual or RMSNorm, k and v swapped, q read from the wrong rows), loaded as a separate
-module.  The real oracle is never modified.
+residual or RMSNorm, k and v swapped, q read from the wrong rows, GEMM weights not rounded),
+loaded as a separate module.  The real oracle is never modified.
 """
 import os
 import types
@@ -31,6 +31,8 @@ MUTANTS = {
     "block_without_rmsnorm": ("xn = rmsnorm(x_bf16, gamma_bf16, eps)", "xn = x_bf16"),
     "block_k_v_swapped": ("v = qkv[:, qd + kd:].reshape", "v = qkv[:, qd:qd + kd].reshape"),
     "block_q_from_wrong_rows": ("q = qkv[:, :qd].reshape", "q = qkv[:, kd:kd + qd].reshape"),
+    "gemm_weights_not_rounded": ("@ bf16_to_f64(dequant_bf16(codes, scales_bf16, zeros)).T",
+                                 "@ dequant(codes, scales_bf16, zeros).T"),
 }
 
 

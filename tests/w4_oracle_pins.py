@@ -176,4 +176,30 @@ def pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v(W):
         want = W.to_bf16_bits(W.bf16_to_f64(x[b]) + W.bf16_to_f64(W.to_bf16_bits(o)))
         assert (h[b] == want).all()
 
-ALL_PINS = [pin_packer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v]
+def pin_gemm_rounds_each_weight_once(W):
+    """The prefill-side reading: W_bf16 = bf16((q - z) s).  With power-of-two scales every
+    (q - z) s is exact, so the GEMM equals the exact product; with other scales it equals
+    Python loops over the rounded weights."""
+    T, N, K = 3, 5, 256
+    x = gen.normal_bf16("w4pin", "gm_x", (T, K), 1.0)
+    codes = gen.uint4_codes("w4pin", "gm_c", (N, K))
+    zeros = gen.uint4_codes("w4pin", "gm_z", (N, K // 128))
+    p2 = gen.f32_to_bf16_bits(np.array([[2.0 ** -(5 + (n + g) % 4) for g in range(K // 128)] for n in range(N)],
+                                       np.float32))
+    assert (W.gemm_bf16w(codes, p2, zeros, x) == W.gemv(codes, p2, zeros, x)).all()
+    s = gen.normal_bf16("w4pin", "gm_s", (N, K // 128), 0.02)
+    wb = W.dequant_bf16(codes, s, zeros)
+    sf = W.bf16_to_f64(s)
+    for n in range(N):
+        for k in range(0, K, 37):
+            v = (int(codes[n, k]) - int(zeros[n, k // 128])) * float(sf[n, k // 128])
+            assert int(wb[n, k]) == int(W.to_bf16_bits(np.array([v]))[0])
+    ref = np.zeros((T, N))
+    xf, wf = W.bf16_to_f64(x), W.bf16_to_f64(wb)
+    for t in range(T):
+        for n in range(N):
+            ref[t, n] = sum(float(xf[t, k]) * float(wf[n, k]) for k in range(K))
+    assert np.allclose(W.gemm_bf16w(codes, s, zeros, x), ref, rtol=1e-12, atol=1e-12)
+
+
+ALL_PINS = [pin_gemm_rounds_each_weight_once, pin_packer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v]
