@@ -6,7 +6,7 @@ import pytest
 import torch
 
 from paper_2607_15865_gb300 import _lib
-from paper_2607_15865_gb300.w4 import TILE_BYTES, pack_codes, pack_tiles, w4bf16_gemv, w4bf16_gemv_fused
+from paper_2607_15865_gb300.w4 import TILE_BYTES, pack_codes, pack_tiles, w4bf16_gemm, w4bf16_gemv, w4bf16_gemv_fused
 
 
 def test_wrappers_refuse_host_tensors_and_bad_shapes():
@@ -16,6 +16,8 @@ def test_wrappers_refuse_host_tensors_and_bad_shapes():
         w4bf16_gemv(tiles, x, 32)  # host tensors
     with pytest.raises(TypeError):
         w4bf16_gemv_fused(tiles, x, 32, rms_gamma=torch.ones(256, dtype=torch.bfloat16))
+    with pytest.raises(TypeError):
+        w4bf16_gemm(torch.zeros(8 * 2 * TILE_BYTES, dtype=torch.uint8), x, 128)
 
 
 def test_pack_tiles_rejects_bad_shapes():
@@ -45,3 +47,5 @@ def test_entry_points_check_arguments_before_the_device():
     assert lib.attn_w4bf16_gemv(16, 16, 1, 8, 100, 16, None, 0, None) == _lib.ATTN_EINVAL  # K % 128
     assert lib.attn_decode_layer(None, None, None, 0.0, None, None, 128, None, None, None, None, 0,
                                  None) == _lib.ATTN_EINVAL
+    assert lib.attn_w4bf16_gemm(16, 16, 1, 100, 128, 16, None, None) == _lib.ATTN_EINVAL  # N % 128
+    assert lib.attn_w4bf16_gemm(16, 16, 0, 128, 128, 16, None, None) == _lib.ATTN_EINVAL  # no tokens
