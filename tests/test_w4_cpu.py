@@ -49,3 +49,25 @@ def test_entry_points_check_arguments_before_the_device():
                                  None) == _lib.ATTN_EINVAL
     assert lib.attn_w4bf16_gemm(16, 16, 1, 100, 128, 16, None, None) == _lib.ATTN_EINVAL  # N % 128
     assert lib.attn_w4bf16_gemm(16, 16, 0, 128, 128, 16, None, None) == _lib.ATTN_EINVAL  # no tokens
+
+
+def test_tile_stream_round_trips_for_any_shape():
+    """Packer (product) and reader (oracle) agree for any row count and group count."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+    from oracle import w4_oracle as W
+
+    @hyp.settings(max_examples=40, deadline=None)
+    @hyp.given(st.integers(1, 70), st.integers(1, 5), st.integers(0, 2 ** 31 - 1))
+    def prop(N, ng, seed):
+        rng = np.random.default_rng(seed)
+        K = 128 * ng
+        codes = rng.integers(0, 16, (N, K), dtype=np.uint8)
+        scales = rng.integers(0, 1 << 16, (N, ng), dtype=np.uint16)
+        zeros = rng.integers(0, 16, (N, ng), dtype=np.uint8)
+        buf = pack_tiles(pack_codes(codes), scales, zeros)
+        assert buf.size == (N + 15) // 16 * ng * TILE_BYTES
+        c, s, z = W.unpack_tiles(buf, N, K)
+        assert (c == codes).all() and (s == scales).all() and (z == zeros).all()
+
+    prop()
