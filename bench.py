@@ -698,6 +698,19 @@ def run_sweep(args):
         rows.append({"config": f"W4BF16 7B-class decode step M={M}: 128 GEMVs (CUDA graph, {tag})", "ms": ms,
                      "GB/s": gbs, "frac_hbm": gbs / hbm})
         del mats, gr
+    # The prefill-side W4BF16 GEMM (attn_w4bf16_gemm) over a 4096-token chunk: the stacked QKV and
+    # the o_proj of an 8B-class model; FLOP = 2 T N K.
+    from paper_2607_15865_gb300.w4 import w4bf16_gemm
+    for N, K in ((6144, 4096), (4096, 4096)):
+        T = 4096
+        tiles = w4_inputs(1, N, K)[0]
+        x = rnd((T, K), gen)
+        y = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
+        ms = time_calls(lambda: w4bf16_gemm(tiles, x, N, out=y), args.sweep_reps)
+        tf = 2.0 * T * N * K / (ms * 1e-3) / 1e12
+        rows.append({"config": f"W4BF16 GEMM T={T} N={N} K={K} (prefill projection)", "ms": ms, "TFLOP/s": tf,
+                     "frac_tensor": tf / tc_peak})
+        del tiles, x, y
     # The attention half of a decoder block with W4BF16 weights (attn_decode_layer: RMSNorm ->
     # stacked QKV GEMV -> decode attention -> o_proj + residual), 32 layers of an 8B-class
     # model (hidden 4096, Hq 32, Hkv 8, D 128) at 4096 valid tokens, one CUDA graph.  Bytes =
