@@ -14,7 +14,8 @@ q[n,k] in 0..15, zero point z[n,g] in 0..15 and bf16 scale s[n,g]:
 
 computed here exactly in float64 from the bf16 inputs (``gemv``).
 
-Storage read by ``unpack_tiles`` (this module's own reader of the documented format):
+Storage written by ``write_tiles`` and read by ``unpack_tiles`` (this module's own writer and
+reader of the documented format):
 the matrix is cut into tiles of 16 rows x 128 inputs; tile (T, G) -- rows 16T..16T+15,
 group G -- is the (T * K/128 + G)-th record of 1072 bytes:
   bytes    0..1023  codes: row r of the tile holds 16 little-endian uint32 words at
@@ -65,6 +66,31 @@ def unpack_tiles(buf: np.ndarray, N: int, K: int):
     scales = scales.transpose(0, 2, 1).reshape(nt * TILE_ROWS, ng)
     zeros = zeros.transpose(0, 2, 1).reshape(nt * TILE_ROWS, ng)
     return unpack_row_words(words)[:N], scales[:N].copy(), zeros[:N].copy()
+
+
+def write_tiles(codes, scales_bf16, zeros) -> np.ndarray:
+    """codes uint8 [N, K], scales bf16 bits uint16 [N, K/128], zeros uint8 [N, K/128] -> the
+    tile stream (uint8, ceil(N/16) * K/128 * 1072 bytes), every value placed at the byte the
+    format above names; padding rows of the last row-tile stay zero."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    N, K = codes.shape
+    ng, nt = K // GROUP, (N + TILE_ROWS - 1) // TILE_ROWS
+    assert K % GROUP == 0 and np.shape(scales_bf16) == (N, ng) and np.shape(zeros) == (N, ng)
+    buf = np.zeros(nt * ng * TILE_BYTES, dtype=np.uint8)
+    n = np.arange(N)[:, None]
+    k = np.arange(K)[None, :]
+    rec = (n // TILE_ROWS) * ng + k // GROUP                      # record of (n, k)
+    bit = np.asarray(NIBBLE_SHIFT)[k % 8]                          # bit of the code in its word
+    byte = rec * TILE_BYTES + 64 * (n % TILE_ROWS) + 4 * ((k % GROUP) // 8) + bit // 8
+    np.bitwise_or.at(buf, byte.ravel(), ((codes & 15) << (bit % 8)).astype(np.uint8).ravel())
+    g = np.arange(ng)[None, :]
+    rec = (n // TILE_ROWS) * ng + g                                # record of (n, group)
+    s = np.asarray(scales_bf16, dtype=np.uint16)
+    at = rec * TILE_BYTES + SCALE_OFFSET + 2 * (n % TILE_ROWS)
+    buf[at.ravel()] = (s & 0xFF).astype(np.uint8).ravel()          # little-endian bf16 bits
+    buf[(at + 1).ravel()] = (s >> 8).astype(np.uint8).ravel()
+    buf[(rec * TILE_BYTES + ZERO_OFFSET + n % TILE_ROWS).ravel()] = np.asarray(zeros, np.uint8).ravel()
+    return buf
 
 
 def bf16_to_f64(bits: np.ndarray) -> np.ndarray:

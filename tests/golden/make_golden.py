@@ -40,7 +40,6 @@ def tiny_chain():
 
 def w4_tiny():
     from oracle import w4_oracle as W
-    from paper_2607_15865_gb300.w4 import pack_codes, pack_tiles
     from synthetic import gen
     from synthetic.workloads import Shape
     N, K, M = 40, 256, 3
@@ -49,7 +48,7 @@ def w4_tiny():
     scales = gen.normal_bf16("golden_w4", "scales", (N, K // 128), 0.02)
     x = gen.normal_bf16("golden_w4", "x", (M, K), 1.0)
     gamma = gen.normal_bf16("golden_w4", "gamma", (K,), 0.5)
-    out = {"tiles": pack_tiles(pack_codes(codes), scales, zeros).view(np.uint16),
+    out = {"tiles": W.write_tiles(codes, scales, zeros).view(np.uint16),
            "gemv": W.to_bf16_bits(W.gemv(codes, scales, zeros, x)),
            "rmsnorm": W.rmsnorm(x, gamma, 1e-6),
            "gemm": W.to_bf16_bits(W.gemm_bf16w(codes, scales, zeros, x))}

@@ -52,7 +52,7 @@ def test_entry_points_check_arguments_before_the_device():
 
 
 def test_tile_stream_round_trips_for_any_shape():
-    """Packer (product) and reader (oracle) agree for any row count and group count."""
+    """Packer (product), writer and reader (oracle) agree for any row count and group count."""
     hyp = pytest.importorskip("hypothesis")
     st = pytest.importorskip("hypothesis.strategies")
     from oracle import w4_oracle as W
@@ -69,5 +69,6 @@ def test_tile_stream_round_trips_for_any_shape():
         assert buf.size == (N + 15) // 16 * ng * TILE_BYTES
         c, s, z = W.unpack_tiles(buf, N, K)
         assert (c == codes).all() and (s == scales).all() and (z == zeros).all()
+        assert (buf == W.write_tiles(codes, scales, zeros)).all()  # byte for byte, padding included
 
     prop()

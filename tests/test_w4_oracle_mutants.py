@@ -2,7 +2,8 @@
 oracle fails one of them.
 
 Each mutant is oracle/w4_oracle.py with one plausible mistake substituted in (a wrong
-nibble order or tile transpose, a dropped zero point, a wrong group, a wrong bf16 decode
+nibble order or tile transpose, a tile writer that misplaces a scale byte, a code row or a
+zero point, a dropped zero point, a wrong group, a wrong bf16 decode
 or rounding, RMSNorm without eps or gamma or with a sum for the mean, a block without its
 residual or RMSNorm, k and v swapped, q read from the wrong rows, GEMM weights not rounded),
 loaded as a separate module.  The real oracle is never modified.
@@ -31,6 +32,10 @@ MUTANTS = {
     "block_without_rmsnorm": ("xn = rmsnorm(x_bf16, gamma_bf16, eps)", "xn = x_bf16"),
     "block_k_v_swapped": ("v = qkv[:, qd + kd:].reshape", "v = qkv[:, qd:qd + kd].reshape"),
     "block_q_from_wrong_rows": ("q = qkv[:, :qd].reshape", "q = qkv[:, kd:kd + qd].reshape"),
+    "writer_scale_bytes_swapped": ("buf[at.ravel()] = (s & 0xFF)", "buf[at.ravel()] = (s >> 8)"),
+    "writer_code_byte_ignores_row": ("+ 64 * (n % TILE_ROWS) + 4 *", "+ 4 *"),
+    "writer_zero_point_in_scale_bytes": ("buf[(rec * TILE_BYTES + ZERO_OFFSET + n % TILE_ROWS)",
+                                         "buf[(rec * TILE_BYTES + SCALE_OFFSET + n % TILE_ROWS)"),
     "gemm_weights_not_rounded": ("@ bf16_to_f64(dequant_bf16(codes, scales_bf16, zeros)).T",
                                  "@ dequant(codes, scales_bf16, zeros).T"),
 }

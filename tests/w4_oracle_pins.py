@@ -2,9 +2,9 @@
 same pins run against the real oracle (tests/test_w4_oracle.py) and against copies with a
 planted mistake (tests/test_w4_oracle_mutants.py).  None of them is the oracle's own code:
 
-  * format: the product's packer and the oracle's reader agree on every code, scale and
-    zero point of a matrix whose rows do not fill the last tile, and single values land at
-    the byte and bit the documented format names;
+  * format: the oracle's writer and reader round-trip every code, scale and zero point of
+    a matrix whose rows do not fill the last tile, and single values written by the oracle
+    land at the byte and bit the documented format names (read back here by hand);
   * brute force: y[m, n] = sum_k x[m, k] (q[n, k] - z[n, k // 128]) s[n, k // 128] and RMSNorm
     written as plain Python loops on tiny cases;
   * closed forms: codes equal to the zero points give y = 0; codes one above them with
@@ -16,15 +16,14 @@ planted mistake (tests/test_w4_oracle_mutants.py).  None of them is the oracle's
 import numpy as np
 
 from synthetic import gen
-from paper_2607_15865_gb300.w4 import pack_codes, pack_tiles
 
 
-def pin_packer_and_reader_agree_on_the_format(W):
+def pin_writer_and_reader_agree_on_the_format(W):
     N, K = 37, 384
     codes = gen.uint4_codes("w4pin", "codes", (N, K))
     zeros = gen.uint4_codes("w4pin", "zeros", (N, K // 128))
     scales = gen.normal_bf16("w4pin", "scales", (N, K // 128), 0.02)
-    buf = pack_tiles(pack_codes(codes), scales, zeros)
+    buf = W.write_tiles(codes, scales, zeros)
     assert buf.size == 3 * 3 * W.TILE_BYTES
     c, s, z = W.unpack_tiles(buf, N, K)
     assert (c == codes).all() and (s == scales).all() and (z == zeros).all()
@@ -38,7 +37,7 @@ def pin_single_values_land_where_the_format_says(W):
     scales[17, 1] = 0x3F80  # 1.0: tile (1, 1), row 1
     zeros = np.zeros((N, 2), np.uint8)
     zeros[18, 0] = 7  # tile (1, 0), row 2
-    buf = pack_tiles(pack_codes(codes), scales, zeros)
+    buf = W.write_tiles(codes, scales, zeros)
     rec = buf.reshape(4, W.TILE_BYTES)  # records (T, G) = (0,0), (0,1), (1,0), (1,1)
     word = rec[3, 64 * 3 + 4 * 5: 64 * 3 + 4 * 5 + 4].view("<u4")[0]
     assert int(word) == 9 << 20
@@ -202,4 +201,4 @@ def pin_gemm_rounds_each_weight_once(W):
     assert np.allclose(W.gemm_bf16w(codes, s, zeros, x), ref, rtol=1e-12, atol=1e-12)
 
 
-ALL_PINS = [pin_gemm_rounds_each_weight_once, pin_packer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v]
+ALL_PINS = [pin_gemm_rounds_each_weight_once, pin_writer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v]
