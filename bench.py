@@ -16,6 +16,9 @@ e2e       the same metric through the same C-ABI calls with host buffers: every
           (copies on their own streams, overlapping the neighbouring steps' compute).
 roofline  the dominant kernel (flash_fwd) against the measured bf16 tensor peak.
 stages    per-stage times; prefill stages in TFLOP/s, decode in HBM GB/s.
+configs   every configuration's stage on its own (7B-class prefill 512, prefill_kv 512 over
+          1536, the decode sweep, the long-context stages): median of CUDA-event-timed calls
+          with L2 flushed before each, TFLOP/s or GB/s and the fraction of the measured peak.
           (value comes from a pass with one event pair per step; stages, per-kernel
           times and the roofline from a second, instrumented pass over the same steps.)
 cpu_baseline  the CPU oracle on a bounded row sample of the same step.
@@ -393,6 +396,12 @@ def run_ours(args):
     clocks = sampler.stop()
     e2e_ms = max_over_ranks(e2e_start.elapsed_time(e2e_end) / K, dist, dev)
 
+    # ------------------------------------------------------------ the other configurations, stage by stage
+    # (after the timed step: CUDA events around each stage call, L2 flushed before each)
+    cfg_rows = None
+    if rank == 0 and not args.no_configs:
+        cfg_rows, _, _, _ = config_rows(dev, args.config_reps, graphs=False)
+
     # ------------------------------------------------------------ parity of the timed outputs + CPU baseline
     result = {}
     if rank == 0:
@@ -462,6 +471,7 @@ def run_ours(args):
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
                     "copies": "pinned host, own streams, overlapping the neighbouring steps",
                     "l2": "not flushed: each step's inputs arrive by copy; inputs + caches exceed L2"},
+            "configs": cfg_rows,
             "gpu_launches": launches,
             "clocks": clocks,
             "parity": parity,
@@ -477,21 +487,18 @@ def run_ours(args):
 # ----------------------------------------------------------------------------- per-config sweep
 
 
-def run_sweep(args):
-    """Times every configuration's stage on one GPU (CUDA events around the stage call,
-    inputs resident, L2 flushed before each timed call) and writes a table to
-    --sweep-out; the default JSON line is not printed in this mode."""
+def config_rows(dev, reps: int, graphs: bool):
+    """Per-configuration stage rows (the paper's workloads: 7B-class prefill 512, prefill_kv
+    512 over 1536, the decode sweep B in {1,4,16} x hist in {1024, 4096, 8191}, and the
+    long-context stages one by one).  Each row is the median of `reps` calls timed with CUDA
+    events around the stage call, inputs resident, L2 flushed (256 MB write + 256 MB read)
+    before every call and a short GPU sleep in front of it, so the host's launch cost stays
+    outside the events.  graphs: also time each decode step replayed from a CUDA graph."""
     import torch
-
-    import __graft_entry__
-    __graft_entry__.build()
     from paper_2607_15865_gb300.attention import Attention
-    from synthetic.workloads import Shape
-    dev = torch.device("cuda", 0)
-    torch.cuda.set_device(dev)
     flush_w = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
-    peaks, kind = load_peaks()
+    peaks, _ = load_peaks()
     tc_peak, hbm = float(peaks["bf16_tflops"]), float(peaks["hbm_gbs"])
 
     def rnd(shape, gen):
@@ -527,7 +534,7 @@ def run_sweep(args):
         kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
         vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
         out = torch.empty_like(q)
-        ms = time_calls(lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out), args.sweep_reps)
+        ms = time_calls(lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out), reps)
         tf = attn_flops(sh, prefill_pairs(hist, chunk)) / (ms * 1e-3) / 1e12
         rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
         attn.close()
@@ -549,11 +556,15 @@ def run_sweep(args):
                 kc, vc = caches[it[0] % len(caches)]
                 it[0] += 1
                 attn.decode(q, k, v, hl, kc, vc, out)
-            ms = time_calls(call, args.sweep_reps)
+            ms = time_calls(call, reps)
             gbs = decode_bytes(sh, hist) / (ms * 1e-3) / 1e9
+            row = {"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm}
+            rows.append(row)
+            if not graphs:
+                continue
             # the same step replayed from a CUDA graph (one graph per cache pair): what a
             # serving loop that captures its decode step sees
-            graphs = []
+            grs = []
             for kc, vc in caches:
                 attn.decode(q, k, v, hl, kc, vc, out)  # tensor maps built outside the capture
                 gr = torch.cuda.CUDAGraph()
@@ -562,18 +573,16 @@ def run_sweep(args):
                 with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
                     attn.decode(q, k, v, hl, kc, vc, out)
                 torch.cuda.current_stream().wait_stream(side)
-                graphs.append(gr)
+                grs.append(gr)
             torch.cuda.synchronize()
             git = [0]
 
             def replay():
-                graphs[git[0] % len(graphs)].replay()
+                grs[git[0] % len(grs)].replay()
                 git[0] += 1
-            ms_g = time_calls(replay, args.sweep_reps)
-            gbs_g = decode_bytes(sh, hist) / (ms_g * 1e-3) / 1e9
-            rows.append({"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm,
-                         "graph_ms": ms_g, "graph_GB/s": gbs_g})
-            del graphs
+            ms_g = time_calls(replay, reps)
+            row["graph_ms"], row["graph_GB/s"] = ms_g, decode_bytes(sh, hist) / (ms_g * 1e-3) / 1e9
+            del grs
         attn.close()
     attn = Attention.for_shape(S)
     kc = rnd((1, 8, 32768, 128), gen)
@@ -581,11 +590,29 @@ def run_sweep(args):
     q, k, v = rnd((1, 1, 40, 128), gen), rnd((1, 1, 8, 128), gen), rnd((1, 1, 8, 128), gen)
     out = torch.empty_like(q)
     hl = torch.full((1,), w.LONG_DECODE_HIST, dtype=torch.int32, device=dev)
-    ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), args.sweep_reps)
+    ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), reps)
     gbs = DECODE_BYTES / (ms * 1e-3) / 1e9
     rows.append({"config": "long decode hist 32767", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
     attn.close()
     del kc, vc
+    return rows, time_calls, rnd, gen
+
+
+def run_sweep(args):
+    """Times every configuration's stage on one GPU (CUDA events around the stage call,
+    inputs resident, L2 flushed before each timed call) and writes a table to
+    --sweep-out; the default JSON line is not printed in this mode."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.attention import Attention
+    from synthetic.workloads import Shape
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks, kind = load_peaks()
+    tc_peak, hbm = float(peaks["bf16_tflops"]), float(peaks["hbm_gbs"])
+    rows, time_calls, rnd, gen = config_rows(dev, args.sweep_reps, graphs=True)
     # The stage driver (Sections 4.1 and 4.5).  A 32768-token prompt as 1 prefill + 7
     # prefill_kv of 4096 tokens (the paper's 80K-prompt example scaled to this cache),
     # beside the same prompt in one prefill call.
@@ -892,6 +919,8 @@ def main():
     ap.add_argument("--sweep", action="store_true", help="time every configuration's stage instead (table to --sweep-out)")
     ap.add_argument("--sweep-out", default="sweep.json")
     ap.add_argument("--sweep-reps", type=int, default=20)
+    ap.add_argument("--config-reps", type=int, default=15, help="calls per configuration row of the JSON line")
+    ap.add_argument("--no-configs", action="store_true", help="leave the per-configuration rows out of the line")
     ap.add_argument("--stage", choices=tuple(STAGES), help="run only this stage (for profiler captures)")
     ap.add_argument("--reps", type=int, default=2)
     ap.add_argument("--hist", type=int)

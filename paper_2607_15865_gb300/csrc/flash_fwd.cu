@@ -39,6 +39,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <vector>
 
 #include "internal.h"
 #include "sm100_ptx.cuh"
@@ -122,21 +123,31 @@ struct Item {
     __device__ __forceinline__ int nkv(int t) const { return t ? nkvb : nkva; }
 };
 
+// The launch's work list: chunk S at history H, Hq query heads, batch sequences, n_pairs
+// query-tile pairs per (head, sequence); `head` items whole, the rest cut into nsplit
+// pieces; with the divisors the kernels use, as fast divisions (every division of the
+// schedule ran as a generic integer division before: about 1 us per decoded unit).
+struct Sched {
+    int S, H, Hq, batch, n_pairs, head, nsplit, n_units;
+    FastDiv fd_grid, fd_hqb, fd_hq, fd_g, fd_ns;
+};
+
 // Item order: longest query-tile pairs first across every (head, sequence), so a
 // causal launch starts its longest items first and ends with the shortest.
-__device__ __forceinline__ Item decode_item(int lin, int S, int H, int Hq, int G, int hq_b, int n_pairs) {
+__device__ __forceinline__ Item decode_item(int lin, const Sched& sc) {
     Item it;
-    const int pt = n_pairs - 1 - lin / hq_b;
-    const int rem = lin % hq_b;
-    it.h = rem % Hq;
-    it.b = rem / Hq;
-    it.g = it.h / G;
+    const int qt = fdiv(lin, sc.fd_hqb);
+    const int rem = lin - qt * (sc.Hq * sc.batch);
+    const int pt = sc.n_pairs - 1 - qt;
+    it.b = fdiv(rem, sc.fd_hq);
+    it.h = rem - it.b * sc.Hq;
+    it.g = fdiv(it.h, sc.fd_g);
     it.q0a = pt * 2 * BM;
     it.q0b = it.q0a + BM;
-    it.rowsa = max(0, min(BM, S - it.q0a));
-    it.rowsb = max(0, min(BM, S - it.q0b));
-    it.nkva = it.rowsa ? (H + it.q0a + it.rowsa + BN - 1) / BN : 0;
-    it.nkvb = it.rowsb ? (H + it.q0b + it.rowsb + BN - 1) / BN : 0;
+    it.rowsa = max(0, min(BM, sc.S - it.q0a));
+    it.rowsb = max(0, min(BM, sc.S - it.q0b));
+    it.nkva = it.rowsa ? (sc.H + it.q0a + it.rowsa + BN - 1) / BN : 0;
+    it.nkvb = it.rowsb ? (sc.H + it.q0b + it.rowsb + BN - 1) / BN : 0;
     it.n_kv = max(it.nkva, it.nkvb);
     return it;
 }
@@ -152,21 +163,22 @@ struct Unit {
     __device__ __forceinline__ int cnt(int t) const { return max(0, min(kv_hi, it.nkv(t)) - kv_lo); }
 };
 
-__device__ __forceinline__ Unit decode_unit(int lin, int S, int H, int Hq, int G, int hq_b, int n_pairs, int head,
-                                            int nsplit) {
+__device__ __forceinline__ Unit decode_unit(int lin, const Sched& sc) {
     Unit u;
-    int item = lin, s = 0, ns = 1;
     u.piece = -1;
-    if (lin >= head) {
-        const int v = lin - head;
-        item = head + v / nsplit;
-        s = v % nsplit;
-        ns = nsplit;
-        if (nsplit > 1) u.piece = v;
+    if (lin >= sc.head && sc.nsplit > 1) {
+        const int v = lin - sc.head;
+        const int tail = fdiv(v, sc.fd_ns);
+        const int s = v - tail * sc.nsplit;
+        u.piece = v;
+        u.it = decode_item(sc.head + tail, sc);
+        u.kv_lo = fdiv(u.it.n_kv * s, sc.fd_ns);
+        u.kv_hi = fdiv(u.it.n_kv * (s + 1), sc.fd_ns);
+    } else {
+        u.it = decode_item(lin, sc);
+        u.kv_lo = 0;
+        u.kv_hi = u.it.n_kv;
     }
-    u.it = decode_item(item, S, H, Hq, G, hq_b, n_pairs);
-    u.kv_lo = (u.it.n_kv * s) / ns;
-    u.kv_hi = (u.it.n_kv * (s + 1)) / ns;
     return u;
 }
 
@@ -175,10 +187,10 @@ __device__ __forceinline__ Unit decode_unit(int lin, int S, int H, int Hq, int G
 // one of the shortest of the next: with items sorted longest-first this evens out the
 // CTAs' totals (causal prefill 4096, 40 heads: the slowest CTA walks 74 KV tiles instead
 // of 88).  The last, partial round keeps its order.  A bijection on [0, n_units).
-__device__ __forceinline__ int unit_of(int lin, int n_units) {
-    const int g = static_cast<int>(gridDim.x), r = lin / g;
-    if ((r & 1) == 0 || (r + 1) * g > n_units) return lin;
-    return r * g + (g - 1 - lin % g);
+__device__ __forceinline__ int unit_of(int lin, const Sched& sc) {
+    const int g = static_cast<int>(gridDim.x), r = fdiv(lin, sc.fd_grid);
+    if ((r & 1) == 0 || (r + 1) * g > sc.n_units) return lin;
+    return r * g + (g - 1 - (lin - r * g));
 }
 
 // RoPE tables of one position in registers: cos/sin of pairs j = 0 .. D/2-1.  They are
@@ -253,8 +265,8 @@ __device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint3
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     flash_fwd_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                     const __grid_constant__ CUtensorMap map_v, int S, int s_stride, int H, int Hq, int Hkv, int batch,
-                     int n_pairs, int head, int nsplit, float scale_log2, const float* __restrict__ cos_t,
+                     const __grid_constant__ CUtensorMap map_v, const Sched sc, int s_stride, int Hkv,
+                     float scale_log2, const float* __restrict__ cos_t,
                      const float* __restrict__ sin_t, int tab_stride, uint16_t* __restrict__ out, float* __restrict__ ws_o,
                      float* __restrict__ ws_ml, int* __restrict__ err) {
     using L = Layout<D>;
@@ -268,12 +280,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int G = Hq / Hkv;
-    const int hq_b = Hq * batch;
-    const int n_items = n_pairs * hq_b;
-    const int n_units = head + (n_items - head) * nsplit;
+    const int S = sc.S, H = sc.H, Hq = sc.Hq, n_units = sc.n_units;
 
-    if (threadIdx.x == 0) {
+    if (warp == kWarpTma && lane == 0) {
+        // Barriers, then the first unit's q tiles right away: their copy overlaps the TMEM
+        // allocation and the register hand-over (q is the caller's input, complete before
+        // K1 began, so it may be read before this grid waits on K1).
         *abort_flag = 0;
         mbar_init(bar(B_QFULL), 1);
         mbar_init(bar(B_QREADY), 2 * BM / 32);
@@ -290,6 +302,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        if (static_cast<int>(blockIdx.x) < n_units) {
+            const Item it = decode_unit(unit_of(blockIdx.x, sc), sc).it;
+            mbar_arrive_expect_tx(bar(B_QFULL), 2 * L::Q_TILE);
+#pragma unroll
+            for (int t = 0; t < 2; ++t)
+#pragma unroll
+                for (int c = 0; c < L::DCH; ++c)
+                    tma_load_4d(base + L::OFF_Q + t * L::Q_TILE + c * L::CHUNK, &map_q, c * 64, it.h, it.q0(t),
+                                it.b, bar(B_QFULL));
+        }
     }
     if (warp == kWarpMma) {
         tmem_alloc(base + L::OFF_TMEM, kTmemCols);
@@ -307,28 +332,39 @@ __global__ void __launch_bounds__(kThreads, 1)
             // ---------------------------------------------------- q tiles and the group ring
             // A unit of n KV tiles takes n + 1 groups: group j holds K(j) (j < kv_hi) and
             // V(j-1) (j > kv_lo), the last one only the V the final PV reads.
-            tma_prefetch_desc(&map_q);
-            tma_prefetch_desc(&map_k);
-            tma_prefetch_desc(&map_v);
             uint32_t gc = 0;  // groups issued
             int items = 0;
             bool ok = true;
             bool kv_visible = false;  // K1's cache writes complete (dependent launch)
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
-                const Unit un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Unit un = decode_unit(unit_of(lin, sc), sc);
                 const Item& it = un.it;
-                if (items > 0 && !mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
-                    ok = false;
-                    break;
+                if (items > 0) {  // (the first unit's q tiles were issued in the prologue)
+                    if (!mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(bar(B_QFULL), 2 * L::Q_TILE);
+#pragma unroll
+                    for (int t = 0; t < 2; ++t)
+#pragma unroll
+                        for (int c = 0; c < L::DCH; ++c)
+                            tma_load_4d(base + L::OFF_Q + t * L::Q_TILE + c * L::CHUNK, &map_q, c * 64, it.h,
+                                        it.q0(t), it.b, bar(B_QFULL));
                 }
-                mbar_arrive_expect_tx(bar(B_QFULL), 2 * L::Q_TILE);
-#pragma unroll
-                for (int t = 0; t < 2; ++t)
-#pragma unroll
-                    for (int c = 0; c < L::DCH; ++c)
-                        tma_load_4d(base + L::OFF_Q + t * L::Q_TILE + c * L::CHUNK, &map_q, c * 64, it.h, it.q0(t),
-                                    it.b, bar(B_QFULL));
                 ++items;
+                {
+                    // the next unit's q tiles into L2, so that their copy after this unit is short
+                    const int nxt = lin + static_cast<int>(gridDim.x);
+                    if (nxt < n_units) {
+                        const Item nt = decode_unit(unit_of(nxt, sc), sc).it;
+#pragma unroll
+                        for (int t = 0; t < 2; ++t)
+                            if (nt.rows(t) > 0)
+#pragma unroll
+                                for (int c = 0; c < L::DCH; ++c) tma_prefetch_l2_4d(&map_q, c * 64, nt.h, nt.q0(t), nt.b);
+                    }
+                }
                 const int kv_row = it.b * Hkv + it.g;
                 if (!kv_visible) {
                     // This grid may start while K1 still appends the chunk's k and v: the q
@@ -416,7 +452,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 gslot = gslot + 1 == GS ? 0 : gslot + 1;
             };
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
-                const Unit un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                const Unit un = decode_unit(unit_of(lin, sc), sc);
                 const Item& it = un.it;
                 if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag)) {
                     ok = false;
@@ -504,7 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int lin = blockIdx.x;
         Unit un;
         if (lin < n_units) {
-            un = decode_unit(unit_of(lin, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+            un = decode_unit(unit_of(lin, sc), sc);
             ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
                               un.it.rows(t), H + un.it.q0(t), cos_t, sin_t, tab_stride);
             ++items;
@@ -601,7 +637,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int next = lin + static_cast<int>(gridDim.x);
             Unit nun;
             if (next < n_units) {
-                nun = decode_unit(unit_of(next, n_units), S, H, Hq, G, hq_b, n_pairs, head, nsplit);
+                nun = decode_unit(unit_of(next, sc), sc);
                 ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
                                   row, nun.it.rows(t), H + nun.it.q0(t), cos_t, sin_t, tab_stride);
                 ++items;
@@ -646,33 +682,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                         __syncwarp();
                     }
                 } else {
-                    // O_T / l -> bf16 -> out straight from each thread's row, or for a piece the
-                    // unnormalised O_T
-                    const float inv_l = un.piece < 0 ? 1.f / l_run : 1.f;
-                    uint16_t* orow = out + ((static_cast<size_t>(it.b) * s_stride + it.q0(t) + row) * Hq + it.h) * D;
-                    float* prow_o = ws_o + prow * D;
+                    // a piece: the unnormalised O_T (float) through the same staging area, 32
+                    // columns per pass, so each warp store writes 4 whole 128-byte row segments
+                    const int lane = threadIdx.x & 31, r0 = row & ~31;
+                    uint8_t* stage = gbase + L::OFF_STAGE + warp * L::STAGE_WARP;
+                    float* pbase = ws_o + (static_cast<size_t>(un.piece) * 2 * BM + t * BM + r0) * D;
 #pragma unroll
                     for (int c = 0; c < D / 32; ++c) {
                         uint32_t o[32];
                         tmem_ld32(o_col + 32 * c, o);
                         tmem_wait_ld();
-                        if (row < it.rows(t)) {
-                            const float* f = reinterpret_cast<const float*>(o);
-                            if (un.piece < 0) {
 #pragma unroll
-                                for (int v4 = 0; v4 < 4; ++v4)
-                                    *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v4) = make_uint4(
-                                        pack_bf16x2(f[8 * v4 + 0] * inv_l, f[8 * v4 + 1] * inv_l),
-                                        pack_bf16x2(f[8 * v4 + 2] * inv_l, f[8 * v4 + 3] * inv_l),
-                                        pack_bf16x2(f[8 * v4 + 4] * inv_l, f[8 * v4 + 5] * inv_l),
-                                        pack_bf16x2(f[8 * v4 + 6] * inv_l, f[8 * v4 + 7] * inv_l));
-                            } else {
+                        for (int ch = 0; ch < 8; ++ch)
+                            *reinterpret_cast<uint4*>(stage + lane * 128 + ((ch ^ (lane & 7)) << 4)) =
+                                make_uint4(o[4 * ch], o[4 * ch + 1], o[4 * ch + 2], o[4 * ch + 3]);
+                        __syncwarp();
 #pragma unroll
-                                for (int v4 = 0; v4 < 8; ++v4)
-                                    *reinterpret_cast<float4*>(prow_o + 32 * c + 4 * v4) =
-                                        make_float4(f[4 * v4], f[4 * v4 + 1], f[4 * v4 + 2], f[4 * v4 + 3]);
-                            }
+                        for (int i = 0; i < 8; ++i) {
+                            const int rr = 4 * i + (lane >> 3), ch = lane & 7;
+                            const uint4 u = *reinterpret_cast<const uint4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
+                            if (r0 + rr < it.rows(t))
+                                *reinterpret_cast<uint4*>(pbase + static_cast<size_t>(rr) * D + 32 * c + 4 * ch) = u;
                         }
+                        __syncwarp();
                     }
                 }
                 if (un.piece >= 0 && row < it.rows(t)) {
@@ -708,15 +740,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Block (tail item, query tile, group of 8 rows); one warp per row.
 template <int D>
 __global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restrict__ ws_o,
-                                                            const float* __restrict__ ws_ml, int S, int s_stride, int H,
-                                                            int Hq,
-                                                            int G, int hq_b, int n_pairs, int head, int nsplit,
-                                                            uint16_t* __restrict__ out) {
+                                                            const float* __restrict__ ws_ml, const Sched sc,
+                                                            int s_stride, uint16_t* __restrict__ out) {
     constexpr int PER_LANE = D / 32;
     asm volatile("griddepcontrol.wait;" ::: "memory");  // the pieces are complete and visible
+    const int head = sc.head, nsplit = sc.nsplit, Hq = sc.Hq;
     const int item = head + static_cast<int>(blockIdx.x) / 2;
     const int t = static_cast<int>(blockIdx.x) % 2;
-    const Item it = decode_item(item, S, H, Hq, G, hq_b, n_pairs);
+    const Item it = decode_item(item, sc);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int row = static_cast<int>(blockIdx.y) * 8 + warp;
     if (row < it.rows(t)) {
@@ -752,31 +783,68 @@ __global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restr
     }
 }
 
-// Host schedule: `head` items fill whole rounds of the persistent CTAs; the tail
-// items are cut into nsplit KV pieces (at most one piece per CTA, at most 16 per
-// item, never more than the shortest tail item has KV tiles).
-struct Schedule {
+// Host schedule: `head` items fill whole rounds of the persistent CTAs; the tail items
+// (the last, partial round) may be cut into nsplit KV pieces, at most one per CTA, that
+// the merge kernel combines.  The piece count minimises a model of the slowest CTA's
+// time, dealt as the kernel deals (rounds of alternating direction): per unit a fixed
+// cost (its q copy and RoPE hand-over, epilogue), per KV step of the two query tiles the
+// tensor-core time of four 128 x 128 x D MMAs, and for a split launch the partial writes
+// and the merge kernel.
+struct HostSchedule {
     int n_pairs, n_items, head, nsplit, n_units, grid;
 };
 
-Schedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
-    Schedule sc;
+constexpr int kMaxSplit = 16;
+
+int unit_of_host(int lin, int g, int n_units) {
+    const int r = lin / g;
+    if ((r & 1) == 0 || (r + 1) * g > n_units) return lin;
+    return r * g + (g - 1 - lin % g);
+}
+
+HostSchedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
+    HostSchedule sc;
     const int n_qtiles = (chunk + BM - 1) / BM;
     sc.n_pairs = (n_qtiles + 1) / 2;
     sc.n_items = sc.n_pairs * s.n_q_heads * s.batch;
-    sc.head = (sc.n_items / num_sms) * num_sms;
-    const int tail = sc.n_items - sc.head;
-    sc.nsplit = 1;
-    if (tail > 0) {
-        const int nkv_min = (hist + std::min(2 * BM, chunk) + BN - 1) / BN;  // pair 0 is the shortest
-        long nkv_sum = 0;
-        for (int pt = 0; pt < sc.n_pairs; ++pt) nkv_sum += (hist + std::min(2 * BM * (pt + 1), chunk) + BN - 1) / BN;
-        // Split when there are fewer items than CTAs, or when the tail items are long
-        // enough for the last round to matter (not for the short tail of a causal prefill).
-        if (sc.head == 0 || 2L * nkv_min * sc.n_pairs >= nkv_sum)
-            sc.nsplit = std::max(1, std::min({num_sms / tail, 16, nkv_min}));
+    const int hq_b = s.n_q_heads * s.batch;
+    auto n_kv = [&](int item) {  // KV tiles of an item (longest pairs first)
+        const int pt = sc.n_pairs - 1 - item / hq_b;
+        return (hist + std::min(2 * BM * (pt + 1), chunk) + BN - 1) / BN;
+    };
+    // costs in KV steps of both query tiles (about 1.3 us each)
+    const double c_unit = 1.6, c_split = 2.5, c_step = 1.0;
+    const int full_rounds = sc.n_items / num_sms;
+    const int tail = sc.n_items - full_rounds * num_sms;
+    const int nkv_min = tail > 0 ? n_kv(sc.n_items - 1) : 1;  // the tail's shortest item
+    int best_ns = 1;
+    double best = 1e300;
+    std::vector<double> load;
+    for (int ns = 1; ns <= kMaxSplit; ++ns) {
+        if (ns > 1 && (tail == 0 || tail * ns > num_sms || ns > nkv_min)) break;
+        const int head = ns > 1 ? full_rounds * num_sms : sc.n_items;
+        const int n_units = head + (sc.n_items - head) * ns;
+        const int grid = std::min(n_units, num_sms);
+        load.assign(grid, 0.0);
+        for (int lin = 0; lin < n_units; ++lin) {
+            const int u = unit_of_host(lin, grid, n_units);
+            double cost = c_unit;
+            if (u < head) {
+                cost += c_step * n_kv(u);
+            } else {
+                const int v = u - head, nk = n_kv(head + v / ns), sp = v % ns;
+                cost += c_step * (nk * (sp + 1) / ns - nk * sp / ns);
+            }
+            load[lin % grid] += cost;
+        }
+        const double mk = *std::max_element(load.begin(), load.end()) + (ns > 1 ? c_split : 0.0);
+        if (mk < best - 1e-9) {
+            best = mk;
+            best_ns = ns;
+        }
     }
-    if (sc.nsplit == 1) sc.head = sc.n_items;
+    sc.nsplit = best_ns;
+    sc.head = best_ns > 1 ? full_rounds * num_sms : sc.n_items;
     sc.n_units = sc.head + (sc.n_items - sc.head) * sc.nsplit;
     sc.grid = std::min(sc.n_units, num_sms);
     return sc;
@@ -786,12 +854,26 @@ template <int D>
 cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride, const float* cos_t,
                      const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
                      cudaStream_t st, int* n_launched) {
-    const Schedule sc = make_schedule(s, hist, chunk, num_sms);
+    const HostSchedule hs = make_schedule(s, hist, chunk, num_sms);
+    Sched sc;
+    sc.S = chunk;
+    sc.H = hist;
+    sc.Hq = s.n_q_heads;
+    sc.batch = s.batch;
+    sc.n_pairs = hs.n_pairs;
+    sc.head = hs.head;
+    sc.nsplit = hs.nsplit;
+    sc.n_units = hs.n_units;
+    sc.fd_grid = make_fastdiv(hs.grid);
+    sc.fd_hqb = make_fastdiv(s.n_q_heads * s.batch);
+    sc.fd_hq = make_fastdiv(s.n_q_heads);
+    sc.fd_g = make_fastdiv(s.n_q_heads / s.n_kv_heads);
+    sc.fd_ns = make_fastdiv(hs.nsplit);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     // Dependent launch after K1 (programmatic stream serialization): only the producer's
     // first K/V copy waits for K1 (griddep_wait).
     cudaLaunchConfig_t kcfg = {};
-    kcfg.gridDim = dim3(static_cast<unsigned>(sc.grid));
+    kcfg.gridDim = dim3(static_cast<unsigned>(hs.grid));
     kcfg.blockDim = dim3(kThreads);
     kcfg.dynamicSmemBytes = Layout<D>::ALLOC;
     kcfg.stream = st;
@@ -800,13 +882,12 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     kattr[0].val.programmaticStreamSerializationAllowed = 1;
     kcfg.attrs = kattr;
     kcfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&kcfg, flash_fwd_kernel<D>, maps.q, maps.k, maps.v, chunk, s_stride, hist,
-                                       s.n_q_heads, s.n_kv_heads, s.batch, sc.n_pairs, sc.head, sc.nsplit, scale_log2,
-                                       cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
+    cudaError_t e = cudaLaunchKernelEx(&kcfg, flash_fwd_kernel<D>, maps.q, maps.k, maps.v, sc, s_stride,
+                                       s.n_kv_heads, scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
     *n_launched = 1;
-    if (e != cudaSuccess || sc.nsplit == 1) return e;
+    if (e != cudaSuccess || hs.nsplit == 1) return e;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(2 * (sc.n_items - sc.head)), BM / 8);
+    cfg.gridDim = dim3(static_cast<unsigned>(2 * (hs.n_items - hs.head)), BM / 8);
     cfg.blockDim = dim3(256);
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
@@ -814,9 +895,7 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const int G = s.n_q_heads / s.n_kv_heads;
-    e = cudaLaunchKernelEx(&cfg, flash_combine_kernel<D>, ws_o, ws_ml, chunk, s_stride, hist, s.n_q_heads, G,
-                           s.n_q_heads * s.batch, sc.n_pairs, sc.head, sc.nsplit, out);
+    e = cudaLaunchKernelEx(&cfg, flash_combine_kernel<D>, ws_o, ws_ml, sc, s_stride, out);
     *n_launched = 2;
     return e;
 }

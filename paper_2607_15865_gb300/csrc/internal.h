@@ -17,6 +17,28 @@ struct Shape {
     int batch, n_q_heads, n_kv_heads, head_dim, max_len;
 };
 
+// Division by a divisor fixed at launch time (Granlund and Montgomery, "Division by
+// invariant integers using multiplication", 1994): with s = ceil(log2 d) and
+// m = floor(2^32 (2^s - d) / d) + 1, n / d = (umulhi(n, m) + n) >> s for 0 <= n < 2^31
+// and 1 <= d < 2^31.  The host builds it; kernels divide with fdiv() in a few
+// instructions instead of the dozens of a generic integer division.
+struct FastDiv {
+    uint32_t d, m, s;
+};
+inline FastDiv make_fastdiv(int div) {
+    FastDiv f;
+    f.d = static_cast<uint32_t>(div);
+    f.s = 0;
+    while ((1ull << f.s) < f.d) ++f.s;
+    f.m = static_cast<uint32_t>(((1ull << 32) * ((1ull << f.s) - f.d)) / f.d + 1);
+    return f;
+}
+#ifdef __CUDACC__
+__device__ __forceinline__ int fdiv(int n, const FastDiv& f) {
+    return static_cast<int>((__umulhi(static_cast<uint32_t>(n), f.m) + static_cast<uint32_t>(n)) >> f.s);
+}
+#endif
+
 // K1: RoPE of the new k (table gather, Section 4.6.2) and the in-place append of
 // k and v into cache slots hist+i (Listing 2 "Concat"; Section 4.6.3).
 // hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.  k and v
