@@ -192,9 +192,31 @@ int attn_decode_steps(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const
 int attn_device_error(attn_ctx* ctx, attn_stream_t stream, int* flags);
 
 /*
- * Kernel timing (tracing).  The library launches four kernels:
+ * Failure detection (no counterpart in the paper, which runs on a static TPU schedule):
+ * every wait inside a kernel of this library -- on a copy, a tensor-core result or a
+ * hand-over between the kernel's warps -- gives up after a time limit, records
+ * ATTN_DEVERR_TIMEOUT in the device error word, lets the copies and MMAs it has already
+ * issued finish, releases its tensor memory and returns; nothing spins forever and
+ * nothing traps, so the context stays usable.
+ *
+ * attn_set_wait_limit sets that limit for the kernels this context launches from the
+ * next call on: limit_ns > 0 is the limit in nanoseconds, limit_ns <= 0 restores the
+ * default of 1 s.  The waits that drain copies and MMAs already in flight always keep
+ * the default.  With a limit far below a kernel's latency (a test of the failure path)
+ * the next stage calls give up at their first wait that is not already satisfied: the
+ * error word gets ATTN_DEVERR_TIMEOUT, and their outputs and the cache slots they would
+ * have written are undefined (every other cache slot is left as it was).  Restore the
+ * default and read the error word (attn_device_error) before relying on results again.
+ * Returns ATTN_OK, or ATTN_EINVAL for a null context.  Host-only; enqueues nothing.
+ */
+int attn_set_wait_limit(attn_ctx* ctx, long long limit_ns);
+
+/*
+ * Kernel timing (tracing).  The attention entry points launch these kernels (the
+ * W4BF16 kernels, which take no context, are not timed):
  *   ATTN_KERNEL_ROPE_APPEND     RoPE of the new keys + in-place cache append (every stage)
- *   ATTN_KERNEL_FLASH_FWD       causal flash attention (prefill, prefill_kv)
+ *   ATTN_KERNEL_FLASH_FWD       causal flash attention (prefill, prefill_kv), with the
+ *                               merge kernel of its split tail when it runs one
  *   ATTN_KERNEL_DECODE_SPLIT    split-KV decode (decode); with head_dim 128 it also
  *                               merges the splits and writes out itself
  *   ATTN_KERNEL_DECODE_COMBINE  log-sum-exp merge of the partials (decode, head_dim 64)

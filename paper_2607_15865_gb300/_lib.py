@@ -18,7 +18,8 @@ W4_WEIGHTS_STATIC = 1
 DEVERR_HIST_RANGE, DEVERR_TIMEOUT = 1, 2
 
 EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "attn_decode",
-            "attn_decode_multi", "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_timing_enable", "attn_timing_read",
+            "attn_decode_multi", "attn_prompt", "attn_decode_steps", "attn_device_error", "attn_set_wait_limit",
+            "attn_timing_enable", "attn_timing_read",
             "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc", "attn_w4bf16_gemv",
             "attn_w4bf16_rows_per_launch", "attn_w4bf16_gemv_fused", "attn_decode_layer",
             "attn_w4bf16_gemm")
@@ -73,6 +74,8 @@ def load(path: str = LIB_PATH):
     lib.attn_decode_steps.restype = i32
     lib.attn_device_error.argtypes = [vp, vp, ctypes.POINTER(ctypes.c_int)]
     lib.attn_device_error.restype = i32
+    lib.attn_set_wait_limit.argtypes = [vp, ctypes.c_longlong]
+    lib.attn_set_wait_limit.restype = i32
     lib.attn_timing_enable.argtypes = [vp, i32]
     lib.attn_timing_enable.restype = i32
     lib.attn_timing_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_longlong)]

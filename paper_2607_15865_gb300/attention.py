@@ -204,6 +204,11 @@ class Attention:
         self._check(self.lib.attn_timing_read(self._ctx, ms, n), "attn_timing_read")
         return {name: (ms[i], n[i]) for i, name in enumerate(_lib.KERNELS)}
 
+    def set_wait_limit(self, limit_ns: int):
+        """Time limit of the kernels' bounded waits for the following calls, in nanoseconds
+        (<= 0 restores the default of 1 s); see attn_set_wait_limit."""
+        self._check(self.lib.attn_set_wait_limit(self._ctx, int(limit_ns)), "attn_set_wait_limit")
+
     def device_error(self, stream=None) -> int:
         """Synchronise, read and clear the device error word; returns its DEVERR_* bits."""
         flags = ctypes.c_int(0)

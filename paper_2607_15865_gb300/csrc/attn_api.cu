@@ -54,6 +54,7 @@ struct attn_ctx {
     std::vector<int> ev_kind;
     int ev_used;
     long long launches[ATTN_NUM_KERNELS];
+    uint64_t wait_ns;  // limit of the kernels' bounded waits (attn_set_wait_limit)
 };
 
 namespace {
@@ -163,7 +164,7 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");
     e = timed(c, ATTN_KERNEL_FLASH_FWD, st, [&](int* n) {
         return attn::launch_flash_fwd(s, maps, hist, chunk, seq_stride, c->d_cos_t, c->d_sin_t, out, c->d_flash_o,
-                                      c->d_flash_ml, c->d_err, c->num_sms, st, n);
+                                      c->d_flash_ml, c->d_err, c->num_sms, st, n, c->wait_ns);
     });
     if (e != cudaSuccess) return cuda_fail(e, "flash_fwd launch");
     return ATTN_OK;
@@ -192,6 +193,7 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     c->device = dev;
     c->num_sms = prop.multiProcessorCount;
     c->nsplit_max = 256;
+    c->wait_ns = attn::kWaitLimitNs;
 
     cudaDriverEntryPointQueryResult qres;
     void* fn = nullptr;
@@ -335,9 +337,9 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
-                                          c->d_err, after_decode, ntok, st, producer_early);
+                                          c->d_err, after_decode, ntok, st, producer_early, c->wait_ns);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
-                                         c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st);
+                                         c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st, c->wait_ns);
     });
     if (e != cudaSuccess) return cuda_fail(e, "decode_split launch");
     if (tc) return ATTN_OK;  // the tensor-core decode merges its splits itself
@@ -404,6 +406,12 @@ int attn_decode_steps(attn_ctx* c, const uint16_t* q, const uint16_t* k, const u
                                   v_cache, out + t * q_step, st);
         if (rc != ATTN_OK) return rc;
     }
+    return ATTN_OK;
+}
+
+int attn_set_wait_limit(attn_ctx* c, long long limit_ns) {
+    if (c == nullptr) return ATTN_EINVAL;
+    c->wait_ns = limit_ns > 0 ? static_cast<uint64_t>(limit_ns) : attn::kWaitLimitNs;
     return ATTN_OK;
 }
 

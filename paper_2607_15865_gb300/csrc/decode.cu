@@ -98,7 +98,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) decode_split_kernel(
     const int32_t* __restrict__ d_hist, int hist_add, uint16_t* __restrict__ k_cache, uint16_t* __restrict__ v_cache,
     const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv, int G, int passes,
     int max_len, int nsplit, float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml,
-    int* __restrict__ err) {
+    int* __restrict__ err, uint64_t wait_ns) {
     using L = DecLayout<D, GM>;
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
@@ -210,7 +210,7 @@ __global__ void __launch_bounds__(NTHREADS, 2) decode_split_kernel(
     int j = 0;
     for (; j < ntiles; ++j) {
         const int st = j % NSTAGE;
-        ok = mbar_wait(bar(st), static_cast<uint32_t>(j / NSTAGE) & 1u, nullptr);
+        ok = mbar_wait(bar(st), static_cast<uint32_t>(j / NSTAGE) & 1u, nullptr, wait_ns);
         if (__syncthreads_or(!ok)) {
             ok = false;
             break;
@@ -413,11 +413,11 @@ cudaError_t launch_split_t(const Shape& s, const DecodeMaps& maps, dim3 grid, co
                            const uint16_t* k_new, const uint16_t* v_new, const int32_t* d_hist, int hist_add,
                            uint16_t* kc, uint16_t* vc, const float* cos_tab, const float* sin_tab, int G, int passes,
                            int nsplit,
-                           float scale_log2, float* part_o, float* part_ml, int* err, cudaStream_t st) {
+                           float scale_log2, float* part_o, float* part_ml, int* err, cudaStream_t st, uint64_t wait_ns) {
     decode_split_kernel<D, GM><<<grid, NTHREADS, DecLayout<D, GM>::ALLOC, st>>>(
         maps.k, maps.v, q, k_new, v_new, d_hist, hist_add, kc, vc, cos_tab, sin_tab, s.n_q_heads, s.n_kv_heads, G,
         passes,
-        s.max_len, nsplit, scale_log2, part_o, part_ml, err);
+        s.max_len, nsplit, scale_log2, part_o, part_ml, err, wait_ns);
     return cudaGetLastError();
 }
 
@@ -425,7 +425,7 @@ template <int D>
 cudaError_t launch_split_d(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
                            const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* kc, uint16_t* vc,
                            const float* cos_tab, const float* sin_tab, int nsplit, float* part_o, float* part_ml,
-                           int* err, cudaStream_t st) {
+                           int* err, cudaStream_t st, uint64_t wait_ns) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const int G = s.n_q_heads / s.n_kv_heads;
     const int passes = (G + 7) / 8;
@@ -436,7 +436,7 @@ cudaError_t launch_split_d(const Shape& s, const DecodeMaps& maps, const uint16_
 #define ATTN_SPLIT_CASE(N)                                                                                     \
     case N:                                                                                                    \
         return launch_split_t<D, N>(s, maps, grid, q, k_new, v_new, d_hist, hist_add, kc, vc, cos_tab, sin_tab, G, \
-                                    passes, nsplit, scale_log2, part_o, part_ml, err, st);
+                                    passes, nsplit, scale_log2, part_o, part_ml, err, st, wait_ns);
         ATTN_SPLIT_CASE(1) ATTN_SPLIT_CASE(2) ATTN_SPLIT_CASE(3) ATTN_SPLIT_CASE(4)
         ATTN_SPLIT_CASE(5) ATTN_SPLIT_CASE(6) ATTN_SPLIT_CASE(7) ATTN_SPLIT_CASE(8)
 #undef ATTN_SPLIT_CASE
@@ -507,12 +507,12 @@ cudaError_t make_decode_maps(PFN_encodeTiled encode, const Shape& s, const uint1
 cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
                                 const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                                 uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
-                                float* part_ml, int nsplit, int* err, cudaStream_t st) {
+                                float* part_ml, int nsplit, int* err, cudaStream_t st, uint64_t wait_ns) {
     if (s.head_dim == 128)
         return launch_split_d<128>(s, maps, q, k_new, v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab,
-                                   nsplit, part_o, part_ml, err, st);
+                                   nsplit, part_o, part_ml, err, st, wait_ns);
     return launch_split_d<64>(s, maps, q, k_new, v_new, d_hist, hist_add, k_cache, v_cache, cos_tab, sin_tab, nsplit,
-                              part_o, part_ml, err, st);
+                              part_o, part_ml, err, st, wait_ns);
 }
 
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,

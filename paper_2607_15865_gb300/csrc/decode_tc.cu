@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
     int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
-    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early) {
+    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -309,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             for (int j = 0;; ++j) {
                 const int tile = cur < T ? cur : -1;
                 const int ks = j % KST, vs = j % VST;
-                if (j >= KST && !mbar_wait(bar(B_KEMPTY0 + ks), static_cast<uint32_t>(j / KST - 1) & 1u, abort_flag)) {
+                if (j >= KST && !mbar_wait(bar(B_KEMPTY0 + ks), static_cast<uint32_t>(j / KST - 1) & 1u, abort_flag, wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -324,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     tma_load_3d(base + L::OFF_K + ks * L::TILE + c * L::BOX, &map_k, c * 64, tile * KT, kv_row,
                                 bar(B_KFULL0 + ks));
                 issued_k = j + 1;
-                if (j >= VST && !mbar_wait(bar(B_VEMPTY0 + vs), static_cast<uint32_t>(j / VST - 1) & 1u, abort_flag)) {
+                if (j >= VST && !mbar_wait(bar(B_VEMPTY0 + vs), static_cast<uint32_t>(j / VST - 1) & 1u, abort_flag, wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -387,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         constexpr uint32_t kIdPV = idesc_bf16_f32(D, NH, true, false);
         const uint32_t sQ = base + L::OFF_Q;
         auto wait_all = [&](int barrier, uint32_t parity) -> bool {
-            return __all_sync(0xFFFFFFFFu, mbar_wait(bar(barrier), parity, abort_flag));
+            return __all_sync(0xFFFFFFFFu, mbar_wait(bar(barrier), parity, abort_flag, wait_ns));
         };
         auto issue_pv = [&](int jj) -> bool {
             if (!wait_all(B_PFULL0 + (jj & 1), static_cast<uint32_t>(jj >> 1) & 1u)) return false;
@@ -531,8 +531,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         }
         bool ok = true;
         int n = 0;  // tiles processed
+        // The four softmax warps meet at named barriers (the lazy-max test, the tile maxima,
+        // the epilogue): a wait that ran out in one warp is made known to all four through a
+        // barrier that every one of them reaches, before any of them leaves the loop, so that
+        // no warp is left waiting at a barrier the others never reach.
         for (int j = 0;; ++j) {
-            ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + (j & 1)), static_cast<uint32_t>(j >> 1) & 1u, abort_flag));
+            ok = !named_or_128(!mbar_wait(bar(B_SFULL0 + (j & 1)), static_cast<uint32_t>(j >> 1) & 1u, abort_flag, wait_ns));
             if (!ok) break;
             const int tile = meta[j % 8];
             if (tile < 0) {
@@ -577,8 +581,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 }
                 if (j > 0 && any_move) {  // the same decision in every thread (same tile maxima)
                     // O^T holds PV through tile j-1 once PV(j-1) completed (S(j) completed after PV(j-2)).
-                    ok = __all_sync(0xFFFFFFFFu,
-                                    mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(j - 1) & 1u, abort_flag));
+                    ok = !named_or_128(!mbar_wait(bar(B_PVDONE), static_cast<uint32_t>(j - 1) & 1u, abort_flag, wait_ns));
                     if (!ok) break;
                     tc_fence_after();
                     uint32_t o[NHP];
@@ -613,7 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         } else if (ok) {
             // (PVDONE could be two phases behind here -- PV(n-2) may still run -- so the
             // epilogue waits on its own barrier, committed once after the last PV.)
-            ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL), 0u, abort_flag));
+            ok = !named_or_128(!mbar_wait(bar(B_OFULL), 0u, abort_flag, wait_ns));
         }
         if (ok && n > 0) {
             // row sums: every thread holds a partial over its keys
@@ -798,7 +801,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
                              float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
-                             int ntok, cudaStream_t st, bool producer_early) {
+                             int ntok, cudaStream_t st, bool producer_early, uint64_t wait_ns) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
@@ -819,7 +822,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
-                              producer_early ? 1 : 0);
+                              producer_early ? 1 : 0, wait_ns);
 }
 
 }  // namespace attn

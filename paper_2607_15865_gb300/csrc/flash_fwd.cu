@@ -251,10 +251,10 @@ template <int D>
 __device__ __forceinline__ bool rope_item(uint32_t qfull, uint32_t qready, uint32_t parity, const volatile int* abort,
                                           uint8_t* qtile, int row, int rows, int pos0,
                                           const float* __restrict__ cos_t, const float* __restrict__ sin_t,
-                                          int stride) {
+                                          int stride, uint64_t wait_ns) {
     RopeRow<D> tabs;
     rope_load<D>(tabs, row < rows ? pos0 + row : pos0, cos_t, sin_t, stride);
-    const bool w = __all_sync(0xFFFFFFFFu, mbar_wait(qfull, parity, abort));
+    const bool w = __all_sync(0xFFFFFFFFu, mbar_wait(qfull, parity, abort, wait_ns));
     if (w && row < rows) rope_row_smem<D>(qtile, row, tabs);
     fence_proxy_async_smem();
     __syncwarp();
@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap map_v, const Sched sc, int s_stride, int Hkv,
                      float scale_log2, const float* __restrict__ cos_t,
                      const float* __restrict__ sin_t, int tab_stride, uint16_t* __restrict__ out, float* __restrict__ ws_o,
-                     float* __restrict__ ws_ml, int* __restrict__ err) {
+                     float* __restrict__ ws_ml, int* __restrict__ err, uint64_t wait_ns) {
     using L = Layout<D>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -340,7 +340,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const Unit un = decode_unit(unit_of(lin, sc), sc);
                 const Item& it = un.it;
                 if (items > 0) {  // (the first unit's q tiles were issued in the prologue)
-                    if (!mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag)) {
+                    if (!mbar_wait(bar(B_QEMPTY), static_cast<uint32_t>(items - 1) & 1u, abort_flag, wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -375,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 for (int j = un.kv_lo; j <= un.kv_hi; ++j, ++gc) {
                     const int st = static_cast<int>(gc % GS);
-                    if (gc >= GS && !mbar_wait(bar(B_GEMPTY0 + st), (gc / GS - 1u) & 1u, abort_flag)) {
+                    if (gc >= GS && !mbar_wait(bar(B_GEMPTY0 + st), (gc / GS - 1u) & 1u, abort_flag, wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -440,9 +440,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             };
             // P_t of the previous KV tile in TMEM, and O_t free when it is the unit's first PV
             auto wait_p = [&](int t, bool first) -> bool {
-                if (!mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag)) return false;
+                if (!mbar_wait(bar(B_PFULL0 + t), p_cnt[t] & 1u, abort_flag, wait_ns)) return false;
                 ++p_cnt[t];
-                if (first && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag))
+                if (first && o_cnt[t] > 0 && !mbar_wait(bar(B_OEMPTY0 + t), (o_cnt[t] - 1u) & 1u, abort_flag, wait_ns))
                     return false;
                 return true;
             };
@@ -454,14 +454,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int lin = blockIdx.x; lin < n_units && ok; lin += gridDim.x) {
                 const Unit un = decode_unit(unit_of(lin, sc), sc);
                 const Item& it = un.it;
-                if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag)) {
+                if (!mbar_wait(bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, wait_ns)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 for (int j = un.kv_lo; j < un.kv_hi && ok; ++j) {
                     // group j: K(j), and V(j-1) for the PV MMAs of the previous tile
-                    if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag)) {
+                    if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag, wait_ns)) {
                         ok = false;
                         break;
                     }
@@ -493,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!ok) break;
                 umma_commit(bar(B_QEMPTY));  // every S MMA of the unit is issued
                 // the last group: V of the final tile
-                if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag)) ok = false;
+                if (!mbar_wait(bar(B_GFULL0 + gslot), (gc / GS) & 1u, abort_flag, wait_ns)) ok = false;
                 tc_fence_after();
 #pragma unroll
                 for (int t = 0; t < 2; ++t)
@@ -542,7 +542,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lin < n_units) {
             un = decode_unit(unit_of(lin, sc), sc);
             ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile, row,
-                              un.it.rows(t), H + un.it.q0(t), cos_t, sin_t, tab_stride);
+                              un.it.rows(t), H + un.it.q0(t), cos_t, sin_t, tab_stride, wait_ns);
             ++items;
         }
         while (lin < n_units && ok) {
@@ -553,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int min_pos = H + it.q0(t);        // smallest row position of the tile
             const int n_tiles = un.cnt(t);
             for (int j = un.kv_lo; j < un.kv_lo + n_tiles; ++j) {
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + t), s_cnt & 1u, abort_flag));
+                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_SFULL0 + t), s_cnt & 1u, abort_flag, wait_ns));
                 if (!ok) break;
                 ++s_cnt;
                 tc_fence_after();
@@ -639,14 +639,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (next < n_units) {
                 nun = decode_unit(unit_of(next, sc), sc);
                 ok = rope_item<D>(bar(B_QFULL), bar(B_QREADY), static_cast<uint32_t>(items) & 1u, abort_flag, qtile,
-                                  row, nun.it.rows(t), H + nun.it.q0(t), cos_t, sin_t, tab_stride);
+                                  row, nun.it.rows(t), H + nun.it.q0(t), cos_t, sin_t, tab_stride, wait_ns);
                 ++items;
                 if (!ok) break;
             }
             // epilogue: O_T / l -> bf16 -> out, or for a piece the unnormalised O_T and (m, l)
             const size_t prow = (static_cast<size_t>(un.piece) * 2 * BM + t * BM + row);
             if (n_tiles > 0) {
-                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL0 + t), o_cnt & 1u, abort_flag));
+                ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_OFULL0 + t), o_cnt & 1u, abort_flag, wait_ns));
                 if (!ok) break;
                 ++o_cnt;
                 tc_fence_after();
@@ -853,7 +853,7 @@ HostSchedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
 template <int D>
 cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride, const float* cos_t,
                      const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err, int num_sms,
-                     cudaStream_t st, int* n_launched) {
+                     cudaStream_t st, int* n_launched, uint64_t wait_ns) {
     const HostSchedule hs = make_schedule(s, hist, chunk, num_sms);
     Sched sc;
     sc.S = chunk;
@@ -883,7 +883,8 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     kcfg.attrs = kattr;
     kcfg.numAttrs = 1;
     cudaError_t e = cudaLaunchKernelEx(&kcfg, flash_fwd_kernel<D>, maps.q, maps.k, maps.v, sc, s_stride,
-                                       s.n_kv_heads, scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err);
+                                       s.n_kv_heads, scale_log2, cos_t, sin_t, s.max_len, out, ws_o, ws_ml, err,
+                                       wait_ns);
     *n_launched = 1;
     if (e != cudaSuccess || hs.nsplit == 1) return e;
     cudaLaunchConfig_t cfg = {};
@@ -920,11 +921,12 @@ cudaError_t configure_flash_fwd() {
 
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride,
                              const float* cos_t, const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
-                             int num_sms, cudaStream_t st, int* n_launched) {
+                             int num_sms, cudaStream_t st, int* n_launched, uint64_t wait_ns) {
     if (s.head_dim == 128)
         return launch_d<128>(s, maps, hist, chunk, s_stride, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st,
-                             n_launched);
-    return launch_d<64>(s, maps, hist, chunk, s_stride, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched);
+                             n_launched, wait_ns);
+    return launch_d<64>(s, maps, hist, chunk, s_stride, cos_t, sin_t, out, ws_o, ws_ml, err, num_sms, st, n_launched,
+                        wait_ns);
 }
 
 }  // namespace attn

@@ -12,6 +12,11 @@ namespace attn {
 // Error-word bits (mirrors ATTN_DEVERR_* of attn.h).
 constexpr int kDevErrHistRange = 1;
 constexpr int kDevErrTimeout = 2;
+// Default limit of every bounded wait of the kernels (1 s).  The launchers of flash_fwd,
+// decode_split and decode_tc take a limit for the waits of their main loops; the waits
+// that let copies and MMAs already issued finish (before a CTA that gave up exits) always
+// keep this default.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
 struct Shape {
     int batch, n_q_heads, n_kv_heads, head_dim, max_len;
@@ -64,7 +69,7 @@ cudaError_t configure_flash_fwd();
 // q map carries the same stride).
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride,
                              const float* cos_t, const float* sin_t, uint16_t* out, float* ws_o, float* ws_ml, int* err,
-                             int num_sms, cudaStream_t st, int* n_launched);
+                             int num_sms, cudaStream_t st, int* n_launched, uint64_t wait_ns = kWaitLimitNs);
 
 // K3 + K4: decode.  The maps cover the whole caches as 3-D {D, max_len, B*Hkv}
 // with 64-key boxes (built once per cache pair).  K3 also rotates the new key and
@@ -84,7 +89,7 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
                                 const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                                 uint16_t* v_cache,
                                 const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
-                                int nsplit, int* err, cudaStream_t st);
+                                int nsplit, int* err, cudaStream_t st, uint64_t wait_ns = kWaitLimitNs);
 // K3 for head_dim 128 on the tensor cores (decode_tc.cu): one CTA per SM, maps with
 // 128-key boxes; same partial layout as launch_decode_split, but the merge is fused
 // in (the last CTA of each (b, kv head) merges and writes `out`), so no K4 follows.
@@ -108,7 +113,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              uint16_t* v_cache,
                              const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                              int* counters, int nsplit, uint16_t* out, int* err, bool after_decode, int ntok,
-                             cudaStream_t st, bool producer_early = false);
+                             cudaStream_t st, bool producer_early = false, uint64_t wait_ns = kWaitLimitNs);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
                                   const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
 

@@ -54,11 +54,29 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Limits below this are only used to exercise the failure path: such a wait gives up at
+// once unless its phase has already completed (a try_wait may itself block for a while).
+constexpr uint64_t kMinBlockingWaitNs = 1000;
+
 // Wait until the phase with the given parity has completed.  Gives up after
 // `limit_ns` nanoseconds, or as soon as *abort becomes non-zero when `abort` is
 // not null; returns false then.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int* abort,
                                           uint64_t limit_ns = 1000000000ull) {
+    if (limit_ns < kMinBlockingWaitNs) return mbar_test(bar, parity);
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
