@@ -267,8 +267,15 @@ int attn_timing_read(attn_ctx* ctx, double* ms, long long* launches);
  * on different streams, or from several threads -- race on it and must be
  * serialised by the caller.  The first call on each device looks up the array's
  * device address (cudaGetSymbolAddress, with that device current) and caches
- * it; make that first call before any stream capture.  The other arguments and
- * the errors are those of attn_decode; cfg is read on the host only.
+ * it; make that first call before any stream capture.  cudaDeviceReset discards
+ * that set-up (the array and the kernels' attributes are reloaded with new
+ * addresses), so a process that resets a device must not call this entry point on
+ * it afterwards.  A call whose kernels were abandoned part-way (a stream torn down
+ * while they ran) leaves the shared counters undefined until the process exits;
+ * a wait that ran out (ATTN_DEVERR_TIMEOUT) does not: those kernels still finish
+ * and clear them.  The other arguments and the errors are those of attn_decode
+ * (an ATTN_ECUDA leaves its text for attn_last_cuda_error_string); cfg is read on
+ * the host only.
  */
 #define ATTN_NOALLOC_SCRATCH_FLOATS (1 << 20)
 int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, const float* d_sin, const uint16_t* q,

@@ -69,6 +69,14 @@ int cuda_fail(cudaError_t e, const char* where) {
     std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
     return ATTN_ECUDA;
 }
+}  // namespace
+
+namespace attn {
+int record_cuda_error(cudaError_t e, const char* where) { return cuda_fail(e, where); }
+void record_error_text(const char* text) { std::snprintf(g_cuda_msg, sizeof g_cuda_msg, "%s", text); }
+}  // namespace attn
+
+namespace {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

@@ -17,7 +17,9 @@
 // Host code must not pass `g_noalloc_scratch` itself to a kernel: in host code that
 // name denotes a host-side shadow, not device memory.  The device address is looked
 // up with cudaGetSymbolAddress once per device (with that device current) on the
-// first call made on that device, and cached.
+// first call made on that device, and cached.  A cudaDeviceReset unloads the module and
+// with it that set-up (the cached addresses and the kernels' shared-memory limits):
+// after one, the process must not call this entry point on that device again.
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -51,25 +53,32 @@ int setup_device(int dev, float** scratch, int** counters, int* num_sms) {
     if (g_encode == nullptr) {
         cudaDriverEntryPointQueryResult qres;
         void* fn = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qres) !=
-                cudaSuccess ||
-            qres != cudaDriverEntryPointSuccess || fn == nullptr)
+        const cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                                               &qres);
+        if (e != cudaSuccess) return attn::record_cuda_error(e, "attn_decode_noalloc: cuTensorMapEncodeTiled entry point");
+        if (qres != cudaDriverEntryPointSuccess || fn == nullptr) {
+            attn::record_error_text("attn_decode_noalloc: the driver has no cuTensorMapEncodeTiled");
             return ATTN_ECUDA;
+        }
         g_encode = reinterpret_cast<attn::PFN_encodeTiled>(fn);
     }
     if (g_scratch_ptr[dev] == nullptr) {
         int major = 0, minor = 0, sms = 0;
-        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-            return ATTN_ECUDA;
+        cudaError_t e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return attn::record_cuda_error(e, "attn_decode_noalloc: device attributes");
         if (major != 10 || minor != 3) return ATTN_EARCH;
         void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return ATTN_ECUDA;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return attn::record_cuda_error(e, "attn_decode_noalloc: scratch array address");
         void* pc = nullptr;
-        if (cudaGetSymbolAddress(&pc, g_noalloc_counters) != cudaSuccess || pc == nullptr) return ATTN_ECUDA;
+        e = cudaGetSymbolAddress(&pc, g_noalloc_counters);
+        if (e != cudaSuccess) return attn::record_cuda_error(e, "attn_decode_noalloc: counter array address");
+        e = attn::configure_decode();
+        if (e == cudaSuccess) e = attn::configure_decode_tc();
+        if (e != cudaSuccess) return attn::record_cuda_error(e, "attn_decode_noalloc: kernel attributes");
         g_counter_ptr[dev] = static_cast<int*>(pc);
-        if (attn::configure_decode() != cudaSuccess || attn::configure_decode_tc() != cudaSuccess) return ATTN_ECUDA;
         g_num_sms[dev] = sms;
         g_scratch_ptr[dev] = static_cast<float*>(p);
     }
@@ -103,7 +112,12 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     if (per_split > ATTN_NOALLOC_SCRATCH_FLOATS) return ATTN_EINVAL;
 
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ATTN_ECUDA;
+    const cudaError_t de = cudaGetDevice(&dev);
+    if (de != cudaSuccess) return attn::record_cuda_error(de, "attn_decode_noalloc: cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) {
+        attn::record_error_text("attn_decode_noalloc: device ordinal beyond the library's table of 64 devices");
+        return ATTN_ECUDA;
+    }
     float* scratch = nullptr;
     int* counters = nullptr;
     int num_sms = 0;
@@ -123,7 +137,10 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     attn::DecodeMaps maps;
     const cudaError_t me = tc ? attn::make_decode_tc_maps(g_encode, s, k_cache, v_cache, &maps)
                               : attn::make_decode_maps(g_encode, s, k_cache, v_cache, &maps);
-    if (me != cudaSuccess) return ATTN_ECUDA;
+    if (me != cudaSuccess) {
+        attn::record_error_text("attn_decode_noalloc: cuTensorMapEncodeTiled failed for the caches");
+        return ATTN_ECUDA;
+    }
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (tc && static_cast<long long>(cfg->batch) * cfg->n_kv_heads > kNoallocCounters) return ATTN_EINVAL;
     cudaError_t e = tc ? attn::launch_decode_tc(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin, part_o,
@@ -131,5 +148,5 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
                        : attn::launch_decode_split(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin,
                                                    part_o, part_ml, nsplit, d_err, st);
     if (e == cudaSuccess && !tc) e = attn::launch_decode_combine(s, d_hist_len, 0, part_o, part_ml, nsplit, out, st);
-    return e == cudaSuccess ? ATTN_OK : ATTN_ECUDA;
+    return e == cudaSuccess ? ATTN_OK : attn::record_cuda_error(e, "attn_decode_noalloc: launch");
 }

@@ -12,6 +12,12 @@ namespace attn {
 // Error-word bits (mirrors ATTN_DEVERR_* of attn.h).
 constexpr int kDevErrHistRange = 1;
 constexpr int kDevErrTimeout = 2;
+// The thread's last failure text, read by attn_last_cuda_error_string (attn_api.cu).
+// record_cuda_error formats a CUDA error with the failing step and returns ATTN_ECUDA
+// (-3); record_error_text stores a plain text.
+int record_cuda_error(cudaError_t e, const char* where);
+void record_error_text(const char* text);
+
 // Default limit of every bounded wait of the kernels (1 s).  The launchers of flash_fwd,
 // decode_split and decode_tc take a limit for the waits of their main loops; the waits
 // that let copies and MMAs already issued finish (before a CTA that gave up exits) always

@@ -42,24 +42,39 @@ def rope_tables(shape):
     return np.cos(ang).astype(np.float32), np.sin(ang).astype(np.float32)
 
 
-def test_noalloc_decode_matches_attn_decode_on_two_calls(env):
+# head_dim 128 runs the tensor-core decode (its merge fused in, counters in the static
+# array); head_dim 64 runs the CUDA-core split kernel and the merge kernel, both reading
+# and writing the static partials.  The scratch cap never binds below attn_decode's own
+# split count for these kernels' split rules (it would need more than 50 query heads per
+# kv head), so both calls run attn_decode's split count.
+CASES = [
+    ("d128_b4", Shape("noalloc128", 4, 32, 8, 128, 8192, 5.0e5), 8191,
+     ([1024, 4096, 8191, 17], [5, 0, 8000, 3000])),
+    ("d64_b3", Shape("noalloc64", 3, 4, 2, 64, 64, 1.0e4), 60, ([24, 5, 63], [0, 40, 27])),
+]
+
+
+@pytest.mark.parametrize("name,shape,n_hist,calls", CASES, ids=[c[0] for c in CASES])
+def test_noalloc_decode_matches_attn_decode_and_the_oracle_on_two_calls(env, name, shape, n_hist, calls):
+    from oracle import oracle as O
     torch, _lib, lib = env
     from paper_2607_15865_gb300.attention import Attention
-    shape = Shape("noalloc", 4, 32, 8, 128, 8192, 5.0e5)
     cfg = _lib.AttnCfg(shape.batch, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.max_len,
                        shape.rope_theta)
     ctab, stab = rope_tables(shape)
     d_cos, d_sin = torch.from_numpy(ctab).cuda(), torch.from_numpy(stab).cuda()
     attn = Attention.for_shape(shape)
-    kc, vc = w.cache(shape, "noalloc", 8191, fill="random")
+    kc, vc = w.cache(shape, "noalloc", n_hist, fill="random")
     ref_k, ref_v = to_dev(kc), to_dev(vc)
     new_k, new_v = to_dev(kc), to_dev(vc)
+    ork, orv = kc.copy(), vc.copy()  # the oracle's own caches
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
     stream = torch.cuda.current_stream()
-    for call, hist in enumerate(([1024, 4096, 8191, 17], [5, 0, 8000, 3000])):
+    for call, hist in enumerate(calls):
         q, k, v = w.tokens(shape, f"noalloc{call}", 1)
         hl = torch.tensor(hist, dtype=torch.int32, device="cuda")
         ref = attn.decode(to_dev(q), to_dev(k), to_dev(v), hl, ref_k, ref_v)
+        oref = O.decode(shape, q, k, v, np.asarray(hist, np.int32), ork, orv)
         dq, dk, dv = to_dev(q), to_dev(k), to_dev(v)
         out = torch.empty_like(dq)
         rc = lib.attn_decode_noalloc(ctypes.byref(cfg), d_cos.data_ptr(), d_sin.data_ptr(), dq.data_ptr(),
@@ -69,9 +84,13 @@ def test_noalloc_decode_matches_attn_decode_on_two_calls(env):
         torch.cuda.synchronize()
         assert int(err.item()) == 0, "the no-alloc decode set an error bit"
         assert attn.device_error() == 0
-        assert_out_close(to_host(out), to_host(ref), f"no-alloc decode, call {call + 1}")
+        got = to_host(out)
+        assert_out_close(got, to_host(ref), f"{name}: no-alloc vs attn_decode, call {call + 1}")
+        assert_out_close(got, oref, f"{name}: no-alloc vs the oracle, call {call + 1}")
         assert ulp_diff(to_host(new_k), to_host(ref_k)).max() <= 1, f"k cache differs, call {call + 1}"
         assert (to_host(new_v) == to_host(ref_v)).all(), f"v cache differs, call {call + 1}"
+        assert ulp_diff(to_host(new_k), ork).max() <= 1, f"k cache differs from the oracle's, call {call + 1}"
+        assert (to_host(new_v) == orv).all(), f"v cache differs from the oracle's, call {call + 1}"
     attn.close()
 
 
