@@ -169,3 +169,31 @@ def dequant_bf16(codes, scales_bf16, zeros) -> np.ndarray:
 def gemm_bf16w(codes, scales_bf16, zeros, x_bf16) -> np.ndarray:
     """Y [T, N] float64 = x [T, K] . W_bf16[N, K]^T."""
     return bf16_to_f64(x_bf16) @ bf16_to_f64(dequant_bf16(codes, scales_bf16, zeros)).T
+
+
+# ----------------------------------------------------------------------------- the block around attention, prefill
+# Listing 1 for a prefill (hist = 0, Section 4.2) or prefill_kv (hist > 0, Section 4.3) chunk
+# of S tokens per sequence, with the prefill-side projections (weights rounded once to bf16):
+#   xn = RMSNorm(x) * gamma               per token
+#   q | k | v = xn . Wqkv_bf16^T          rounded to bf16
+#   o = attention of the chunk over its history (RoPE, cache append, causal mask)
+#   h = x + o . Wo_bf16^T                 rounded to bf16
+
+
+def prefill_layer(shape, x_bf16, gamma_bf16, eps, wqkv, wo, hist, k_cache, v_cache, attn_oracle=None):
+    """h (bf16 bits [B, S, hidden]) of one chunk of S tokens per sequence over `hist`
+    history tokens (the same for every sequence); x is [B, S, hidden].  The caches get the
+    chunk's rotated k and its v at slots hist .. hist + S - 1, as the prefill stages do."""
+    if attn_oracle is None:
+        from oracle import oracle as attn_oracle
+    B, S, hidden = np.shape(x_bf16)
+    D = shape.head_dim
+    qd, kd = shape.n_q_heads * D, shape.n_kv_heads * D
+    x2 = np.asarray(x_bf16, dtype=np.uint16).reshape(B * S, hidden)
+    xn = rmsnorm(x2, gamma_bf16, eps)
+    qkv = to_bf16_bits(gemm_bf16w(*wqkv, xn))
+    q = qkv[:, :qd].reshape(B, S, shape.n_q_heads, D).copy()
+    k = qkv[:, qd:qd + kd].reshape(B, S, shape.n_kv_heads, D).copy()
+    v = qkv[:, qd + kd:].reshape(B, S, shape.n_kv_heads, D).copy()
+    o = attn_oracle.prefill_kv(shape, q, k, v, int(hist), k_cache, v_cache).reshape(B * S, qd)
+    return to_bf16_bits(bf16_to_f64(x2) + gemm_bf16w(*wo, o)).reshape(B, S, hidden)

@@ -7,8 +7,8 @@ tokens over those 16, then 4 decodes (Section 4.1, scenario 2).  It guards the
 oracle against unnoticed drift; the oracle itself is pinned by
 tests/oracle_pins.py.  w4_tiny.json does the same for the W4BF16 oracle
 (oracle/w4_oracle.py, pinned by tests/w4_oracle_pins.py): the tile stream of a small
-matrix, its GEMV, RMSNorm, the prefill-side GEMM and one decode step of the block around
-attention, every float64 result rounded to bf16 before it is hashed.
+matrix, its GEMV, RMSNorm, the prefill-side GEMM, one decode step and one prefill_kv chunk
+of the block around attention, every float64 result rounded to bf16 before it is hashed.
 Run:  python tests/golden/make_golden.py
 """
 import hashlib
@@ -65,6 +65,11 @@ def w4_tiny():
     kc, vc = w.cache(sh, "golden_w4", 20, fill="random")
     out["block_h"] = W.decode_layer(sh, xb, gb, 1e-6, wq, wo, np.array([5, 20], np.int32), kc, vc)
     out["block_k_cache"], out["block_v_cache"] = kc, vc
+    # the prefill side: a 7-token chunk of each of the two sequences over 21 history tokens
+    xp = gen.normal_bf16("golden_w4", "xp", (2, 7, hidden), 1.0)
+    kc, vc = w.cache(sh, "golden_w4_prefill", 21, fill="random")
+    out["prefill_block_h"] = W.prefill_layer(sh, xp, gb, 1e-6, wq, wo, 21, kc, vc)
+    out["prefill_block_k_cache"], out["prefill_block_v_cache"] = kc, vc
     return out
 
 

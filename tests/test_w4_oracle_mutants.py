@@ -5,7 +5,9 @@ Each mutant is oracle/w4_oracle.py with one plausible mistake substituted in (a 
 nibble order or tile transpose, a tile writer that misplaces a scale byte, a code row or a
 zero point, a dropped zero point, a wrong group, a wrong bf16 decode
 or rounding, RMSNorm without eps or gamma or with a sum for the mean, a block without its
-residual or RMSNorm, k and v swapped, q read from the wrong rows, GEMM weights not rounded),
+residual or RMSNorm, k and v swapped, q read from the wrong rows, GEMM weights not rounded; the
+prefill block without its residual or RMSNorm, with k and v swapped, q from the wrong rows,
+unrounded projection weights, or its history ignored),
 loaded as a separate module.  The real oracle is never modified.
 """
 import os
@@ -30,12 +32,20 @@ MUTANTS = {
     "rmsnorm_sum_for_mean": ("np.mean(x * x, axis=-1", "np.sum(x * x, axis=-1"),
     "block_without_residual": ("return to_bf16_bits(bf16_to_f64(x_bf16) + gemv(*wo, o))", "return to_bf16_bits(gemv(*wo, o))"),
     "block_without_rmsnorm": ("xn = rmsnorm(x_bf16, gamma_bf16, eps)", "xn = x_bf16"),
-    "block_k_v_swapped": ("v = qkv[:, qd + kd:].reshape", "v = qkv[:, qd:qd + kd].reshape"),
-    "block_q_from_wrong_rows": ("q = qkv[:, :qd].reshape", "q = qkv[:, kd:kd + qd].reshape"),
+    "block_k_v_swapped": ("v = qkv[:, qd + kd:].reshape(B, 1,", "v = qkv[:, qd:qd + kd].reshape(B, 1,"),
+    "block_q_from_wrong_rows": ("q = qkv[:, :qd].reshape(B, 1,", "q = qkv[:, kd:kd + qd].reshape(B, 1,"),
     "writer_scale_bytes_swapped": ("buf[at.ravel()] = (s & 0xFF)", "buf[at.ravel()] = (s >> 8)"),
     "writer_code_byte_ignores_row": ("+ 64 * (n % TILE_ROWS) + 4 *", "+ 4 *"),
     "writer_zero_point_in_scale_bytes": ("buf[(rec * TILE_BYTES + ZERO_OFFSET + n % TILE_ROWS)",
                                          "buf[(rec * TILE_BYTES + SCALE_OFFSET + n % TILE_ROWS)"),
+    "prefill_block_without_residual": ("return to_bf16_bits(bf16_to_f64(x2) + gemm_bf16w(*wo, o)).reshape(B, S, hidden)",
+                                       "return to_bf16_bits(gemm_bf16w(*wo, o)).reshape(B, S, hidden)"),
+    "prefill_block_without_rmsnorm": ("xn = rmsnorm(x2, gamma_bf16, eps)", "xn = x2"),
+    "prefill_block_k_v_swapped": ("v = qkv[:, qd + kd:].reshape(B, S", "v = qkv[:, qd:qd + kd].reshape(B, S"),
+    "prefill_block_q_from_wrong_rows": ("q = qkv[:, :qd].reshape(B, S", "q = qkv[:, kd:kd + qd].reshape(B, S"),
+    "prefill_block_weights_not_rounded": ("qkv = to_bf16_bits(gemm_bf16w(*wqkv, xn))", "qkv = to_bf16_bits(gemv(*wqkv, xn))"),
+    "prefill_block_history_ignored": ("o = attn_oracle.prefill_kv(shape, q, k, v, int(hist), k_cache, v_cache)",
+                                      "o = attn_oracle.prefill_kv(shape, q, k, v, 0, k_cache, v_cache)"),
     "gemm_weights_not_rounded": ("@ bf16_to_f64(dequant_bf16(codes, scales_bf16, zeros)).T",
                                  "@ dequant(codes, scales_bf16, zeros).T"),
 }

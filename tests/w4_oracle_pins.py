@@ -201,4 +201,91 @@ def pin_gemm_rounds_each_weight_once(W):
     assert np.allclose(W.gemm_bf16w(codes, s, zeros, x), ref, rtol=1e-12, atol=1e-12)
 
 
-ALL_PINS = [pin_gemm_rounds_each_weight_once, pin_writer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v]
+def _prefill_case(shape, S, tag, pow2_scales=False, q_zero=False, wo_kind="random"):
+    """Inputs of one prefill-block chunk for the pins: (x [B, S, hidden], gamma, wqkv, wo)."""
+    D, hq, hkv = shape.head_dim, shape.n_q_heads, shape.n_kv_heads
+    qd, kd, hidden = hq * D, hkv * D, hq * D
+    x = gen.normal_bf16("w4pin", f"{tag}_x", (shape.batch, S, hidden), 1.0)
+    gamma = gen.normal_bf16("w4pin", f"{tag}_g", (hidden,), 1.0)
+
+    def scales(name, rows, groups):
+        if pow2_scales:  # every (q - z) s exact in bf16: the GEMM reading equals the exact product
+            e = gen.uint4_codes("w4pin", f"{tag}_{name}e", (rows, groups)) % 4
+            return gen.f32_to_bf16_bits((2.0 ** -(5.0 + e)).astype(np.float32))
+        return gen.normal_bf16("w4pin", f"{tag}_{name}", (rows, groups), 0.02) & np.uint16(0x7FFF)
+
+    zq = gen.uint4_codes("w4pin", f"{tag}_zq", (qd + 2 * kd, hidden // 128)) % 15
+    cq = gen.uint4_codes("w4pin", f"{tag}_cq", (qd + 2 * kd, hidden))
+    if q_zero:
+        cq[:qd] = np.repeat(zq[:qd], 128, axis=1)
+    sq = scales("sq", qd + 2 * kd, hidden // 128)
+    zo = gen.uint4_codes("w4pin", f"{tag}_zo", (hidden, qd // 128)) % 15
+    so = scales("so", hidden, qd // 128)
+    if wo_kind == "zero":
+        co = np.repeat(zo, 128, axis=1)
+    elif wo_kind == "identity":
+        co = np.repeat(zo, 128, axis=1)
+        co[np.arange(hidden), np.arange(hidden)] += 1
+        so = gen.f32_to_bf16_bits(np.ones((hidden, qd // 128), np.float32))
+    else:
+        co = gen.uint4_codes("w4pin", f"{tag}_co", (hidden, qd))
+    return x, gamma, (cq, sq, zq), (co, so, zo)
+
+
+def pin_prefill_layer_equals_a_chain_of_decode_layers(W):
+    """Section 4.1: a chunk through the prefill block equals its tokens one by one through the
+    decode block (with weights exact in bf16 the two projection readings coincide): h and the
+    caches bit for bit."""
+    from synthetic import workloads as w
+    from synthetic.workloads import Shape
+    shape = Shape("w4pre_a", 2, 4, 2, 64, 320, 1.0e4)
+    S, hist = 9, 131
+    x, gamma, wqkv, wo = _prefill_case(shape, S, "pc", pow2_scales=True)
+    kc, vc = w.cache(shape, "pc_cache", hist, fill="random")
+    kc2, vc2 = kc.copy(), vc.copy()
+    h = W.prefill_layer(shape, x, gamma, 1e-6, wqkv, wo, hist, kc, vc)
+    for t in range(S):
+        ht = W.decode_layer(shape, x[:, t].copy(), gamma, 1e-6, wqkv, wo, np.full(shape.batch, hist + t, np.int32),
+                            kc2, vc2)
+        assert (h[:, t] == ht).all(), t
+    assert (kc == kc2).all() and (vc == vc2).all()
+
+
+def pin_prefill_layer_residual_only_when_o_proj_is_zero(W):
+    from synthetic import workloads as w
+    from synthetic.workloads import Shape
+    shape = Shape("w4pre_b", 1, 4, 1, 128, 300, 1.0e4)
+    x, gamma, wqkv, wo = _prefill_case(shape, 70, "pz", wo_kind="zero")
+    kc, vc = w.cache(shape, "pz_cache", 0, fill="random")
+    assert (W.prefill_layer(shape, x, gamma, 1e-6, wqkv, wo, 0, kc, vc) == x).all()
+
+
+def pin_prefill_layer_with_q_zero_and_identity_o_proj_averages_v(W):
+    """q = 0: token i of the chunk weighs its hist + i + 1 visible keys equally, so with
+    o_proj = I the block returns x + the mean of those v rows (the chunk's own v rows being
+    its v projection of RMSNorm(x))."""
+    from synthetic import workloads as w
+    from synthetic.workloads import Shape
+    shape = Shape("w4pre_c", 2, 4, 2, 64, 256, 1.0e4)
+    S, hist = 6, 40
+    x, gamma, wqkv, wo = _prefill_case(shape, S, "pq", q_zero=True, wo_kind="identity")
+    kc, vc = w.cache(shape, "pq_cache", hist, fill="random")
+    h = W.prefill_layer(shape, x, gamma, 1e-6, wqkv, wo, hist, kc, vc)
+    G, D = shape.n_q_heads // shape.n_kv_heads, shape.head_dim
+    qd, kd = shape.n_q_heads * D, shape.n_kv_heads * D
+    wv = tuple(a[qd + kd:] for a in wqkv)
+    hidden = x.shape[-1]
+    xn = W.rmsnorm(x.reshape(-1, hidden), gamma, 1e-6)
+    v_new = W.to_bf16_bits(W.gemm_bf16w(*wv, xn)).reshape(shape.batch, S, shape.n_kv_heads, D)
+    for b in range(shape.batch):
+        for i in range(S):
+            assert (vc[b, :, hist + i] == v_new[b, i]).all()
+            o = np.concatenate([W.bf16_to_f64(vc[b, hq // G, :hist + i + 1]).mean(axis=0)
+                                for hq in range(shape.n_q_heads)])
+            want = W.to_bf16_bits(W.bf16_to_f64(x[b, i]) + W.bf16_to_f64(W.to_bf16_bits(o)))
+            assert (h[b, i] == want).all(), (b, i)
+
+
+ALL_PINS = [pin_gemm_rounds_each_weight_once, pin_writer_and_reader_agree_on_the_format, pin_single_values_land_where_the_format_says, pin_gemv_matches_brute_force, pin_gemv_closed_forms, pin_bf16_rounding_is_nearest_even, pin_rmsnorm_brute_force_and_closed_forms, pin_decode_layer_residual_only_when_o_proj_is_zero, pin_decode_layer_with_q_zero_and_identity_o_proj_averages_v,
+            pin_prefill_layer_equals_a_chain_of_decode_layers, pin_prefill_layer_residual_only_when_o_proj_is_zero,
+            pin_prefill_layer_with_q_zero_and_identity_o_proj_averages_v]
