@@ -354,6 +354,35 @@ int attn_decode_layer(attn_ctx* ctx, const uint16_t* x, const uint16_t* rms_gamm
                       const void* wqkv_tiles, const void* wo_tiles, int hidden, const int32_t* d_hist_len,
                       uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, int flags, attn_stream_t stream);
 
+/*
+ * The attention half of a decoder block for a prefill (hist_len = 0, Section 4.2) or
+ * prefill_kv (Section 4.3) chunk, with W4BF16 weights (Listing 1's dataflow):
+ *   xn = bf16(x * r * rms_gamma), r = 1 / sqrt(mean(x^2) + rms_eps)    per token
+ *   q | k | v = bf16(xn . Wqkv^T)        each weight rounded once to bf16 (attn_w4bf16_gemm)
+ *   out = the prefill_kv stage of q, k, v over hist_len history tokens (RoPE, in-place
+ *         cache append at slots hist_len .. hist_len + chunk_len - 1, causal GQA attention)
+ *   h_out = bf16(x + out . Wo^T)
+ *   x, h_out   device bf16 [batch][chunk_len][hidden], 16-byte aligned; h_out may be x
+ *   rms_gamma  device bf16 [hidden];  rms_eps >= 0, finite
+ *   wqkv_tiles the tile stream (attn_w4bf16_gemv's format) of the stacked
+ *              [(n_q_heads + 2 n_kv_heads) head_dim, hidden] matrix: q_proj rows, then
+ *              k_proj, then v_proj;  wo_tiles: that of the [hidden, n_q_heads head_dim] o_proj
+ *   k_cache, v_cache as for attn_prefill_kv
+ *   workspace  device memory of at least attn_prefill_layer_workspace(ctx, hidden,
+ *              chunk_len) bytes, 256-byte aligned, owned by the caller (the normalised x,
+ *              q, k, v and the attention output live there; nothing is allocated)
+ * hidden, n_q_heads head_dim and (n_q_heads + 2 n_kv_heads) head_dim multiples of 128;
+ * 1 <= chunk_len, hist_len + chunk_len <= max_len, batch * chunk_len <= 65535 * 128.
+ * Enqueues four launches on `stream` (RMSNorm, QKV GEMM, attention, o_proj GEMM); a
+ * wait that runs out sets ATTN_DEVERR_TIMEOUT in the context's error word.  Returns
+ * ATTN_OK, ATTN_EINVAL, ATTN_EARCH or ATTN_ECUDA.
+ */
+size_t attn_prefill_layer_workspace(const attn_ctx* ctx, int hidden, int chunk_len);
+int attn_prefill_layer(attn_ctx* ctx, const uint16_t* x, const uint16_t* rms_gamma, float rms_eps,
+                       const void* wqkv_tiles, const void* wo_tiles, int hidden, int hist_len, int chunk_len,
+                       uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, void* workspace,
+                       size_t workspace_bytes, attn_stream_t stream);
+
 /* W4BF16 weight GEMM of the prefill-side projections (Listing 1's q/k/v/o_proj over a
  * chunk of T tokens; Section 5.1 W4BF16), on the tensor cores:
  *   y[t][n] = bf16( sum_{k<K} x[t][k] * W[n][k] ),  W[n][k] = bf16((q - z) * s)

@@ -22,7 +22,7 @@ EXPORTED = ("attn_create", "attn_destroy", "attn_prefill", "attn_prefill_kv", "a
             "attn_timing_enable", "attn_timing_read",
             "attn_strerror", "attn_last_cuda_error_string", "attn_decode_noalloc", "attn_w4bf16_gemv",
             "attn_w4bf16_rows_per_launch", "attn_w4bf16_gemv_fused", "attn_decode_layer",
-            "attn_w4bf16_gemm")
+            "attn_w4bf16_gemm", "attn_prefill_layer", "attn_prefill_layer_workspace")
 NOALLOC_SCRATCH_FLOATS = 1 << 20
 KERNELS = ("rope_append", "flash_fwd", "decode_split", "decode_combine")
 
@@ -90,6 +90,11 @@ def load(path: str = LIB_PATH):
     lib.attn_w4bf16_gemv_fused.restype = i32
     lib.attn_decode_layer.argtypes = [vp, u16p, u16p, ctypes.c_float, vp, vp, i32, vp, u16p, u16p, u16p, i32, vp]
     lib.attn_decode_layer.restype = i32
+    lib.attn_prefill_layer.argtypes = [vp, u16p, u16p, ctypes.c_float, vp, vp, i32, i32, i32, u16p, u16p, u16p, vp,
+                                       ctypes.c_size_t, vp]
+    lib.attn_prefill_layer.restype = i32
+    lib.attn_prefill_layer_workspace.argtypes = [vp, i32, i32]
+    lib.attn_prefill_layer_workspace.restype = ctypes.c_size_t
     lib.attn_w4bf16_gemm.argtypes = [vp, u16p, i32, i32, i32, u16p, vp, vp]
     lib.attn_w4bf16_gemm.restype = i32
     lib.attn_w4bf16_rows_per_launch.argtypes = [i32]

@@ -162,6 +162,42 @@ class Attention:
         self._check(rc, "attn_decode_layer")
         return out
 
+    def prefill_layer(self, x, rms_gamma, rms_eps: float, wqkv_tiles, wo_tiles, hist_len: int, k_cache, v_cache,
+                      out=None, workspace=None, stream=None) -> torch.Tensor:
+        """The attention half of a decoder block over a prefill / prefill_kv chunk with W4BF16
+        weights (attn_prefill_layer): x [B, S, hidden] -> x + o_proj(attention(qkv_proj(RMSNorm(x)))),
+        the chunk at positions hist_len ..  workspace: a uint8 CUDA tensor of at least
+        prefill_layer_workspace(hidden, S) bytes (allocated here when None)."""
+        if x.dim() != 3 or x.shape[0] != self.batch:
+            raise ValueError("x must be [batch, chunk_len, hidden]")
+        S, hidden = x.shape[1], x.shape[2]
+        for t, name in ((wqkv_tiles, "wqkv_tiles"), (wo_tiles, "wo_tiles")):
+            if not (isinstance(t, torch.Tensor) and t.is_cuda and t.is_contiguous() and t.dtype == torch.uint8):
+                raise TypeError(f"{name} must be a contiguous uint8 CUDA tensor (a W4BF16 tile stream)")
+        qd, kd = self.n_q_heads * self.head_dim, self.n_kv_heads * self.head_dim
+        if wqkv_tiles.numel() != (qd + 2 * kd + 15) // 16 * (hidden // 128) * 1072 or \
+                wo_tiles.numel() != (hidden + 15) // 16 * (qd // 128) * 1072:
+            raise ValueError("tile streams must hold [(Hq + 2 Hkv) D, hidden] and [hidden, Hq D] matrices")
+        need = self.prefill_layer_workspace(hidden, S)
+        if workspace is None:
+            workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+        if not (isinstance(workspace, torch.Tensor) and workspace.is_cuda and workspace.dtype == torch.uint8
+                and workspace.is_contiguous() and workspace.numel() >= need):
+            raise TypeError(f"workspace must be a contiguous uint8 CUDA tensor of at least {need} bytes")
+        xs = (self.batch, S, hidden)
+        out = self._new_out(x, out)
+        rc = self.lib.attn_prefill_layer(self._ctx, _ptr(x, "x", xs), _ptr(rms_gamma, "rms_gamma", (hidden,)),
+                                         float(rms_eps), wqkv_tiles.data_ptr(), wo_tiles.data_ptr(), hidden,
+                                         int(hist_len), S, _ptr(k_cache, "k_cache", self._cache_shape()),
+                                         _ptr(v_cache, "v_cache", self._cache_shape()), _ptr(out, "out", xs),
+                                         workspace.data_ptr(), workspace.numel(), _stream(stream))
+        self._check(rc, "attn_prefill_layer")
+        return out
+
+    def prefill_layer_workspace(self, hidden: int, chunk_len: int) -> int:
+        """Bytes of device workspace attn_prefill_layer needs (host only)."""
+        return int(self.lib.attn_prefill_layer_workspace(self._ctx, int(hidden), int(chunk_len)))
+
     def prompt(self, q, k, v, hist_len: int, seg_len: int, k_cache, v_cache, out=None,
                stream=None) -> torch.Tensor:
         """The whole prompt q [B,P,Hq,D], k/v [B,P,Hkv,D] at positions hist_len.. in segments of seg_len."""

@@ -532,6 +532,74 @@ int attn_w4bf16_gemv_fused(const void* w_tiles, const uint16_t* x, int M, int N,
     return ATTN_OK;
 }
 
+namespace {
+// Workspace of attn_prefill_layer: xn [T][hidden], q [T][qd], k and v [T][kd], the attention
+// output [T][qd] (T = batch * chunk_len), each region starting at a 256-byte boundary.
+struct PrefillWs {
+    size_t xn, q, k, v, o, bytes;
+};
+PrefillWs prefill_ws(const attn_cfg& cfg, int hidden, int chunk_len) {
+    const size_t T = static_cast<size_t>(cfg.batch) * chunk_len;
+    const size_t qd = static_cast<size_t>(cfg.n_q_heads) * cfg.head_dim, kd = static_cast<size_t>(cfg.n_kv_heads) * cfg.head_dim;
+    auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
+    PrefillWs w;
+    w.xn = 0;
+    w.q = w.xn + up(T * hidden * 2);
+    w.k = w.q + up(T * qd * 2);
+    w.v = w.k + up(T * kd * 2);
+    w.o = w.v + up(T * kd * 2);
+    w.bytes = w.o + up(T * qd * 2);
+    return w;
+}
+}  // namespace
+
+size_t attn_prefill_layer_workspace(const attn_ctx* c, int hidden, int chunk_len) {
+    if (c == nullptr || hidden < 1 || chunk_len < 1) return 0;
+    return prefill_ws(c->cfg, hidden, chunk_len).bytes;
+}
+
+int attn_prefill_layer(attn_ctx* c, const uint16_t* x, const uint16_t* rms_gamma, float rms_eps,
+                       const void* wqkv_tiles, const void* wo_tiles, int hidden, int hist_len, int chunk_len,
+                       uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, void* workspace, size_t workspace_bytes,
+                       attn_stream_t stream) {
+    if (c == nullptr || x == nullptr || rms_gamma == nullptr || wqkv_tiles == nullptr || wo_tiles == nullptr ||
+        k_cache == nullptr || v_cache == nullptr || h_out == nullptr || workspace == nullptr)
+        return ATTN_EINVAL;
+    const int qd = c->cfg.n_q_heads * c->cfg.head_dim, kd = c->cfg.n_kv_heads * c->cfg.head_dim;
+    if (hidden < 128 || hidden % 128 != 0 || qd % 128 != 0 || (qd + 2 * kd) % 128 != 0) return ATTN_EINVAL;
+    if (chunk_len < 1 || hist_len < 0 || static_cast<long>(hist_len) + chunk_len > c->cfg.max_len) return ATTN_EINVAL;
+    const long long T = static_cast<long long>(c->cfg.batch) * chunk_len;
+    if (T > 65535LL * 128 || !std::isfinite(rms_eps) || rms_eps < 0.f) return ATTN_EINVAL;
+    if (!aligned16(x) || !aligned16(rms_gamma) || !aligned16(wqkv_tiles) || !aligned16(wo_tiles) ||
+        !aligned16(h_out) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
+        return ATTN_EINVAL;
+    const PrefillWs ws = prefill_ws(c->cfg, hidden, chunk_len);
+    if (workspace_bytes < ws.bytes) return ATTN_EINVAL;
+    uint8_t* wb = static_cast<uint8_t*>(workspace);
+    uint16_t* xn = reinterpret_cast<uint16_t*>(wb + ws.xn);
+    uint16_t* q = reinterpret_cast<uint16_t*>(wb + ws.q);
+    uint16_t* k = reinterpret_cast<uint16_t*>(wb + ws.k);
+    uint16_t* v = reinterpret_cast<uint16_t*>(wb + ws.v);
+    uint16_t* o = reinterpret_cast<uint16_t*>(wb + ws.o);
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    // input_layernorm: one factor per token, a pre-pass over the chunk
+    cudaError_t e = attn::launch_rmsnorm_rows(x, rms_gamma, rms_eps, static_cast<int>(T), hidden, xn, st);
+    if (e != cudaSuccess) return cuda_fail(e, "prefill layer RMSNorm");
+    // q/k/v projections: one GEMM over the stacked rows, the output split three ways
+    attn::W4GemmEpi split = {qd, qd + kd, k, v, nullptr};
+    e = attn::launch_w4_gemm(static_cast<const uint8_t*>(wqkv_tiles), xn, static_cast<int>(T), qd + 2 * kd, hidden, q,
+                             c->d_err, st, &split);
+    if (e != cudaSuccess) return cuda_fail(e, "prefill layer QKV GEMM");
+    // RoPE of q and k, cache append, causal attention over the history (the prefill stages)
+    const int rc = run_prefill(c, q, k, v, hist_len, chunk_len, chunk_len, k_cache, v_cache, o, st);
+    if (rc != ATTN_OK) return rc;
+    // o_proj with the residual in the epilogue (h may be x)
+    attn::W4GemmEpi res = {hidden, hidden, nullptr, nullptr, x};
+    e = attn::launch_w4_gemm(static_cast<const uint8_t*>(wo_tiles), o, static_cast<int>(T), hidden, qd, h_out, c->d_err,
+                             st, &res);
+    return e == cudaSuccess ? ATTN_OK : cuda_fail(e, "prefill layer o_proj GEMM");
+}
+
 int attn_decode_layer(attn_ctx* c, const uint16_t* x, const uint16_t* rms_gamma, float rms_eps,
                       const void* wqkv_tiles, const void* wo_tiles, int hidden, const int32_t* d_hist_len,
                       uint16_t* k_cache, uint16_t* v_cache, uint16_t* h_out, int flags, attn_stream_t stream) {

@@ -150,8 +150,23 @@ cudaError_t launch_w4_gemv(const uint8_t* tiles, const uint16_t* x, int M, int N
 // W4BF16 GEMM (w4_gemm.cu): y[t, n] = sum_k x[t, k] bf16((q - z) s)[n, k] for T tokens;
 // N and K multiples of 128; x bf16 [T][K] and y bf16 [T][N] 16-byte aligned; tiles: the
 // tile stream of attn_w4bf16_gemv.
+// Epilogue options (all optional): the output columns split three ways -- [0, n0) -> y
+// (row stride n0), [n0, n1) -> y1, [n1, N) -> y2 (n0, n1 multiples of 32; no split: n0 =
+// n1 = N) -- or a bf16 residual [T][N] added in float before rounding (unsplit only; it
+// may be y itself: each element is read before it is written).
+struct W4GemmEpi {
+    int n0, n1;
+    uint16_t* y1;
+    uint16_t* y2;
+    const uint16_t* residual;
+};
 cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N, int K, uint16_t* y, int* err,
-                           cudaStream_t st);
+                           cudaStream_t st, const W4GemmEpi* epi = nullptr);
+// RMSNorm of T rows of x (bf16 [T][K], K a multiple of 8, 16-byte aligned) into xn (same
+// shape): xn = bf16(x * r * gamma), r = 1 / sqrt(mean_k x^2 + eps) per row, float math (the
+// sum of squares in a fixed order); gamma bf16 [K].
+cudaError_t launch_rmsnorm_rows(const uint16_t* x, const uint16_t* gamma, float eps, int T, int K, uint16_t* xn,
+                                cudaStream_t st);
 
 #ifdef __CUDACC__
 // Position of sequence b's decode token: d_hist[b] + hist_add, or -1 (out of range, so

@@ -17,7 +17,10 @@
 //     per word;
 //   * warp 1, one lane: 8 tcgen05.mma (kind::f16, 128 x 128 x 16) per group into one TMEM
 //     accumulator, committing the x stage and the B buffer back to their producers;
-//   * warps 2..5 again: the epilogue, 32 TMEM lanes (tokens) each, rounded to bf16.
+//   * warps 2..5 again: the epilogue, 32 TMEM lanes (tokens) each: optionally the residual
+//     added in float, rounded to bf16, the columns optionally split three ways (q, k, v).
+// rmsnorm_rows_kernel is the block's input_layernorm for a chunk: one factor per token,
+// so it runs as a pre-pass over the chunk before the stacked QKV GEMM.
 // Every wait is bounded (ATTN_DEVERR_TIMEOUT in *err, then the CTA drains and exits).
 #include <cuda_bf16.h>
 
@@ -92,7 +95,7 @@ __device__ __forceinline__ uint32_t code_pair(uint32_t w, int j, uint32_t mask, 
 
 __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_constant__ CUtensorMap map_x,
                                                               const uint8_t* __restrict__ tiles, int T, int N, int K,
-                                                              uint16_t* __restrict__ y, int* err) {
+                                                              uint16_t* __restrict__ y, int* err, const W4GemmEpi epi) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -244,14 +247,41 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                 uint32_t r[32];
                 tmem_ld32(tmem + (static_cast<uint32_t>(q * 32) << 16) + 32u * c, r);
                 tmem_wait_ld();
-                if (m < T && n0 + 32 * c < N) {
-                    uint4* dst = reinterpret_cast<uint4*>(y + static_cast<size_t>(m) * N + n0 + 32 * c);
+                const int col = n0 + 32 * c;
+                if (m < T && col < N) {
+                    // destination of these 32 columns: y, or a part of the split output
+                    uint16_t* base_ptr = y;
+                    int stride = epi.n0, cc = col;
+                    if (col >= epi.n1) {
+                        base_ptr = epi.y2;
+                        stride = N - epi.n1;
+                        cc = col - epi.n1;
+                    } else if (col >= epi.n0) {
+                        base_ptr = epi.y1;
+                        stride = epi.n1 - epi.n0;
+                        cc = col - epi.n0;
+                    }
+                    uint4* dst = reinterpret_cast<uint4*>(base_ptr + static_cast<size_t>(m) * stride + cc);
+                    float f[32];
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) f[e] = __uint_as_float(r[e]);
+                    if (epi.residual != nullptr) {
+                        const uint4* res = reinterpret_cast<const uint4*>(epi.residual + static_cast<size_t>(m) * N + col);
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const uint4 rv = res[u];
+                            const uint32_t w4[4] = {rv.x, rv.y, rv.z, rv.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                f[8 * u + 2 * e] += __uint_as_float(w4[e] << 16);
+                                f[8 * u + 2 * e + 1] += __uint_as_float(w4[e] & 0xFFFF0000u);
+                            }
+                        }
+                    }
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
-                        dst[u] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])),
-                                            pack_bf16x2(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])),
-                                            pack_bf16x2(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])),
-                                            pack_bf16x2(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])));
+                        dst[u] = make_uint4(pack_bf16x2(f[8 * u + 0], f[8 * u + 1]), pack_bf16x2(f[8 * u + 2], f[8 * u + 3]),
+                                            pack_bf16x2(f[8 * u + 4], f[8 * u + 5]), pack_bf16x2(f[8 * u + 6], f[8 * u + 7]));
                 }
             }
         }
@@ -264,6 +294,46 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
     }
 }
 
+// RMSNorm rows: one warp per row of K values.  Pass 1: per-lane float sums of squares over
+// 16-byte chunks in order, then a shuffle tree (a fixed order); pass 2 re-reads the row
+// (L1/L2) and writes bf16((x * r) * gamma).
+__global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const uint16_t* __restrict__ x,
+                                                           const uint16_t* __restrict__ gamma, float eps, int T, int K,
+                                                           uint16_t* __restrict__ xn) {
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (row >= T) return;
+    const uint4* xr = reinterpret_cast<const uint4*>(x + static_cast<size_t>(row) * K);
+    const int nchunk = K / 8;
+    float ss = 0.f;
+    for (int i = lane; i < nchunk; i += 32) {
+        const uint4 v = xr[i];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float a = __uint_as_float(w[e] << 16), b = __uint_as_float(w[e] & 0xFFFF0000u);
+            ss = fmaf(a, a, ss);
+            ss = fmaf(b, b, ss);
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xFFFFFFFFu, ss, off);
+    const float r = 1.0f / sqrtf(ss / static_cast<float>(K) + eps);
+    const uint4* gr = reinterpret_cast<const uint4*>(gamma);
+    uint4* out = reinterpret_cast<uint4*>(xn + static_cast<size_t>(row) * K);
+    for (int i = lane; i < nchunk; i += 32) {
+        const uint4 v = xr[i], g = gr[i];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w}, gw[4] = {g.x, g.y, g.z, g.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float lo = (__uint_as_float(w[e] << 16) * r) * __uint_as_float(gw[e] << 16);
+            const float hi = (__uint_as_float(w[e] & 0xFFFF0000u) * r) * __uint_as_float(gw[e] & 0xFFFF0000u);
+            o[e] = pack_bf16x2(lo, hi);
+        }
+        out[i] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
 std::mutex g_mutex;
 PFN_encodeTiled g_encode = nullptr;
 constexpr int kMaxDevices = 64;
@@ -271,8 +341,14 @@ bool g_configured[kMaxDevices] = {};
 
 }  // namespace
 
+cudaError_t launch_rmsnorm_rows(const uint16_t* x, const uint16_t* gamma, float eps, int T, int K, uint16_t* xn,
+                                cudaStream_t st) {
+    rmsnorm_rows_kernel<<<(T + 7) / 8, 256, 0, st>>>(x, gamma, eps, T, K, xn);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N, int K, uint16_t* y, int* err,
-                           cudaStream_t st) {
+                           cudaStream_t st, const W4GemmEpi* epi_in) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -303,7 +379,9 @@ cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N
                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     const dim3 grid(static_cast<unsigned>(N / kBN), static_cast<unsigned>((T + kBM - 1) / kBM));
-    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, tiles, T, N, K, y, err);
+    W4GemmEpi epi = {N, N, nullptr, nullptr, nullptr};
+    if (epi_in != nullptr) epi = *epi_in;
+    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, tiles, T, N, K, y, err, epi);
     return cudaGetLastError();
 }
 
