@@ -782,6 +782,35 @@ def run_sweep(args):
                      "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
         attn.close()
         del layers_, gr
+    # The attention half of a decoder block over a prefill chunk (attn_prefill_layer: RMSNorm
+    # pre-pass -> stacked QKV GEMM split into q, k, v -> RoPE + cache append + causal attention
+    # -> o_proj GEMM + residual), the same 8B-class layer: a 4096-token prefill and a 4096-token
+    # prefill_kv chunk over 4096 history tokens.  FLOP = the two projections (2 T N K each) + the
+    # attention's 4 D per unmasked (query, key) pair per query head.
+    lsh = w.decode_shape(1)
+    hidden = 4096
+    sh = Shape("prefill_layer", 1, lsh.n_q_heads, lsh.n_kv_heads, lsh.head_dim, lsh.max_len, lsh.rope_theta)
+    qd, kd = sh.n_q_heads * sh.head_dim, sh.n_kv_heads * sh.head_dim
+    attn = Attention.for_shape(sh)
+    tq = w4_inputs(1, qd + 2 * kd, hidden)[0]
+    to = w4_inputs(1, hidden, qd)[0]
+    gamma = (1.0 + 0.1 * torch.randn(hidden, device=dev, generator=gen)).to(torch.bfloat16)
+    kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    for hist, S in ((0, 4096), (4096, 4096)):
+        x = torch.randn(1, S, hidden, device=dev, generator=gen).to(torch.bfloat16)
+        ws = torch.empty(attn.prefill_layer_workspace(hidden, S), dtype=torch.uint8, device=dev)
+        out = torch.empty_like(x)
+        ms = time_calls(lambda: attn.prefill_layer(x, gamma, 1e-6, tq, to, hist, kc, vc, out=out, workspace=ws),
+                        max(3, args.sweep_reps // 2))
+        flop = 2.0 * S * (qd + 2 * kd) * hidden + 2.0 * S * hidden * qd + attn_flops(sh, prefill_pairs(hist, S))
+        tf = flop / (ms * 1e-3) / 1e12
+        rows.append({"config": f"W4BF16 attention half of a decoder block, prefill chunk {S} over {hist} "
+                               f"(hidden {hidden}, Hq {sh.n_q_heads}, Hkv {sh.n_kv_heads})",
+                     "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
+        del x, ws, out
+    attn.close()
+    del tq, to, kc, vc
     doc = {"peaks": {"bf16_tflops": tc_peak, "hbm_gbs": hbm, "source": kind}, "rows": rows}
     with open(args.sweep_out, "w") as f:
         json.dump(doc, f, indent=1)

@@ -1,29 +1,37 @@
-// w4_gemm.cu -- W4BF16 weight GEMM for the prefill-side projections (tcgen05).
+// w4_gemm.cu -- W4BF16 weight GEMM for the prefill-side projections (tcgen05), and the
+// RMSNorm pre-pass of the block's chunk.
 //
 // A prefill chunk of T tokens turns the block's projections (Listing 1: q/k/v_proj, o_proj)
 // into GEMMs, Y[T, N] = X[T, K] . W[N, K]^T, with W in the W4BF16 tile stream of
 // attn_w4bf16_gemv (Section 5.1).  Reading: each weight is decoded once into the tensor
 // cores' operand type, W_bf16 = bf16((q - z) * s), and the products accumulate in f32.
 //
-// One CTA computes a 128-token x 128-feature tile of Y, walking K one 128-input group at a
-// time through a kStages ring:
-//   * warp 0, one lane: the x tile of the group by two 2-D TMA loads (128 tokens x 64 inputs,
-//     128-byte swizzle; rows past T read as zeros) and the 8 weight records of the group's
-//     128 features by 8 bulk copies, all completing on the stage's mbarrier;
-//   * warps 2..5: decode the records into the B operand, double-buffered in shared memory
-//     in the same swizzled K-major layout the TMA gives x: per code word one shift and one
-//     lop3 per pair of codes give (128 + q) bf16 pairs, a bf16x2 subtraction of (128 + z)
-//     leaves q - z exactly, a bf16x2 multiply by s rounds each weight once; one 16-byte store
-//     per word;
-//   * warp 1, one lane: 8 tcgen05.mma (kind::f16, 128 x 128 x 16) per group into one TMEM
-//     accumulator, committing the x stage and the B buffer back to their producers;
-//   * warps 2..5 again: the epilogue, 32 TMEM lanes (tokens) each: optionally the residual
-//     added in float, rounded to bf16, the columns optionally split three ways (q, k, v).
-// rmsnorm_rows_kernel is the block's input_layernorm for a chunk: one factor per token,
-// so it runs as a pre-pass over the chunk before the stacked QKV GEMM.
+// Computed transposed, Y^T = W . X^T, so that the decoded weights are the MMA's A operand,
+// which tcgen05 reads from tensor memory: each decode thread owns one feature row (one TMEM
+// lane), decodes its 128 inputs of a group from the record in shared memory and stores the
+// 64 bf16 pairs straight into TMEM -- no shared-memory round trip, no swizzle arithmetic, a
+// row's scale and zero point read once per group.  X^T is the B operand, K-major from
+// shared memory exactly as TMA lays out a 128-token x 64-input box of X.
+//
+// Persistent CTAs walk output tiles of 256 features (two M = 128 halves) x 128 tokens
+// (the MMA's N), token tiles fastest.  448 threads:
+//   warp 0, one lane   producer: per 128-input group one X tile (two 2-D TMA boxes, 128-byte
+//                      swizzle; tokens past T read as zeros) and the 16 weight records of the
+//                      tile's 256 features (bulk copies) into a kStages ring;
+//   warp 1, one lane   tcgen05 issuer: per group and half, 8 MMAs 128 x 128 x 16 from the
+//                      half's A buffer in TMEM and the X stage, into the half's accumulator;
+//   warps 2-9          decode (warps 2-5 the first half's 128 features, 6-9 the second),
+//                      into two A buffers per half (double-buffered across groups);
+//   warps 10-13        epilogue: each thread one feature of each half, 128 tokens from TMEM,
+//                      optionally the residual added in float, rounded to bf16, written
+//                      to y or, split by feature, to y / y1 / y2.  Each half's accumulator is
+//                      handed back as soon as it is read, so the next tile's MMAs of that
+//                      half start while the epilogue finishes the other half.
+// TMEM (512 columns): A buffers (half h, buffer b) at 64 (2h + b), accumulators at 256 + 128 h.
 // Every wait is bounded (ATTN_DEVERR_TIMEOUT in *err, then the CTA drains and exits).
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cstdint>
 #include <mutex>
 
@@ -33,32 +41,35 @@
 namespace attn {
 namespace {
 
-constexpr int kThreads = 192;
-constexpr int kWarpTma = 0, kWarpMma = 1;  // warps 2..5 decode and run the epilogue
-constexpr int kBM = 128, kBN = 128;
-constexpr int kStages = 3;
-constexpr int kChunk = 128 * 128;          // 128 rows x 64 bf16 (128 bytes), swizzled
-constexpr int kXStage = 2 * kChunk;        // x tile: 128 tokens x 128 inputs
-constexpr int kRecBytes = 1072;            // one weight record: 16 rows x 128 inputs
-constexpr int kRecs = kBN / 16;            // records per stage
+constexpr int kThreads = 448;
+constexpr int kWarpTma = 0, kWarpMma = 1, kWarpDec0 = 2, kWarpEpi0 = 10;
+constexpr int kBT = 128;                    // tokens per tile (MMA N)
+constexpr int kBF = 256;                    // features per tile (two MMA M = 128 halves)
+constexpr int kStages = 4;
+constexpr int kChunk = 128 * 128;           // 128 rows x 64 bf16 (128 bytes), swizzled
+constexpr int kXStage = 2 * kChunk;         // X tile: 128 tokens x 128 inputs
+constexpr int kRecBytes = 1072;             // one weight record: 16 rows x 128 inputs
+constexpr int kRecs = kBF / 16;             // records per stage
 constexpr int kWStage = kRecs * kRecBytes;
-constexpr int kBTile = 2 * kChunk;         // decoded weights: 128 features x 128 inputs
-constexpr uint32_t kTmemCols = 128;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTmA = 0, kTmAcc = 256;
 constexpr uint64_t kWaitNs = 1000000000ull;
 
 struct L {
     static constexpr int OFF_X = 0;
     static constexpr int OFF_W = OFF_X + kStages * kXStage;
-    static constexpr int OFF_B = ((OFF_W + kStages * kWStage + 1023) / 1024) * 1024;
-    static constexpr int OFF_BAR = OFF_B + 2 * kBTile;
-    static constexpr int NBAR = 2 * kStages + 4 + 1;  // FULL, EMPTY, BFULL x2, BEMPTY x2, ACC
+    static constexpr int OFF_BAR = OFF_W + kStages * kWStage;
+    static constexpr int NBAR = 2 * kStages + 2 + 2 + 1 + 2 + 1;
     static constexpr int OFF_TMEM = OFF_BAR + 8 * NBAR;
     static constexpr int OFF_ABORT = OFF_TMEM + 16;
     static constexpr int BYTES = OFF_ABORT + 16;
     static constexpr int ALLOC = BYTES + 1024;  // the dynamic base is aligned up to 1024 in the kernel
 };
 static_assert(L::ALLOC <= 232448, "shared memory");
-enum Bar { B_FULL0 = 0, B_EMPTY0 = kStages, B_BFULL0 = 2 * kStages, B_BEMPTY0 = 2 * kStages + 2, B_ACC = 2 * kStages + 4 };
+enum Bar {
+    B_FULL0 = 0, B_EMPTY0 = kStages, B_AFULL0 = 2 * kStages, B_AEMPTY0 = B_AFULL0 + 2, B_ACCFULL = B_AEMPTY0 + 2,
+    B_ACCEMPTY0 = B_ACCFULL + 1, B_DRAIN = B_ACCEMPTY0 + 2
+};
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int c0, int c1, uint32_t bar) {
     asm volatile(
@@ -66,12 +77,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
         : "memory");
-}
-
-__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
 }
 
 __device__ __forceinline__ uint32_t bf16x2_sub(uint32_t a, uint32_t b) {
@@ -103,21 +108,23 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
     volatile int* abort_flag = reinterpret_cast<volatile int*>(gb + L::OFF_ABORT);
     auto bar = [&](int i) -> uint32_t { return base + L::OFF_BAR + 8u * static_cast<uint32_t>(i); };
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int n0 = blockIdx.x * kBN, m0 = blockIdx.y * kBM;
     const int ngroup = K / 128;
-    const int nrec = min(kRecs, (N - n0 + 15) / 16);  // records of this feature tile
+    const int n_tt = (T + kBT - 1) / kBT, n_ft = (N + kBF - 1) / kBF;
+    const int n_tiles = n_tt * n_ft;
 
     if (tid == 0) {
         *abort_flag = 0;
         for (int s = 0; s < kStages; ++s) {
             mbar_init(bar(B_FULL0 + s), 1);
-            mbar_init(bar(B_EMPTY0 + s), 1 + 4);  // the MMA commit and the four decode warps
+            mbar_init(bar(B_EMPTY0 + s), 1 + 8);  // the MMA commit and the eight decode warps
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(bar(B_BFULL0 + b), 4);
-            mbar_init(bar(B_BEMPTY0 + b), 1);
+            mbar_init(bar(B_AFULL0 + b), 8);
+            mbar_init(bar(B_AEMPTY0 + b), 1);
+            mbar_init(bar(B_ACCEMPTY0 + b), 4);  // per half: the four epilogue warps
         }
-        mbar_init(bar(B_ACC), 1);
+        mbar_init(bar(B_ACCFULL), 1);
+        mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
         tma_prefetch_desc(&map_x);
     }
@@ -132,158 +139,225 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
 
     if (warp == kWarpTma) {
         if (lane == 0) {
-            int issued = 0;
+            uint32_t gs = 0;  // groups issued
             bool ok = true;
-            for (int G = 0; G < ngroup; ++G) {
-                const int s = G % kStages;
-                if (G >= kStages &&
-                    !mbar_wait(bar(B_EMPTY0 + s), static_cast<uint32_t>(G / kStages - 1) & 1u, abort_flag, kWaitNs)) {
-                    ok = false;
-                    break;
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const int ft = tile / n_tt, tt = tile - ft * n_tt;
+                const int f0 = ft * kBF, t0 = tt * kBT;
+                const int nrec = min(kRecs, (N - f0) / 16);
+                for (int G = 0; G < ngroup; ++G, ++gs) {
+                    const int s = static_cast<int>(gs % kStages);
+                    if (gs >= kStages &&
+                        !mbar_wait(bar(B_EMPTY0 + s), (gs / kStages - 1u) & 1u, abort_flag, kWaitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(bar(B_FULL0 + s), kXStage + nrec * kRecBytes);
+                    for (int c = 0; c < 2; ++c)
+                        tma_load_2d(base + L::OFF_X + s * kXStage + c * kChunk, &map_x, G * 128 + c * 64, t0,
+                                    bar(B_FULL0 + s));
+                    for (int r = 0; r < nrec; ++r) {
+                        const size_t rec = static_cast<size_t>(f0 / 16 + r) * ngroup + G;
+                        bulk_g2s(base + L::OFF_W + s * kWStage + r * kRecBytes, tiles + rec * kRecBytes, kRecBytes,
+                                 bar(B_FULL0 + s));
+                    }
                 }
-                mbar_arrive_expect_tx(bar(B_FULL0 + s), kXStage + nrec * kRecBytes);
-                for (int c = 0; c < 2; ++c)
-                    tma_load_2d(base + L::OFF_X + s * kXStage + c * kChunk, &map_x, G * 128 + c * 64, m0,
-                                bar(B_FULL0 + s));
-                for (int r = 0; r < nrec; ++r) {
-                    const size_t rec = static_cast<size_t>(n0 / 16 + r) * ngroup + G;
-                    bulk_load(base + L::OFF_W + s * kWStage + r * kRecBytes, tiles + rec * kRecBytes, kRecBytes,
-                              bar(B_FULL0 + s));
-                }
-                issued = G + 1;
             }
             if (!ok) {
                 *abort_flag = 1;
                 atomicOr(err, kDevErrTimeout);
             }
             // every copy issued must land before the CTA may exit
-            for (int G = issued > kStages ? issued - kStages : 0; G < issued; ++G)
-                mbar_wait(bar(B_FULL0 + G % kStages), static_cast<uint32_t>(G / kStages) & 1u, nullptr, kWaitNs);
+            for (uint32_t g = gs > kStages ? gs - kStages : 0; g < gs; ++g)
+                mbar_wait(bar(B_FULL0 + g % kStages), (g / kStages) & 1u, nullptr, kWaitNs);
         }
     } else if (warp == kWarpMma) {
         if (lane == 0) {
-            constexpr uint32_t kId = idesc_bf16_f32(kBM, kBN, false, false);
+            constexpr uint32_t kId = idesc_bf16_f32(128, kBT, false, false);
             constexpr uint32_t kHi = desc_hi_sw128(1024);
             const uint32_t x_lo0 = desc_lo_sw128(base + L::OFF_X, 16);
-            const uint32_t b_lo0 = desc_lo_sw128(base + L::OFF_B, 16);
+            uint32_t gs = 0;
+            int tiles_done = 0;
             bool ok = true;
-            for (int G = 0; G < ngroup; ++G) {
-                const int s = G % kStages, b = G & 1;
-                if (!mbar_wait(bar(B_FULL0 + s), static_cast<uint32_t>(G / kStages) & 1u, abort_flag, kWaitNs) ||
-                    !mbar_wait(bar(B_BFULL0 + b), static_cast<uint32_t>(G >> 1) & 1u, abort_flag, kWaitNs)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t xa = x_lo0 + ((s * kXStage) >> 4), bb = b_lo0 + ((b * kBTile) >> 4);
+            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tiles_done) {
+                const int ft = tile / n_tt;
+                const bool half1 = ft * kBF + 128 < N;
+                for (int G = 0; G < ngroup; ++G, ++gs) {
+                    const int s = static_cast<int>(gs % kStages), b = static_cast<int>(gs & 1u);
+                    if (!mbar_wait(bar(B_FULL0 + s), (gs / kStages) & 1u, abort_flag, kWaitNs) ||
+                        !mbar_wait(bar(B_AFULL0 + b), (gs >> 1) & 1u, abort_flag, kWaitNs)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t xa = x_lo0 + ((s * kXStage) >> 4);
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint32_t c = ((kk >> 2) * kChunk + (kk & 3) * 32) >> 4;
-                    umma_ss_w(tmem, xa + c, kHi, bb + c, kHi, kId, (G > 0 || kk > 0) ? 1u : 0u);
+                    for (int h = 0; h < 2; ++h) {
+                        if (h == 1 && !half1) break;
+                        // the accumulator of half h is free once the epilogue read the previous tile's
+                        if (G == 0 && tiles_done > 0 &&
+                            !mbar_wait(bar(B_ACCEMPTY0 + h), static_cast<uint32_t>(tiles_done - 1) & 1u, abort_flag,
+                                       kWaitNs)) {
+                            ok = false;
+                            break;
+                        }
+                        if (G == 0) tc_fence_after();
+                        const uint32_t a_col = tmem + kTmA + 64u * (2 * h + b), d_col = tmem + kTmAcc + 128u * h;
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t c = ((kk >> 2) * kChunk + (kk & 3) * 32) >> 4;
+                            umma_ts_w(d_col, a_col + 8u * kk, xa + c, kHi, kId, (G > 0 || kk > 0) ? 1u : 0u);
+                        }
+                    }
+                    if (!ok) break;
+                    umma_commit(bar(B_EMPTY0 + s));
+                    umma_commit(bar(B_AEMPTY0 + b));
                 }
-                umma_commit(bar(B_EMPTY0 + s));
-                umma_commit(bar(B_BEMPTY0 + b));
+                if (!ok) break;
+                umma_commit(bar(B_ACCFULL));  // the tile's products are complete
             }
             if (!ok) {
                 *abort_flag = 1;
                 atomicOr(err, kDevErrTimeout);
             }
-            umma_commit(bar(B_ACC));  // also after an abort: the MMAs issued so far complete on it
-            mbar_wait(bar(B_ACC), 0u, nullptr, kWaitNs);
+            umma_commit(bar(B_DRAIN));  // also after an abort: the MMAs issued so far complete on it
+            mbar_wait(bar(B_DRAIN), 0u, nullptr, kWaitNs);
         }
-    } else {
-        // ------------------------------------------------ decode warps, then the epilogue
-        const int dt = tid - 64;  // 0..127
+    } else if (warp < kWarpEpi0) {
+        // ------------------------------------------------ decode: one feature row per thread
+        const int h = (warp - kWarpDec0) >> 2;        // half of the tile
+        const int q = warp & 3;                       // TMEM lane quadrant of this warp
+        const int fl = q * 32 + lane;                 // feature within the half (= TMEM lane)
+        const int rrow = 128 * h + fl;                // feature within the tile
         const uint32_t magic = 0x43004300u, mask = 0x000F000Fu;
+        uint32_t gs = 0;
         bool ok = true;
-        for (int G = 0; G < ngroup && ok; ++G) {
-            const int s = G % kStages, b = G & 1;
-            ok = mbar_wait(bar(B_FULL0 + s), static_cast<uint32_t>(G / kStages) & 1u, abort_flag, kWaitNs);
-            if (ok && G >= 2)
-                ok = mbar_wait(bar(B_BEMPTY0 + b), static_cast<uint32_t>((G >> 1) - 1) & 1u, abort_flag, kWaitNs);
-            ok = __all_sync(0xFFFFFFFFu, ok);
-            if (!ok) break;
-            const uint8_t* ws = gb + L::OFF_W + s * kWStage;
-            uint8_t* bt = gb + L::OFF_B + b * kBTile;
-#pragma unroll 4
-            for (int j = 0; j < 16; ++j) {
-                const int wi = dt + 128 * j;
-                const int n = wi >> 4, i16 = wi & 15;  // feature row, word of the group
-                const int r = n >> 4, rr = n & 15;
-                uint4 v = make_uint4(0u, 0u, 0u, 0u);
-                if (r < nrec) {
-                    const uint8_t* rec = ws + r * kRecBytes;
-                    const uint32_t w = *reinterpret_cast<const uint32_t*>(rec + rr * 64 + i16 * 4);
-                    const uint32_t sc = *reinterpret_cast<const uint16_t*>(rec + 1024 + rr * 2);
-                    const uint32_t z = rec[1056 + rr];
-                    const uint32_t zp = (0x4300u + z) * 0x00010001u;  // (128 + z) in both halves
-                    const uint32_t sp = sc * 0x00010001u;
-                    v.x = bf16x2_mul(bf16x2_sub(code_pair(w, 0, mask, magic), zp), sp);
-                    v.y = bf16x2_mul(bf16x2_sub(code_pair(w, 1, mask, magic), zp), sp);
-                    v.z = bf16x2_mul(bf16x2_sub(code_pair(w, 2, mask, magic), zp), sp);
-                    v.w = bf16x2_mul(bf16x2_sub(code_pair(w, 3, mask, magic), zp), sp);
+        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const int ft = tile / n_tt;
+            const int f0 = ft * kBF;
+            const bool have = f0 + rrow < N;   // this feature exists (N is a multiple of 16)
+            const bool half_on = f0 + 128 * h < N;
+            for (int G = 0; G < ngroup; ++G, ++gs) {
+                const int s = static_cast<int>(gs % kStages), b = static_cast<int>(gs & 1u);
+                bool w_ok = mbar_wait(bar(B_FULL0 + s), (gs / kStages) & 1u, abort_flag, kWaitNs);
+                if (w_ok && gs >= 2)
+                    w_ok = mbar_wait(bar(B_AEMPTY0 + b), ((gs >> 1) - 1u) & 1u, abort_flag, kWaitNs);
+                ok = __all_sync(0xFFFFFFFFu, w_ok);
+                if (!ok) break;
+                if (half_on) {
+                    uint32_t wv[16];
+                    uint32_t zp = 0x43004300u, sp = 0u;
+                    if (have) {
+                        const uint8_t* rec = gb + L::OFF_W + s * kWStage + (rrow >> 4) * kRecBytes;
+                        const uint4* row = reinterpret_cast<const uint4*>(rec + (rrow & 15) * 64);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const uint4 u = row[i];
+                            wv[4 * i] = u.x;
+                            wv[4 * i + 1] = u.y;
+                            wv[4 * i + 2] = u.z;
+                            wv[4 * i + 3] = u.w;
+                        }
+                        const uint32_t sc = *reinterpret_cast<const uint16_t*>(rec + 1024 + (rrow & 15) * 2);
+                        const uint32_t z = rec[1056 + (rrow & 15)];
+                        zp = (0x4300u + z) * 0x00010001u;  // (128 + z) in both halves
+                        sp = sc * 0x00010001u;
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) wv[i] = 0u;
+                    }
+                    // word i: inputs 8 i .. 8 i + 7; pair p: inputs 8 i + 2 p, + 1 -> TMEM column 4 i + p
+                    const uint32_t a_col = tmem + (static_cast<uint32_t>(q * 32) << 16) + kTmA + 64u * (2 * h + b);
+#pragma unroll
+                    for (int half = 0; half < 2; ++half) {
+                        uint32_t o[32];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i)
+#pragma unroll
+                            for (int p = 0; p < 4; ++p)
+                                o[4 * i + p] = bf16x2_mul(bf16x2_sub(code_pair(wv[8 * half + i], p, mask, magic), zp), sp);
+                        tmem_st32(a_col + 32u * half, o);
+                    }
+                    tmem_wait_st();
                 }
-                // inputs 8 i16 .. 8 i16 + 7 of row n: chunk i16 / 8, 16-byte unit (i16 % 8) ^ (n % 8)
-                *reinterpret_cast<uint4*>(bt + (i16 >> 3) * kChunk + n * 128 + (((i16 & 7) ^ (n & 7)) << 4)) = v;
-            }
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(bar(B_BFULL0 + b));
-                mbar_arrive(bar(B_EMPTY0 + s));
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(bar(B_AFULL0 + b));
+                    mbar_arrive(bar(B_EMPTY0 + s));
+                }
             }
         }
         if (!ok && lane == 0) {
             *abort_flag = 1;
             atomicOr(err, kDevErrTimeout);
         }
-        // epilogue: this warp reads TMEM lanes 32 (warp % 4) .. + 31 (tokens)
-        const bool acc_ok = __all_sync(0xFFFFFFFFu, mbar_wait(bar(B_ACC), 0u, abort_flag, kWaitNs));
-        if (ok && acc_ok) {
+    } else {
+        // ------------------------------------------------ epilogue: one feature of each half per thread
+        const int q = warp & 3;
+        const int fl = q * 32 + lane;
+        int tiles_done = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tiles_done) {
+            const int ft = tile / n_tt, tt = tile - ft * n_tt;
+            const int f0 = ft * kBF, t0 = tt * kBT;
+            ok = __all_sync(0xFFFFFFFFu,
+                            mbar_wait(bar(B_ACCFULL), static_cast<uint32_t>(tiles_done) & 1u, abort_flag, kWaitNs));
+            if (!ok) break;
             tc_fence_after();
-            const int q = warp & 3;
-            const int m = m0 + q * 32 + lane;
-            for (int c = 0; c < kBN / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld32(tmem + (static_cast<uint32_t>(q * 32) << 16) + 32u * c, r);
-                tmem_wait_ld();
-                const int col = n0 + 32 * c;
-                if (m < T && col < N) {
-                    // destination of these 32 columns: y, or a part of the split output
-                    uint16_t* base_ptr = y;
-                    int stride = epi.n0, cc = col;
-                    if (col >= epi.n1) {
-                        base_ptr = epi.y2;
+#pragma unroll 1
+            for (int h = 0; h < 2; ++h) {
+                const int n = f0 + 128 * h + fl;
+                if (f0 + 128 * h < N) {
+                    // destination of feature n: y, or a part of the split output
+                    uint16_t* dst = y;
+                    int stride = epi.n0, cc = n;
+                    if (n >= epi.n1) {
+                        dst = epi.y2;
                         stride = N - epi.n1;
-                        cc = col - epi.n1;
-                    } else if (col >= epi.n0) {
-                        base_ptr = epi.y1;
+                        cc = n - epi.n1;
+                    } else if (n >= epi.n0) {
+                        dst = epi.y1;
                         stride = epi.n1 - epi.n0;
-                        cc = col - epi.n0;
+                        cc = n - epi.n0;
                     }
-                    uint4* dst = reinterpret_cast<uint4*>(base_ptr + static_cast<size_t>(m) * stride + cc);
-                    float f[32];
+                    const uint32_t d_col = tmem + (static_cast<uint32_t>(q * 32) << 16) + kTmAcc + 128u * h;
+#pragma unroll 1
+                    for (int c = 0; c < kBT / 32; ++c) {
+                        uint32_t r[32];
+                        tmem_ld32(d_col + 32u * c, r);
+                        tmem_wait_ld();
+                        if (c == kBT / 32 - 1) {
+                            // this half's accumulator is read: the next tile's MMAs may overwrite it
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(bar(B_ACCEMPTY0 + h));
+                        }
+                        const int tb = t0 + 32 * c;
+                        if (n < N) {
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) f[e] = __uint_as_float(r[e]);
-                    if (epi.residual != nullptr) {
-                        const uint4* res = reinterpret_cast<const uint4*>(epi.residual + static_cast<size_t>(m) * N + col);
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const uint4 rv = res[u];
-                            const uint32_t w4[4] = {rv.x, rv.y, rv.z, rv.w};
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                f[8 * u + 2 * e] += __uint_as_float(w4[e] << 16);
-                                f[8 * u + 2 * e + 1] += __uint_as_float(w4[e] & 0xFFFF0000u);
+                            for (int e = 0; e < 32; ++e) {
+                                const int t = tb + e;
+                                if (t < T) {
+                                    float v = __uint_as_float(r[e]);
+                                    if (epi.residual != nullptr)
+                                        v += __uint_as_float(static_cast<uint32_t>(
+                                                                 epi.residual[static_cast<size_t>(t) * N + n])
+                                                             << 16);
+                                    dst[static_cast<size_t>(t) * stride + cc] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+                                }
                             }
                         }
                     }
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        dst[u] = make_uint4(pack_bf16x2(f[8 * u + 0], f[8 * u + 1]), pack_bf16x2(f[8 * u + 2], f[8 * u + 3]),
-                                            pack_bf16x2(f[8 * u + 4], f[8 * u + 5]), pack_bf16x2(f[8 * u + 6], f[8 * u + 7]));
+                } else {
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(B_ACCEMPTY0 + h));  // an absent half is free at once
                 }
             }
+        }
+        if (!ok && lane == 0) {
+            *abort_flag = 1;
+            atomicOr(err, kDevErrTimeout);
         }
     }
     tc_fence_before();
@@ -372,13 +446,17 @@ cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N
     CUtensorMap map;
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
-    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBM)};
+    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBT)};
     const cuuint32_t estr[2] = {1, 1};
     const CUresult r = g_encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(x), dims, strides, box,
                                 estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    const dim3 grid(static_cast<unsigned>(N / kBN), static_cast<unsigned>((T + kBM - 1) / kBM));
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const long long n_tiles = static_cast<long long>((T + kBT - 1) / kBT) * ((N + kBF - 1) / kBF);
+    const unsigned grid = static_cast<unsigned>(std::min<long long>(n_tiles, sms));
     W4GemmEpi epi = {N, N, nullptr, nullptr, nullptr};
     if (epi_in != nullptr) epi = *epi_in;
     w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, tiles, T, N, K, y, err, epi);
