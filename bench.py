@@ -660,7 +660,8 @@ def run_sweep(args):
     # Multi-token decode (a speculative draft of n tokens verified in one call) against the
     # same n tokens as one prefill_kv chunk: bytes = the history's K/V read once plus the
     # new tokens' q, k, v and out.
-    for sh, hist, n in ((w.decode_shape(1), 8188, 4), (S, w.LONG_DECODE_HIST - 2, 3)):
+    for sh, hist, n in ((w.decode_shape(1), 8188, 4), (S, w.LONG_DECODE_HIST - 2, 3), (w.decode_shape(1), 8184, 8),
+                        (S, w.LONG_DECODE_HIST - 7, 8)):
         attn = Attention.for_shape(sh)
         kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
         vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)

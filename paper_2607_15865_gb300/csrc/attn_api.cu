@@ -61,6 +61,11 @@ namespace {
 
 thread_local char g_cuda_msg[256] = "no error";
 
+// New tokens per sequence of one multi-token decode call, and the column groups of 16
+// (query head, token) columns that many take at the largest group size (16 heads).
+constexpr int kMaxDraftTokens = 16;
+constexpr int kMaxColumnGroups = 16;
+
 // Per device: whether it is an sm_103 part (attn_w4bf16_gemv checks once per device).
 constexpr int kArchCacheDevices = 64;
 std::atomic<int> g_arch_ok[kArchCacheDevices];
@@ -251,7 +256,8 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     oom |= cudaMalloc(&c->d_lk, kd * sizeof(uint16_t)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_lv, kd * sizeof(uint16_t)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_lo, qd * sizeof(uint16_t)) != cudaSuccess;
-    const size_t n_counters = 2 * static_cast<size_t>(cfg->batch) * cfg->n_kv_heads;  // merge + tile claims
+    // merge counts and tile claims per (sequence, kv head, column group of the multi-token decode)
+    const size_t n_counters = 2 * static_cast<size_t>(cfg->batch) * cfg->n_kv_heads * kMaxColumnGroups;
     oom |= cudaMalloc(&c->d_counters, n_counters * sizeof(int)) != cudaSuccess;
     if (oom) {
         cudaGetLastError();
@@ -337,9 +343,10 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         c->dec_k = k_cache;
         c->dec_v = v_cache;
     }
-    if (ntok < 1 || (ntok > 1 && (!tc || (c->cfg.n_q_heads / c->cfg.n_kv_heads) * ntok > 16))) return ATTN_EINVAL;
+    if (ntok < 1 || ntok > kMaxDraftTokens || (ntok > 1 && !tc)) return ATTN_EINVAL;
     // the partials hold batch * Hq * nsplit_max rows: ntok tokens share them
-    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms), c->nsplit_max / ntok)
+    const int ncg = attn::decode_tc_column_groups(c->cfg.n_q_heads / c->cfg.n_kv_heads, ntok);
+    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms, ncg), c->nsplit_max / ntok)
                           : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         if (tc)

@@ -193,7 +193,10 @@ __device__ __forceinline__ bool halving_leader(int lane) {
 }
 
 // NHP: columns the softmax processes (8 when G * ntok <= 8, else 16); the MMA always
-// runs N = 16 with the rows of Q^T past C = G * ntok zero.
+// runs N = 16 with the rows of Q^T past the CTA's C columns zero.  With more than 16
+// columns (G * ntok > 16) the grid's z dimension is (sequence, column group): every column
+// group streams the same key tiles, which its sibling CTAs read at about the same time, so
+// the repeats come from L2.
 template <int NHP, int MAXTOK>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
@@ -202,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
     int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
-    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns) {
+    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -214,10 +217,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     auto bar = [&](int i) -> uint32_t { return base + L::OFF_BAR + 8u * static_cast<uint32_t>(i); };
 
     const int G = Hq / Hkv;
-    const int C = G * ntok;  // columns of Q^T: column c = token c / G, head h0 + c % G
+    // Columns: global column c = token c / G, head h0 + c % G, of G * ntok; this CTA takes the
+    // 16-column group cg, columns c0 .. c0 + C - 1 (its local column h is global column c0 + h).
     const int s = blockIdx.x;
     const int g = blockIdx.y;
-    const int b = blockIdx.z;
+    const int b = static_cast<int>(blockIdx.z) / ncg;
+    const int cg = static_cast<int>(blockIdx.z) - b * ncg;
+    const int c0 = cg * NH;
+    const int C = min(NH, G * ntok - c0);
     const int h0 = g * G;
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
@@ -232,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     }
 
     if (tid < NH) {
-        const int c = min(tid, G * ntok - 1);
+        const int c = c0 + min(tid, C - 1);
         const size_t r = (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G;
         reinterpret_cast<size_t*>(gb + L::OFF_OROW)[tid] = r;
         reinterpret_cast<size_t*>(gb + L::OFF_CROW)[tid] = r * nsplit;
@@ -280,10 +287,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     }
 
     const bool hist_ok = hist >= 0 && hist <= max_len - ntok;
-    if (!hist_ok && s == 0 && g == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
+    if (!hist_ok && s == 0 && g == 0 && cg == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
     const int nkeys = hist + ntok;        // slots [0, hist) and the new tokens' [hist, hist + ntok)
     const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds the last new slot
     const int kv_row = b * Hkv + g;
+    const int ctr_row = kv_row * ncg + cg;  // counters of this (sequence, kv head, column group)
     // Rows of column c (token c / G, head h0 + c % G), tabulated once in the prologue:
     // q / out row (b * ntok + c / G) * Hq + h0 + c % G, and partial row of split 0 that
     // times nsplit (split sp adds sp).  Columns past C repeat column C - 1.
@@ -301,7 +309,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         // while the current tile's copies are issued.  One thread feeds both rings: the
         // V slot of tile j frees (PV(j-4) done) before the K slot does (S(j-2) done).
         if (lane == 0) {
-            int* tile_ctr = counters + gridDim.y * gridDim.z + kv_row;
+            int* tile_ctr = counters + gridDim.y * gridDim.z + ctr_row;
             int cur = s < T ? s : T;
             int nxt = (nsplit > 1 && cur < T) ? nsplit + atomicAdd(tile_ctr, 1) : cur + 1;
             int issued_k = 0, issued_v = 0;
@@ -503,7 +511,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 const uint16_t* qrow = q + orow[cc] * D;
                 qx[c] = bf16_at(qrow + t);
                 qy[c] = bf16_at(qrow + tp);
-                const size_t pos = static_cast<size_t>(hist + cc / G);
+                const size_t pos = static_cast<size_t>(hist + (c0 + cc) / G);
                 c_t[c] = cos_tab[pos * HALF + t % HALF];
                 s_t[c] = sin_tab[pos * HALF + t % HALF];
             }
@@ -547,9 +555,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             uint32_t r[NHP];
             tmem_ld_cols<NHP>(tmem + lane_base + (j & 1) * NH, r);
             tmem_wait_ld();
-            // key tile * KT + t is visible to column c (token c / G) iff it is <= hist + c / G,
+            // key tile * KT + t is visible to global column c (token c / G) iff it is <= hist + c / G,
             // i.e. iff c >= (key - hist) * G (always for a history key: key - hist < 0)
-            const int kg = (tile * KT + t - hist) * G;
+            const int kg = (tile * KT + t - hist) * G - c0;
             float sc[NHP];
             bool exceed = false;
 #pragma unroll
@@ -657,11 +665,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         tc_fence_before();
         __syncthreads();
         if (tid == 0) {
-            int* cnt = counters + kv_row;
+            int* cnt = counters + ctr_row;
             const int last = atomicAdd(cnt, 1) == nsplit - 1;
             if (last) {  // every split of this launch has been counted and has claimed its last tile
                 *cnt = 0;
-                counters[gridDim.y * gridDim.z + kv_row] = 0;
+                counters[gridDim.y * gridDim.z + ctr_row] = 0;
             }
             *last_flag = last;
         }
@@ -772,8 +780,10 @@ cudaError_t configure_decode_tc() {
 
 // One wave of CTAs, one per SM: with fewer (sequence, kv head) items than SMs, each
 // item gets floor(SMs / items) splits; otherwise one split per item.
-int decode_tc_num_splits(const Shape& s, int num_sms) {
-    const long items = static_cast<long>(s.batch) * s.n_kv_heads;
+int decode_tc_column_groups(int G, int ntok) { return (G * ntok + NH - 1) / NH; }
+
+int decode_tc_num_splits(const Shape& s, int num_sms, int ncg) {
+    const long items = static_cast<long>(s.batch) * s.n_kv_heads * ncg;
     const long max_tiles = std::max(1L, static_cast<long>((s.max_len + KT - 1) / KT));
     long ns = items >= num_sms ? 1 : num_sms / items;
     ns = std::min(ns, std::min(max_tiles, 256L));
@@ -803,8 +813,10 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
                              int ntok, cudaStream_t st, bool producer_early, uint64_t wait_ns) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
-    const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch));
     const int G = s.n_q_heads / s.n_kv_heads;
+    const int ncg = decode_tc_column_groups(G, ntok);
+    const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads),
+                    static_cast<unsigned>(s.batch * ncg));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(kThreads);
@@ -816,13 +828,13 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     cfg.attrs = attr;
     // dependent launch only right after another decode step, or with producer_early
     cfg.numAttrs = (after_decode || producer_early) ? 1 : 0;
-    if (ntok < 1 || ntok > kMaxTok || G * ntok > NH) return cudaErrorInvalidValue;
+    if (ntok < 1 || ntok > kMaxTok || G > NH) return cudaErrorInvalidValue;
     const auto kernel = ntok == 1 ? (G <= 8 ? decode_tc_kernel<8, 1> : decode_tc_kernel<16, 1>)
                                   : (G * ntok <= 8 ? decode_tc_kernel<8, kMaxTok> : decode_tc_kernel<16, kMaxTok>);
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
-                              producer_early ? 1 : 0, wait_ns);
+                              producer_early ? 1 : 0, wait_ns, ncg);
 }
 
 }  // namespace attn

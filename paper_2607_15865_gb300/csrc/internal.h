@@ -100,10 +100,10 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
 // 128-key boxes; same partial layout as launch_decode_split, but the merge is fused
 // in (the last CTA of each (b, kv head) merges and writes `out`), so no K4 follows.
 // Splits claim key tiles from a per-(b, kv head) counter.  `counters`: 2*B*Hkv ints
-// (merge counts, then tile claims), zero before the first launch; every launch leaves
-// them zero.  ntok >= 1 new tokens per sequence (q/k/v/out [B, ntok, H, D]) at positions
-// d_hist[b] + hist_add + i, token i attending causally to slots [0, that position];
-// (Hq / Hkv) * ntok <= 16, and the partials need B * ntok * Hq * nsplit rows.
+// (merge counts, then tile claims) per column group, zero before the first launch; every
+// launch leaves them zero.  1 <= ntok <= 16 new tokens per sequence (q/k/v/out
+// [B, ntok, H, D]) at positions d_hist[b] + hist_add + i, token i attending causally to
+// slots [0, that position]; the partials need B * ntok * Hq * nsplit rows.
 // after_decode: the stream's previous kernel is a decode_tc launch (the
 // previous step of a decode loop); this one then starts as a dependent launch whose
 // setup overlaps that step's tail.  Never set it after any other kernel: the inputs
@@ -111,7 +111,10 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
 // producer_early: a dependent launch after a kernel that writes q / the new k, v (and
 // neither the caches, the lengths nor the counters); the K/V stream starts before the wait.
 cudaError_t configure_decode_tc();
-int decode_tc_num_splits(const Shape& s, int num_sms);
+// Column groups of 16 (query head, new token) columns one launch runs for ntok new tokens
+// per sequence: ceil(G * ntok / 16); the counters need 2 * B * Hkv * that many ints.
+int decode_tc_column_groups(int G, int ntok);
+int decode_tc_num_splits(const Shape& s, int num_sms, int ncg = 1);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                                 const uint16_t* v_cache, DecodeMaps* maps);
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,

@@ -3,7 +3,8 @@ per-sequence lengths on the device, token i attending causally to slots [0, hist
 
 Compared with the oracle of the same stage (for each sequence, prefill_kv of its n
 tokens over its own history; pinned in tests/test_oracle_driver.py to n single-token
-decode steps), on group sizes and token counts that fill 8 or 16 MMA columns, new
+decode steps), on group sizes and token counts that fill 8 or 16 MMA columns or several
+groups of 16 columns (up to 16 heads x 16 tokens, and a ragged last group), new
 tokens that straddle a key tile, an empty history, the long-context shape, lengths
 that run past max_len, and the argument checks.
 """
@@ -33,6 +34,11 @@ CASES = [
     ("g2_two_tokens_empty_history", Shape("mt3", 2, 4, 2, 128, 256, 1.0e4), [0, 5], 2),
     ("g1_sixteen_tokens", Shape("mt4", 1, 2, 2, 128, 600, 1.0e4), [300], 16),
     ("g8_two_tokens_batch3", Shape("mt5", 3, 16, 2, 128, 512, 1.0e4), [7, 130, 400], 2),
+    # more than 16 (query head, token) columns: groups of 16 columns on sibling CTAs
+    ("g4_eight_tokens_2_groups", Shape("mt6", 2, 32, 8, 128, 2048, 5.0e5), [100, 1500], 8),
+    ("g8_eight_tokens_4_groups", Shape("mt7", 2, 64, 8, 128, 1024, 1.0e6), [200, 900], 8),
+    ("g16_sixteen_tokens_16_groups", Shape("mt8", 1, 16, 1, 128, 512, 1.0e4), [250], 16),
+    ("g5_seven_tokens_ragged_group", Shape("mt9", 1, 40, 8, 128, 4096, 1.0e6), [4080], 7),
 ]
 
 
@@ -108,7 +114,7 @@ def test_multi_token_decode_past_max_len_flags_and_skips(torch):
 def test_multi_token_decode_rejects_bad_shapes(torch):
     from paper_2607_15865_gb300 import _lib
     from paper_2607_15865_gb300.attention import Attention
-    for shape, n in ((Shape("mt_bad1", 1, 40, 8, 128, 256, 1.0e4), 4),   # 5 heads x 4 tokens > 16
+    for shape, n in ((Shape("mt_bad1", 1, 40, 8, 128, 256, 1.0e4), 17),  # more than 16 new tokens
                      (Shape("mt_bad2", 1, 4, 2, 64, 256, 1.0e4), 2)):     # head_dim 64
         attn = Attention.for_shape(shape)
         q, k, v = (to_dev(a) for a in w.tokens(shape, "bad", n))
