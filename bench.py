@@ -14,8 +14,10 @@ value     algorithmic attention FLOP of the step (4*D per unmasked query-key pai
 e2e       the same metric through the same C-ABI calls with host buffers: every
           step copies its q/k/v from pinned host memory and its outputs back
           (copies on their own streams, overlapping the neighbouring steps' compute).
-roofline  the dominant kernel (flash_fwd) against the measured bf16 tensor peak.
-stages    per-stage times; prefill stages in TFLOP/s, decode in HBM GB/s.
+roofline  the dominant kernel (flash_fwd) against the measured sustained bf16 tensor peak
+          (it is timed inside the step loop; the burst-peak fraction is given beside it).
+stages    per-stage times; prefill stages in TFLOP/s (fraction of the sustained peak),
+          decode in HBM GB/s.
 configs   every configuration's stage on its own (7B-class prefill 512, prefill_kv 512 over
           1536, the decode sweep, the long-context stages): median of CUDA-event-timed calls
           with L2 flushed before each, TFLOP/s or GB/s and the fraction of the measured peak.
@@ -440,6 +442,10 @@ def run_ours(args):
         flash_flops = (FLOPS["prefill"] + FLOPS["prefill_kv"]) * K
         flash_tflops = flash_flops / (flash_ms * 1e-3) / 1e12
         tc_peak = float(peaks["bf16_tflops"])
+        # flash_fwd is timed inside the K-step loop (seconds of back-to-back tensor work under
+        # the power cap): its roofline is the sustained dense bf16 figure; the burst one (a
+        # kernel timed alone, as the per-configuration rows are) is reported beside it.
+        tc_sustained = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
         traffic = flash_traffic_from_profile()
         hbm = float(peaks["hbm_gbs"])
         stages = {}
@@ -451,7 +457,7 @@ def run_ours(args):
                                 "kernel_ms": {k: kern[k][0] / K for k in ("decode_split", "decode_combine")}}
             else:
                 tf = FLOPS[name] / t_s / 1e12
-                stages[name] = {"ms": stage_ms[name], "TFLOP/s": tf, "frac_tensor": tf / tc_peak}
+                stages[name] = {"ms": stage_ms[name], "TFLOP/s": tf, "frac_tensor": tf / tc_sustained}
         launches = int(sum(n for _, n in kern.values()))
         result = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
@@ -460,9 +466,10 @@ def run_ours(args):
             "config": {"workload": WORKLOAD, "l2": "flushed between steps (256 MB write + 256 MB read, untimed)",
                        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "step_gflop": STEP_FLOPS / 1e9},
-            "roofline": {"bound": "tensor", "achieved": flash_tflops, "peak": tc_peak, "unit": "TFLOP/s",
-                         "frac": flash_tflops / tc_peak, "traffic": traffic, "kernel": "flash_fwd",
-                         "peak_source": f"{peak_kind} bf16_tflops (burst)",
+            "roofline": {"bound": "tensor", "achieved": flash_tflops, "peak": tc_sustained, "unit": "TFLOP/s",
+                         "frac": flash_tflops / tc_sustained, "traffic": traffic, "kernel": "flash_fwd",
+                         "peak_source": f"{peak_kind} bf16_tflops_sustained (timed inside the {K}-step loop)",
+                         "frac_of_burst_peak": flash_tflops / tc_peak, "burst_peak": tc_peak,
                          "launch_ms_avg": flash_ms / max(flash_n, 1)},
             "stages": stages,
             "kernels_ms_per_step": {k: v[0] / K for k, v in kern.items()},
