@@ -503,6 +503,7 @@ def config_rows(dev, reps: int, graphs: bool):
     outside the events.  graphs: also time each decode step replayed from a CUDA graph."""
     import torch
     from paper_2607_15865_gb300.attention import Attention
+    from synthetic.workloads import Shape
     flush_w = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     peaks, _ = load_peaks()
@@ -591,6 +592,26 @@ def config_rows(dev, reps: int, graphs: bool):
             row["graph_ms"], row["graph_GB/s"] = ms_g, decode_bytes(sh, hist) / (ms_g * 1e-3) / 1e9
             del grs
         attn.close()
+    # a batch of 16 with lengths spread over 64 .. 8191 (seeded): the split counts follow the
+    # lengths, so the byte rate should stay near the uniform batch's
+    sh = w.decode_shape(16)
+    attn = Attention.for_shape(sh)
+    kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
+    q = rnd((sh.batch, 1, sh.n_q_heads, sh.head_dim), gen)
+    k = rnd((sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+    v = rnd((sh.batch, 1, sh.n_kv_heads, sh.head_dim), gen)
+    out = torch.empty_like(q)
+    lens = np.random.default_rng(16).integers(64, 8192, sh.batch).astype(np.int32)
+    hl = torch.from_numpy(lens).to(dev)
+    ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), reps)
+    one = Shape("one", 1, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.max_len, sh.rope_theta)
+    byts = sum(decode_bytes(one, int(h)) for h in lens)
+    gbs = byts / (ms * 1e-3) / 1e9
+    rows.append({"config": f"decode B16 lengths spread over 64..8191 (mean {int(lens.mean())})", "ms": ms,
+                 "GB/s": gbs, "frac_hbm": gbs / hbm})
+    attn.close()
+    del kc, vc
     attn = Attention.for_shape(S)
     kc = rnd((1, 8, 32768, 128), gen)
     vc = rnd((1, 8, 32768, 128), gen)
