@@ -137,11 +137,16 @@ int attn_decode(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint1
  * hist_len[b] + i, is written to that slot and attends to slots [0, hist_len[b] + i]
  * (causal among the new tokens); lengths are per sequence, read on the device.
  *   q [batch, n_new, Hq, D], k/v [batch, n_new, Hkv, D], out [batch, n_new, Hq, D].
- * head_dim 128, 1 <= n_new <= 16 (ATTN_EINVAL otherwise).  The n_new * (Hq / Hkv)
+ * head_dim 128: 1 <= n_new <= 16 (ATTN_EINVAL otherwise).  The n_new * (Hq / Hkv)
  * (query head, token) columns of a kv head run in groups of 16, one group per CTA of a key
  * range; the groups of one range read the same cache tiles at about the same time, so the
  * repeats come from L2 while the history fits there.  A sequence whose hist_len[b] + n_new
- * exceeds max_len is skipped and flagged as in attn_decode.  n_new = 1 is attn_decode.
+ * exceeds max_len is skipped and flagged as in attn_decode.
+ * head_dim 64: 1 <= n_new <= max_len; the tokens run as n_new attn_decode steps in order
+ * (token t at hist_len[b] + t, the same result), each step's rows copied in and out of the
+ * context's buffers, so the history is streamed n_new times; a token whose position passes
+ * max_len - 1 is flagged and skipped as one attn_decode step would (the tokens before it in
+ * that sequence are computed).  n_new = 1 is attn_decode.
  */
 int attn_decode_multi(attn_ctx* ctx, const uint16_t* q, const uint16_t* k, const uint16_t* v,
                       const int32_t* d_hist_len, int n_new, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,

@@ -377,8 +377,33 @@ int attn_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
 int attn_decode_multi(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v,
                       const int32_t* d_hist_len, int n_new, uint16_t* k_cache, uint16_t* v_cache, uint16_t* out,
                       attn_stream_t stream) {
-    return run_decode(c, q, k, v, d_hist_len, 0, false, k_cache, v_cache, out, reinterpret_cast<cudaStream_t>(stream),
-                      n_new);
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (c == nullptr || c->cfg.head_dim == 128 || n_new == 1)
+        return run_decode(c, q, k, v, d_hist_len, 0, false, k_cache, v_cache, out, st, n_new);
+    // head_dim 64: the n_new tokens as n_new decode steps in order (token t at hist_len[b] + t
+    // sees the tokens before it in the cache, which is the same computation); each step's
+    // rows are gathered into the context's decode-block buffers and its output scattered back.
+    if (q == nullptr || k == nullptr || v == nullptr || out == nullptr || n_new < 1 || n_new > c->cfg.max_len)
+        return ATTN_EINVAL;
+    const size_t D = static_cast<size_t>(c->cfg.head_dim), B = static_cast<size_t>(c->cfg.batch);
+    const size_t qrow = c->cfg.n_q_heads * D * 2, krow = c->cfg.n_kv_heads * D * 2;  // bytes of one token's rows
+    for (int t = 0; t < n_new; ++t) {
+        cudaError_t e = cudaMemcpy2DAsync(c->d_lq, qrow, reinterpret_cast<const uint8_t*>(q) + t * qrow, n_new * qrow,
+                                          qrow, B, cudaMemcpyDeviceToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(c->d_lk, krow, reinterpret_cast<const uint8_t*>(k) + t * krow, n_new * krow, krow, B,
+                                  cudaMemcpyDeviceToDevice, st);
+        if (e == cudaSuccess)
+            e = cudaMemcpy2DAsync(c->d_lv, krow, reinterpret_cast<const uint8_t*>(v) + t * krow, n_new * krow, krow, B,
+                                  cudaMemcpyDeviceToDevice, st);
+        if (e != cudaSuccess) return cuda_fail(e, "decode_multi gather");
+        const int rc = run_decode(c, c->d_lq, c->d_lk, c->d_lv, d_hist_len, t, false, k_cache, v_cache, c->d_lo, st);
+        if (rc != ATTN_OK) return rc;
+        e = cudaMemcpy2DAsync(reinterpret_cast<uint8_t*>(out) + t * qrow, n_new * qrow, c->d_lo, qrow, qrow, B,
+                              cudaMemcpyDeviceToDevice, st);
+        if (e != cudaSuccess) return cuda_fail(e, "decode_multi scatter");
+    }
+    return ATTN_OK;
 }
 
 int attn_prompt(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t* v, int hist_len, int prompt_len,

@@ -39,6 +39,9 @@ CASES = [
     ("g8_eight_tokens_4_groups", Shape("mt7", 2, 64, 8, 128, 1024, 1.0e6), [200, 900], 8),
     ("g16_sixteen_tokens_16_groups", Shape("mt8", 1, 16, 1, 128, 512, 1.0e4), [250], 16),
     ("g5_seven_tokens_ragged_group", Shape("mt9", 1, 40, 8, 128, 4096, 1.0e6), [4080], 7),
+    # head_dim 64: the tokens as decode steps in order
+    ("d64_g2_five_tokens", Shape("mt10", 3, 4, 2, 64, 512, 1.0e4), [0, 77, 400], 5),
+    ("d64_g4_two_tokens_tiny", Shape("mt11", 1, 4, 1, 64, 32, 1.0e4), [24], 2),
 ]
 
 
@@ -115,7 +118,7 @@ def test_multi_token_decode_rejects_bad_shapes(torch):
     from paper_2607_15865_gb300 import _lib
     from paper_2607_15865_gb300.attention import Attention
     for shape, n in ((Shape("mt_bad1", 1, 40, 8, 128, 256, 1.0e4), 17),  # more than 16 new tokens
-                     (Shape("mt_bad2", 1, 4, 2, 64, 256, 1.0e4), 2)):     # head_dim 64
+                     (Shape("mt_bad2", 1, 4, 2, 64, 16, 1.0e4), 17)):     # head_dim 64, more than max_len
         attn = Attention.for_shape(shape)
         q, k, v = (to_dev(a) for a in w.tokens(shape, "bad", n))
         kc, vc = (to_dev(a) for a in w.cache(shape, "bad", 0))
