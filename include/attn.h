@@ -38,15 +38,20 @@
  * context owns only its own device memory: the RoPE tables (2 x max_len x
  * head_dim/2 floats, held twice: position-major and pair-major), the decode
  * split-KV partials (batch x n_q_heads x 256 x (head_dim + 2) floats) and counters
- * (2 x batch x n_kv_heads ints), the prefill partials of split work (SM count x
- * 256 x (head_dim + 2) floats) and a device error word; all allocated by attn_create
+ * (2 x batch x n_kv_heads x 16 ints: one set per column group of the multi-token
+ * decode), the prefill partials of split work (SM count x 256 x (head_dim + 2)
+ * floats), the q, k, v and attention output of one decode block (attn_decode_layer)
+ * and a device error word; all allocated by attn_create
  * and freed by attn_destroy.  No stage call allocates, frees or synchronises: each one only
  * enqueues kernels on `stream` and returns.  Calls that use the same context
  * share its scratch buffers, so they must not run concurrently on different
  * streams.
  *
  * Errors.  Every int-returning call returns ATTN_OK (0) or a negative code and
- * writes nothing when it rejects its arguments.  Launch failures return
+ * writes nothing when it rejects its arguments; that includes shapes whose launch
+ * would exceed a grid limit (a decode with batch x column groups, or head_dim 64
+ * kv heads x head passes, above 65535; a prefill chunk whose pairs of 128-row
+ * query tiles x n_q_heads x batch exceed 2^30).  Launch failures return
  * ATTN_ECUDA (attn_last_cuda_error_string() gives the runtime's text).  The
  * decode lengths live on the device, so a decode whose hist_len[b] is outside
  * [0, max_len - 1] cannot be rejected on the host: the kernels then skip

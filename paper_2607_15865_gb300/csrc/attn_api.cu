@@ -150,6 +150,9 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(kc) || !aligned16(vc) || !aligned16(out))
         return ATTN_EINVAL;
     const attn::Shape& s = c->shape;
+    // flash_fwd's work items (pairs of 128-row query tiles x query heads x sequences) are
+    // counted in int: keep them well inside it
+    if ((static_cast<long long>(chunk) + 255) / 256 * s.n_q_heads * s.batch > (1LL << 30)) return ATTN_EINVAL;
     const cuuint64_t D = static_cast<cuuint64_t>(s.head_dim);
     attn::FlashMaps maps;
     {
@@ -346,6 +349,11 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
     if (ntok < 1 || ntok > kMaxDraftTokens || (ntok > 1 && !tc)) return ATTN_EINVAL;
     // the partials hold batch * Hq * nsplit_max rows: ntok tokens share them
     const int ncg = attn::decode_tc_column_groups(c->cfg.n_q_heads / c->cfg.n_kv_heads, ntok);
+    // grid y and z (kv heads; sequences x column groups, or kv heads x head passes) stay
+    // within the 65535 limit of those grid dimensions
+    const int G = c->cfg.n_q_heads / c->cfg.n_kv_heads;
+    if (tc ? static_cast<long>(c->cfg.batch) * ncg > 65535 : static_cast<long>(c->cfg.n_kv_heads) * ((G + 7) / 8) > 65535)
+        return ATTN_EINVAL;
     const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms, ncg), c->nsplit_max / ntok)
                           : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {

@@ -148,41 +148,6 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// The same for global memory: generic-proxy stores of this thread before the fence are
-// ordered before its later async-proxy accesses (and, with a release/acquire pair between
-// threads, before another thread's TMA reads that follow its own fence).
-__device__ __forceinline__ void fence_proxy_async_global() {
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-
-// ------------------------------------------------------------------ counters shared between CTAs
-
-__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
-    int v;
-    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ void red_release_gpu_add(int* p, int v) {
-    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-// Wait until *p >= target (acquire).  Gives up like mbar_wait: after `limit_ns`, or as
-// soon as *abort becomes non-zero; returns false then.
-__device__ __forceinline__ bool wait_counter_geq(const int* p, int target, const volatile int* abort,
-                                                 uint64_t limit_ns = 1000000000ull) {
-    if (ld_acquire_gpu(p) >= target) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        __nanosleep(32);
-        if (ld_acquire_gpu(p) >= target) return true;
-        if ((it & 15u) == 0) {
-            if (abort != nullptr && *abort) return false;
-            if (globaltimer_ns() - t0 > limit_ns) return false;
-        }
-    }
-}
-
 // ------------------------------------------------------------------ tcgen05 / TMEM
 
 __device__ __forceinline__ void tmem_alloc(uint32_t holder_smem, uint32_t ncols) {
