@@ -826,15 +826,15 @@ def run_sweep(args):
     gamma = (1.0 + 0.1 * torch.randn(hidden, device=dev, generator=gen)).to(torch.bfloat16)
     kc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
     vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
-    for hist, S in ((0, 4096), (4096, 4096)):
-        x = torch.randn(1, S, hidden, device=dev, generator=gen).to(torch.bfloat16)
-        ws = torch.empty(attn.prefill_layer_workspace(hidden, S), dtype=torch.uint8, device=dev)
+    for hist, n_tok in ((0, 4096), (4096, 4096)):
+        x = torch.randn(1, n_tok, hidden, device=dev, generator=gen).to(torch.bfloat16)
+        ws = torch.empty(attn.prefill_layer_workspace(hidden, n_tok), dtype=torch.uint8, device=dev)
         out = torch.empty_like(x)
         ms = time_calls(lambda: attn.prefill_layer(x, gamma, 1e-6, tq, to, hist, kc, vc, out=out, workspace=ws),
                         max(3, args.sweep_reps // 2))
-        flop = 2.0 * S * (qd + 2 * kd) * hidden + 2.0 * S * hidden * qd + attn_flops(sh, prefill_pairs(hist, S))
+        flop = 2.0 * n_tok * (qd + 2 * kd) * hidden + 2.0 * n_tok * hidden * qd + attn_flops(sh, prefill_pairs(hist, n_tok))
         tf = flop / (ms * 1e-3) / 1e12
-        rows.append({"config": f"W4BF16 attention half of a decoder block, prefill chunk {S} over {hist} "
+        rows.append({"config": f"W4BF16 attention half of a decoder block, prefill chunk {n_tok} over {hist} "
                                f"(hidden {hidden}, Hq {sh.n_q_heads}, Hkv {sh.n_kv_heads})",
                      "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
         del x, ws, out
@@ -921,6 +921,33 @@ def run_w4_stage(args):
     return 0 if flags == 0 else 1
 
 
+def run_gemm_stage(args):
+    """Runs the W4BF16 GEMM of --gemm T,N,K (T tokens, N features, K inputs) --warmup + --reps
+    times on random tiles (no timing, no JSON line): the launch pattern of a profiler capture."""
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_15865_gb300.w4 import TILE_BYTES, w4bf16_gemm
+    T, N, K = (int(v) for v in args.gemm.split(","))
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    g = torch.Generator(device=dev).manual_seed(3)
+    tiles = torch.randint(0, 256, ((N + 15) // 16 * (K // 128), TILE_BYTES), dtype=torch.uint8, device=dev,
+                          generator=g)
+    tiles[:, 1024:1056].view(torch.int16).fill_(0x3C00)  # scales 2^-7 (bf16)
+    tiles[:, 1056:] &= 15
+    x = torch.randn(T, K, device=dev, generator=g).to(torch.bfloat16)
+    y = torch.empty((T, N), dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    for _ in range(args.warmup + args.reps):
+        w4bf16_gemm(tiles.view(-1), x, N, out=y, err=err)
+    torch.cuda.synchronize()
+    flags = int(err.item())
+    print(f"w4 GEMM T={T} N={N} K={K}: {args.warmup} + {args.reps} calls, device error word {flags}")
+    return 0 if flags == 0 else 1
+
+
 def run_layer_stage(args):
     """Runs --layer B,HIST: the attention half of one 8B-class decoder block (hidden 4096,
     Hq 32, Hkv 8, D 128) at HIST valid tokens through attn_decode_layer, --warmup + --reps
@@ -985,6 +1012,7 @@ def main():
     ap.add_argument("--chunk", type=int)
     ap.add_argument("--w4", help="M,N,K: run only the W4BF16 GEMV of that shape (for profiler captures)")
     ap.add_argument("--layer", help="B,HIST: run only the W4BF16 decode block (for profiler captures)")
+    ap.add_argument("--gemm", help="T,N,K: run only the W4BF16 GEMM of that shape (for profiler captures)")
     args = ap.parse_args()
     if args.stage:  # no timing in this mode
         return run_stage(args)
@@ -992,6 +1020,8 @@ def main():
         return run_w4_stage(args)
     if args.layer:
         return run_layer_stage(args)
+    if args.gemm:
+        return run_gemm_stage(args)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":

@@ -324,6 +324,17 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                     const uint32_t d_col = tmem + (static_cast<uint32_t>(q * 32) << 16) + kTmAcc + 128u * h;
 #pragma unroll 1
                     for (int c = 0; c < kBT / 32; ++c) {
+                        const int tb = t0 + 32 * c;
+                        // the residual of these 32 tokens, all loads in flight at once (h may be
+                        // x: each element is read here before this thread writes it below)
+                        uint32_t res[32];
+                        if (epi.residual != nullptr && n < N) {
+#pragma unroll
+                            for (int e = 0; e < 32; ++e)
+                                res[e] = tb + e < T ? static_cast<uint32_t>(
+                                                          epi.residual[static_cast<size_t>(tb + e) * N + n])
+                                                    : 0u;
+                        }
                         uint32_t r[32];
                         tmem_ld32(d_col + 32u * c, r);
                         tmem_wait_ld();
@@ -333,17 +344,13 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                             __syncwarp();
                             if (lane == 0) mbar_arrive(bar(B_ACCEMPTY0 + h));
                         }
-                        const int tb = t0 + 32 * c;
                         if (n < N) {
 #pragma unroll
                             for (int e = 0; e < 32; ++e) {
                                 const int t = tb + e;
                                 if (t < T) {
                                     float v = __uint_as_float(r[e]);
-                                    if (epi.residual != nullptr)
-                                        v += __uint_as_float(static_cast<uint32_t>(
-                                                                 epi.residual[static_cast<size_t>(t) * N + n])
-                                                             << 16);
+                                    if (epi.residual != nullptr) v += __uint_as_float(res[e] << 16);
                                     dst[static_cast<size_t>(t) * stride + cc] = __bfloat16_as_ushort(__float2bfloat16_rn(v));
                                 }
                             }
