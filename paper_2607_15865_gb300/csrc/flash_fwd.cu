@@ -128,20 +128,38 @@ struct Item {
 // pieces; with the divisors the kernels use, as fast divisions (every division of the
 // schedule ran as a generic integer division before: about 1 us per decoded unit).
 struct Sched {
-    int S, H, Hq, batch, n_pairs, head, nsplit, n_units;
-    FastDiv fd_grid, fd_hqb, fd_hq, fd_g, fd_ns;
+    int S, H, Hq, G, batch, n_pairs, head, nsplit, n_units;
+    int kvb;  // item order: 0 longest pairs first over all heads, else blocks of kvb kv heads
+    FastDiv fd_grid, fd_hqb, fd_hq, fd_g, fd_ns, fd_pb, fd_per, fd_nb;
 };
 
-// Item order: longest query-tile pairs first across every (head, sequence), so a
-// causal launch starts its longest items first and ends with the shortest.
+// Item order.  By default the longest query-tile pairs come first across every (head,
+// sequence), so a causal launch starts its longest items first and ends with the
+// shortest.  When a long history makes the items about equally long and the K/V the
+// launch reads is a large part of L2, the items are grouped in blocks of kvb kv heads of
+// one sequence instead -- within a block longest pairs first, the block's query heads of
+// a pair together -- so the CTAs of a round walk the K/V of only those kv heads, which
+// stays in L2, and each kv head's cache is read from DRAM about once instead of once per
+// round.
 __device__ __forceinline__ Item decode_item(int lin, const Sched& sc) {
     Item it;
-    const int qt = fdiv(lin, sc.fd_hqb);
-    const int rem = lin - qt * (sc.Hq * sc.batch);
+    int qt;
+    if (sc.kvb) {
+        const int per = sc.kvb * sc.G;        // query heads of a block
+        const int blk = fdiv(lin, sc.fd_pb);  // (sequence, block of kv heads)
+        const int r = lin - blk * (sc.n_pairs * per);
+        qt = fdiv(r, sc.fd_per);
+        it.b = fdiv(blk, sc.fd_nb);
+        it.h = (blk - it.b * fdiv(sc.Hq, sc.fd_per)) * per + (r - qt * per);
+        it.g = fdiv(it.h, sc.fd_g);
+    } else {
+        qt = fdiv(lin, sc.fd_hqb);
+        const int rem = lin - qt * (sc.Hq * sc.batch);
+        it.b = fdiv(rem, sc.fd_hq);
+        it.h = rem - it.b * sc.Hq;
+        it.g = fdiv(it.h, sc.fd_g);
+    }
     const int pt = sc.n_pairs - 1 - qt;
-    it.b = fdiv(rem, sc.fd_hq);
-    it.h = rem - it.b * sc.Hq;
-    it.g = fdiv(it.h, sc.fd_g);
     it.q0a = pt * 2 * BM;
     it.q0b = it.q0a + BM;
     it.rowsa = max(0, min(BM, sc.S - it.q0a));
@@ -791,8 +809,14 @@ __global__ void __launch_bounds__(256) flash_combine_kernel(const float* __restr
 // tensor-core time of four 128 x 128 x D MMAs, and for a split launch the partial writes
 // and the merge kernel.
 struct HostSchedule {
-    int n_pairs, n_items, head, nsplit, n_units, grid;
+    int n_pairs, n_items, head, nsplit, n_units, grid, kvb;
 };
+
+// Items are grouped in blocks of kv heads when the history is at least the chunk and the
+// launch's K/V exceeds kKvBlockFrom; a block's K/V stays within kKvBlockBytes (of 126 MB
+// of L2).  Causal launches without such a history keep the longest-first order, whose
+// balance matters more there.
+constexpr double kKvBlockFrom = 42.0e6, kKvBlockBytes = 48.0e6;
 
 constexpr int kMaxSplit = 16;
 
@@ -807,9 +831,17 @@ HostSchedule make_schedule(const Shape& s, int hist, int chunk, int num_sms) {
     const int n_qtiles = (chunk + BM - 1) / BM;
     sc.n_pairs = (n_qtiles + 1) / 2;
     sc.n_items = sc.n_pairs * s.n_q_heads * s.batch;
-    const int hq_b = s.n_q_heads * s.batch;
-    auto n_kv = [&](int item) {  // KV tiles of an item (longest pairs first)
-        const int pt = sc.n_pairs - 1 - item / hq_b;
+    const int hq_b = s.n_q_heads * s.batch, G = s.n_q_heads / s.n_kv_heads;
+    const double head_bytes = 4.0 * (static_cast<double>(hist) + chunk) * s.head_dim;  // K/V of one kv head
+    sc.kvb = 0;
+    if (hist >= chunk && head_bytes * s.batch * s.n_kv_heads > kKvBlockFrom) {
+        sc.kvb = 1;
+        for (int d = 1; d <= s.n_kv_heads; ++d)
+            if (s.n_kv_heads % d == 0 && d * head_bytes <= kKvBlockBytes) sc.kvb = d;
+    }
+    auto n_kv = [&](int item) {  // KV tiles of an item (longest pairs first, in either order)
+        const int qt = sc.kvb ? item % (sc.n_pairs * sc.kvb * G) / (sc.kvb * G) : item / hq_b;
+        const int pt = sc.n_pairs - 1 - qt;
         return (hist + std::min(2 * BM * (pt + 1), chunk) + BN - 1) / BN;
     };
     // costs in KV steps of both query tiles (about 1.3 us each)
@@ -859,7 +891,9 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     sc.S = chunk;
     sc.H = hist;
     sc.Hq = s.n_q_heads;
+    sc.G = s.n_q_heads / s.n_kv_heads;
     sc.batch = s.batch;
+    sc.kvb = hs.kvb;
     sc.n_pairs = hs.n_pairs;
     sc.head = hs.head;
     sc.nsplit = hs.nsplit;
@@ -869,6 +903,10 @@ cudaError_t launch_d(const Shape& s, const FlashMaps& maps, int hist, int chunk,
     sc.fd_hq = make_fastdiv(s.n_q_heads);
     sc.fd_g = make_fastdiv(s.n_q_heads / s.n_kv_heads);
     sc.fd_ns = make_fastdiv(hs.nsplit);
+    const int per = std::max(hs.kvb, 1) * sc.G;
+    sc.fd_pb = make_fastdiv(hs.n_pairs * per);
+    sc.fd_per = make_fastdiv(per);
+    sc.fd_nb = make_fastdiv(s.n_q_heads / per);
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     // Dependent launch after K1 (programmatic stream serialization): only the producer's
     // first K/V copy waits for K1 (griddep_wait).

@@ -157,6 +157,15 @@ def test_long_prefill_kv_4096_over_28672(torch):
     check_full_size(torch, w.LONG, "long_pkv", w.LONG_PKV_HIST, w.LONG_PKV_CHUNK, n_pos=6, heads=10)
 
 
+# A prefill_kv whose history is at least its chunk and whose K/V exceeds about 42 MB:
+# flash_fwd then groups its work items in blocks of kv heads of one sequence (blocks of 2
+# kv heads on the long-context shape, of 1 here) instead of by query-tile pair.
+def test_kv_head_blocks_batch2_every_row(torch):
+    """A ragged 333-token chunk over 79000 history tokens, two sequences, 4 kv heads of
+    GQA 3 (40.6 MB of K/V per kv head: one kv head per block), every row."""
+    check_every_row(torch, Shape("kvb_b2", 2, 12, 4, 128, 79400, 1.0e6), "kvb_b2", 79000, 333)
+
+
 def check_every_row(torch, shape, tag, hist, chunk):
     """Every output row of a full-size stage against the oracle, run on all host cores."""
     q, k, v = w.tokens(shape, tag, chunk)
