@@ -33,9 +33,10 @@
 //              copies of the tiles that hold those slots (zeroing the V rows past the
 //              last new slot: slots past it may hold anything, and 0 * NaN would poison
 //              O), so the MMA itself produces the new keys' scores.
-// Merge: with one split the CTA writes the normalised output.  Otherwise each CTA
-// writes its partial (m, l, acc[D]) per column; the last CTA of (b, kv head) to finish
-// (a device counter, reset by that CTA) merges them:
+// Merge: with one working split (splits past the sequence's T tiles get none) the CTA
+// writes the normalised output.  Otherwise each working CTA writes its partial
+// (m, l, acc[D]) per column; the last of them to finish (a device counter, reset by
+// that CTA) merges them:
 //   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its copies
 // and MMAs finish, releases TMEM and still takes part in the merge count.
@@ -89,8 +90,8 @@ struct L {
     static constexpr int ALLOC = BYTES + 1024;
 };
 static_assert(L::ALLOC <= 232448, "shared memory of one CTA");
-static_assert(NH * 256 * 8 + NH * 4 + (kThreads / 32) * NH * D * 4 <= KST * L::TILE + VST * L::TILE,
-              "merge buffers fit in the rings");
+static_assert((kThreads / 32) * NH * 8 + (kThreads / 32) * NH * D * 4 <= KST * L::TILE,
+              "merge buffers fit in the K ring");
 
 __device__ __forceinline__ float bf16_at(const uint16_t* p) { return __uint_as_float(static_cast<uint32_t>(*p) << 16); }
 __device__ __forceinline__ uint16_t to_bf16(float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
@@ -205,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
     int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
-    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg) {
+    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg, int spec) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -233,18 +234,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     // starts (it is a dependent launch only after another decode step, which lets its
     // dependents start only once its own predecessors are complete).
     const int hist = decode_hist(d_hist, b, hist_add);  // in flight while the barriers and TMEM are set up
+    const int kv_row = b * Hkv + g;
+    // The producer sets up the barriers and, unless the previous kernel may have written the
+    // cache (a decode step right after another, spec = 0), issues the copies of its first
+    // tile, tile s, before the length is known: the K slot's arrival is held back until the
+    // producer knows whether tile s holds keys of the sequence (the copies read in-range
+    // slots or the map's zero fill either way; a tile past the sequence is not used).
+    const bool spec_first = spec != 0 && s * KT < max_len;
     if (warp == kWarpTma && lane == 0) {
-        tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_v);
-    }
-
-    if (tid < NH) {
-        const int c = c0 + min(tid, C - 1);
-        const size_t r = (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G;
-        reinterpret_cast<size_t*>(gb + L::OFF_OROW)[tid] = r;
-        reinterpret_cast<size_t*>(gb + L::OFF_CROW)[tid] = r * nsplit;
-    }
-    if (tid == 0) {
         *abort_flag = 0;
         mbar_init(bar(B_QREADY), 128);
         for (int st = 0; st < KST; ++st) {
@@ -263,6 +260,25 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         mbar_init(bar(B_OFULL), 1);
         mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        if (spec_first) {
+            mbar_expect_tx(bar(B_KFULL0), L::TILE);
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+                tma_load_3d(base + L::OFF_K + c * L::BOX, &map_k, c * 64, s * KT, kv_row, bar(B_KFULL0));
+            mbar_arrive_expect_tx(bar(B_VFULL0), L::TILE);
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+                tma_load_3d(base + L::OFF_V + c * L::BOX, &map_v, c * 64, s * KT, kv_row, bar(B_VFULL0));
+        }
+    }
+
+    if (tid < NH) {
+        const int c = c0 + min(tid, C - 1);
+        const size_t r = (static_cast<size_t>(b) * ntok + c / G) * Hq + h0 + c % G;
+        reinterpret_cast<size_t*>(gb + L::OFF_OROW)[tid] = r;
+        reinterpret_cast<size_t*>(gb + L::OFF_CROW)[tid] = r * nsplit;
     }
     if (warp == kWarpMma) {
         tmem_alloc(base + L::OFF_TMEM, kTmemCols);
@@ -290,7 +306,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     if (!hist_ok && s == 0 && g == 0 && cg == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
     const int nkeys = hist + ntok;        // slots [0, hist) and the new tokens' [hist, hist + ntok)
     const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds the last new slot
-    const int kv_row = b * Hkv + g;
+    // Splits s < T each take at least tile s; splits past T get no tile, write nothing and
+    // stay out of the merge, which combines the n_work = min(nsplit, T) working splits.
+    const bool working = s < T;
+    const int n_work = min(nsplit, T);
     const int ctr_row = kv_row * ncg + cg;  // counters of this (sequence, kv head, column group)
     // Rows of column c (token c / G, head h0 + c % G), tabulated once in the prologue:
     // q / out row (b * ntok + c / G) * Hq + h0 + c % G, and partial row of split 0 that
@@ -300,7 +319,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     int* meta = reinterpret_cast<int*>(gb + L::OFF_META);  // tile index of local tile j at [j % 8]; -1 ends
 
     if (!hist_ok) {
-        // sequence skipped: nothing written
+        // sequence skipped: nothing written (the speculative copies land before the CTA ends)
+        if (spec_first && warp == kWarpTma && lane == 0) {
+            mbar_arrive(bar(B_KFULL0));
+            mbar_wait(bar(B_KFULL0), 0u, nullptr);
+            mbar_wait(bar(B_VFULL0), 0u, nullptr);
+        }
     } else if (warp == kWarpTma) {
         // ------------------------------------------------------------ TMA producer (lane 0)
         // Tiles are claimed, not fixed: split s starts with tile s, then takes tickets
@@ -311,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         if (lane == 0) {
             int* tile_ctr = counters + gridDim.y * gridDim.z + ctr_row;
             int cur = s < T ? s : T;
-            int nxt = (nsplit > 1 && cur < T) ? nsplit + atomicAdd(tile_ctr, 1) : cur + 1;
+            int nxt = (n_work > 1 && cur < T) ? nsplit + atomicAdd(tile_ctr, 1) : cur + 1;
             int issued_k = 0, issued_v = 0;
             bool ok = true;
             for (int j = 0;; ++j) {
@@ -322,6 +346,22 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     break;
                 }
                 meta[j % 8] = tile;
+                if (j == 0 && spec_first) {
+                    // tile s is in flight: its K slot's arrival publishes meta[0]
+                    mbar_arrive(bar(B_KFULL0));
+                    issued_k = issued_v = 1;
+                    if (tile < 0) {  // tile s holds no keys of the sequence: the copies still land
+                        mbar_wait(bar(B_VFULL0), 0u, nullptr);
+                        break;
+                    }
+                    cur = nxt;
+                    if (n_work > 1) {
+                        if (cur < T) nxt = nsplit + atomicAdd(tile_ctr, 1);
+                    } else {
+                        nxt = cur + 1;
+                    }
+                    continue;
+                }
                 if (tile < 0) {  // no more tiles: complete the K slot's phase without data
                     mbar_arrive(bar(B_KFULL0 + ks));
                     break;
@@ -343,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                                 bar(B_VFULL0 + vs));
                 issued_v = j + 1;
                 cur = nxt;
-                if (nsplit > 1) {
+                if (n_work > 1) {
                     if (cur < T) nxt = nsplit + atomicAdd(tile_ctr, 1);
                 } else {
                     nxt = cur + 1;
@@ -617,7 +657,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             mbar_arrive(bar(B_PFULL0 + (j & 1)));
         }
         if (ok && n == 0) {
-            if (t < C) {  // no tile came to this CTA: weight 0 in the merge
+            if (working && n_work > 1 && t < C) {  // (not reached: a working split has tile s)
                 part_ml[(crow[t] + s) * 2 + 0] = -INFINITY;
                 part_ml[(crow[t] + s) * 2 + 1] = 0.f;
             }
@@ -640,7 +680,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                 if (h < C) {
                     const float4 l4 = reinterpret_cast<const float4*>(ls)[h];
                     const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
-                    if (nsplit == 1) {
+                    if (n_work == 1) {
                         out[orow[h] * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
                     } else {
                         const size_t row = crow[h] + s;
@@ -659,14 +699,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     }
 
     // ---------------------------------------------------------------- merge of the splits
-    if (hist_ok && nsplit > 1) {
+    if (hist_ok && n_work > 1 && working) {
         int* last_flag = reinterpret_cast<int*>(gb + L::OFF_LAST);
         __threadfence();  // this CTA's partials are visible before it is counted
         tc_fence_before();
         __syncthreads();
         if (tid == 0) {
             int* cnt = counters + ctr_row;
-            const int last = atomicAdd(cnt, 1) == nsplit - 1;
+            const int last = atomicAdd(cnt, 1) == n_work - 1;
             if (last) {  // every split of this launch has been counted and has claimed its last tile
                 *cnt = 0;
                 counters[gridDim.y * gridDim.z + ctr_row] = 0;
@@ -676,83 +716,78 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         __syncthreads();
         tc_fence_after();
         if (*last_flag) {
-            // All six warps merge; shared memory of the (idle) K ring holds
-            //   wml  [G][nsplit] float2: (m_s, l_s), then (weight_s, -) per head and split
-            //   winv [G]         1 / L per head
-            //   racc [6 warps][G][D] float: each warp's weighted sum over its splits.
-            // Splits without keys have l = 0 and weight 0; their accumulators were never
-            // written, and what is read there is discarded.
+            // All six warps merge in one pass over the partials: warp w takes splits w, w+6, ...,
+            // lane l dimensions 4l .. 4l+3 of every column, and keeps a running (M, L, acc) per
+            // column, rescaled as a larger split maximum comes in; then the six warps' results
+            // meet in shared memory (the idle K ring):
+            //   wml  [6 warps][16] float2 (M_w, L_w);  racc [6 warps][16][D] float acc_w.
+            // Splits without keys have l = 0 and are skipped; their accumulators were never
+            // written, and what is read there is discarded by a select.
             __threadfence();
             float2* wml = reinterpret_cast<float2*>(gb + L::OFF_K);
-            float* winv = reinterpret_cast<float*>(gb + L::OFF_K + NH * 256 * 8);
-            float* racc = winv + NH;
-            for (int p = tid; p < C * nsplit; p += kThreads) {  // pair p = (column p / nsplit, split p % nsplit)
-                const int c = p / nsplit;
-                wml[p] = __ldcg(reinterpret_cast<const float2*>(part_ml) + crow[c] + (p - c * nsplit));
-            }
-            __syncthreads();
-            for (int h = warp; h < C; h += kThreads / 32) {  // per column: M, weights, 1/L
-                float mm = -INFINITY;
-                for (int sp = lane; sp < nsplit; sp += 32) {
-                    const float2 ml = wml[h * nsplit + sp];
-                    if (ml.y > 0.f) mm = fmaxf(mm, ml.x);
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xFFFFFFFFu, mm, off));
-                float ll = 0.f;
-                for (int sp = lane; sp < nsplit; sp += 32) {
-                    const float2 ml = wml[h * nsplit + sp];
-                    const float wgt = ml.y > 0.f ? fast_exp2(ml.x - mm) : 0.f;
-                    wml[h * nsplit + sp].x = wgt;
-                    ll += ml.y * wgt;
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) ll += __shfl_xor_sync(0xFFFFFFFFu, ll, off);
-                if (lane == 0) winv[h] = 1.f / ll;
-            }
-            __syncthreads();
-            // warp w: splits w, w+6, ...; lane l: dimensions 4l .. 4l+3 of every head
+            float* racc = reinterpret_cast<float*>(gb + L::OFF_K + (kThreads / 32) * NH * 8);
             float4 acc[NHP];
+            float mw[NHP], lw[NHP];
 #pragma unroll
-            for (int h = 0; h < NHP; ++h) acc[h] = make_float4(0.f, 0.f, 0.f, 0.f);
-            // (Every load is issued unconditionally -- padded heads re-read head G-1 -- and
-            // weight-0 values are dropped by a select, so that the loads of a split for
-            // all heads are in flight together instead of each waiting on a branch.)
+            for (int h = 0; h < NHP; ++h) {
+                acc[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+                mw[h] = -INFINITY;
+                lw[h] = 0.f;
+            }
+            // (Every load is issued unconditionally -- padded columns re-read column C-1 --
+            // so that the loads of a split for all columns are in flight together.)
 #pragma unroll 2
-            for (int sp = warp; sp < nsplit; sp += kThreads / 32) {
+            for (int sp = warp; sp < n_work; sp += kThreads / 32) {
                 float4 o4[NHP];
-                float wgt[NHP];
+                float2 ml[NHP];
 #pragma unroll
                 for (int h = 0; h < NHP; ++h) {
                     const int hh = min(h, C - 1);
-                    wgt[h] = h < C ? wml[hh * nsplit + sp].x : 0.f;
+                    ml[h] = __ldcg(reinterpret_cast<const float2*>(part_ml) + crow[hh] + sp);
                     o4[h] = __ldcg(reinterpret_cast<const float4*>(part_o + (crow[hh] + sp) * D) + lane);
                 }
 #pragma unroll
                 for (int h = 0; h < NHP; ++h) {
-                    const bool use = wgt[h] != 0.f;
-                    acc[h].x = use ? fmaf(wgt[h], o4[h].x, acc[h].x) : acc[h].x;
-                    acc[h].y = use ? fmaf(wgt[h], o4[h].y, acc[h].y) : acc[h].y;
-                    acc[h].z = use ? fmaf(wgt[h], o4[h].z, acc[h].z) : acc[h].z;
-                    acc[h].w = use ? fmaf(wgt[h], o4[h].w, acc[h].w) : acc[h].w;
+                    const bool use = h < C && ml[h].y > 0.f;
+                    const float mn = use ? fmaxf(mw[h], ml[h].x) : mw[h];
+                    const float a = use ? fast_exp2(mw[h] - mn) : 1.f;  // rescale of what came before
+                    const float wgt = use ? fast_exp2(ml[h].x - mn) : 0.f;
+                    acc[h].x = use ? fmaf(wgt, o4[h].x, acc[h].x * a) : acc[h].x;
+                    acc[h].y = use ? fmaf(wgt, o4[h].y, acc[h].y * a) : acc[h].y;
+                    acc[h].z = use ? fmaf(wgt, o4[h].z, acc[h].z * a) : acc[h].z;
+                    acc[h].w = use ? fmaf(wgt, o4[h].w, acc[h].w * a) : acc[h].w;
+                    lw[h] = use ? fmaf(wgt, ml[h].y, lw[h] * a) : lw[h];
+                    mw[h] = mn;
                 }
             }
 #pragma unroll
             for (int h = 0; h < NHP; ++h)
-                if (h < C) reinterpret_cast<float4*>(racc + (warp * NH + h) * D)[lane] = acc[h];
+                if (h < C) {
+                    reinterpret_cast<float4*>(racc + (warp * NH + h) * D)[lane] = acc[h];
+                    if (lane == 0) wml[warp * NH + h] = make_float2(mw[h], lw[h]);
+                }
             __syncthreads();
             for (int p = tid; p < C * (D / 4); p += kThreads) {  // (column, 4 dimensions)
                 const int h = p / (D / 4), c = p % (D / 4);
+                float mm = -INFINITY;
+#pragma unroll
+                for (int w = 0; w < kThreads / 32; ++w) mm = fmaxf(mm, wml[w * NH + h].x);
                 float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+                float l_tot = 0.f;
 #pragma unroll
                 for (int w = 0; w < kThreads / 32; ++w) {
-                    const float4 v4 = reinterpret_cast<const float4*>(racc + (w * NH + h) * D)[c];
-                    sum.x += v4.x;
-                    sum.y += v4.y;
-                    sum.z += v4.z;
-                    sum.w += v4.w;
+                    const float2 m_l = wml[w * NH + h];
+                    if (m_l.y > 0.f) {  // a warp without keys has M_w = -inf and nothing to add
+                        const float f = fast_exp2(m_l.x - mm);
+                        const float4 v4 = reinterpret_cast<const float4*>(racc + (w * NH + h) * D)[c];
+                        sum.x = fmaf(f, v4.x, sum.x);
+                        sum.y = fmaf(f, v4.y, sum.y);
+                        sum.z = fmaf(f, v4.z, sum.z);
+                        sum.w = fmaf(f, v4.w, sum.w);
+                        l_tot = fmaf(f, m_l.y, l_tot);
+                    }
                 }
-                const float inv = winv[h];
+                const float inv = 1.f / l_tot;
                 const uint2 packed = make_uint2(
                     to_bf16(sum.x * inv) | (static_cast<uint32_t>(to_bf16(sum.y * inv)) << 16),
                     to_bf16(sum.z * inv) | (static_cast<uint32_t>(to_bf16(sum.w * inv)) << 16));
@@ -834,7 +869,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
-                              producer_early ? 1 : 0, wait_ns, ncg);
+                              producer_early ? 1 : 0, wait_ns, ncg, after_decode ? 0 : 1);
 }
 
 }  // namespace attn
