@@ -17,7 +17,11 @@
 // (the MMA's N), token tiles fastest.  448 threads:
 //   warp 0, one lane   producer: per 128-input group one X tile (two 2-D TMA boxes, 128-byte
 //                      swizzle; tokens past T read as zeros) and the 16 weight records of the
-//                      tile's 256 features (bulk copies) into a kStages ring;
+//                      tile's 256 features into a kStages ring: their codes as one 4-D TMA box
+//                      with 64-byte swizzle (row r's 16-byte chunk c lands at chunk
+//                      c ^ ((r >> 1) & 3), so the eight rows that a quarter-warp of decode
+//                      threads reads at once sit in eight different bank groups), their
+//                      scales and zero points as one 3-D box;
 //   warp 1, one lane   tcgen05 issuer: per group and half, 8 MMAs 128 x 128 x 16 from the
 //                      half's A buffer in TMEM and the X stage, into the half's accumulator;
 //   warps 2-9          decode (warps 2-5 the first half's 128 features, 6-9 the second),
@@ -50,15 +54,17 @@ constexpr int kChunk = 128 * 128;           // 128 rows x 64 bf16 (128 bytes), s
 constexpr int kXStage = 2 * kChunk;         // X tile: 128 tokens x 128 inputs
 constexpr int kRecBytes = 1072;             // one weight record: 16 rows x 128 inputs
 constexpr int kRecs = kBF / 16;             // records per stage
-constexpr int kWStage = kRecs * kRecBytes;
+constexpr int kWcStage = kRecs * 16 * 64;   // their codes: 256 rows x 64 bytes, 64-byte swizzle
+constexpr int kWsStage = kRecs * 48;        // their scales and zero points: 16 x 48 bytes
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmA = 0, kTmAcc = 256;
 constexpr uint64_t kWaitNs = 1000000000ull;
 
 struct L {
     static constexpr int OFF_X = 0;
-    static constexpr int OFF_W = OFF_X + kStages * kXStage;
-    static constexpr int OFF_BAR = OFF_W + kStages * kWStage;
+    static constexpr int OFF_WC = OFF_X + kStages * kXStage;
+    static constexpr int OFF_WS = OFF_WC + kStages * kWcStage;
+    static constexpr int OFF_BAR = OFF_WS + kStages * kWsStage;
     static constexpr int NBAR = 2 * kStages + 2 + 2 + 1 + 2 + 1;
     static constexpr int OFF_TMEM = OFF_BAR + 8 * NBAR;
     static constexpr int OFF_ABORT = OFF_TMEM + 16;
@@ -99,7 +105,8 @@ __device__ __forceinline__ uint32_t code_pair(uint32_t w, int j, uint32_t mask, 
 }
 
 __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_constant__ CUtensorMap map_x,
-                                                              const uint8_t* __restrict__ tiles, int T, int N, int K,
+                                                              const __grid_constant__ CUtensorMap map_wc,
+                                                              const __grid_constant__ CUtensorMap map_ws, int T, int N, int K,
                                                               uint16_t* __restrict__ y, int* err, const W4GemmEpi epi) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -127,6 +134,8 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
         mbar_init(bar(B_DRAIN), 1);
         fence_mbar_init();
         tma_prefetch_desc(&map_x);
+        tma_prefetch_desc(&map_wc);
+        tma_prefetch_desc(&map_ws);
     }
     if (warp == kWarpMma) {
         tmem_alloc(base + L::OFF_TMEM, kTmemCols);
@@ -144,7 +153,6 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
             for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
                 const int ft = tile / n_tt, tt = tile - ft * n_tt;
                 const int f0 = ft * kBF, t0 = tt * kBT;
-                const int nrec = min(kRecs, (N - f0) / 16);
                 for (int G = 0; G < ngroup; ++G, ++gs) {
                     const int s = static_cast<int>(gs % kStages);
                     if (gs >= kStages &&
@@ -152,15 +160,13 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(bar(B_FULL0 + s), kXStage + nrec * kRecBytes);
+                    // (row tiles past N read as zeros; every box counts its full size)
+                    mbar_arrive_expect_tx(bar(B_FULL0 + s), kXStage + kWcStage + kWsStage);
                     for (int c = 0; c < 2; ++c)
                         tma_load_2d(base + L::OFF_X + s * kXStage + c * kChunk, &map_x, G * 128 + c * 64, t0,
                                     bar(B_FULL0 + s));
-                    for (int r = 0; r < nrec; ++r) {
-                        const size_t rec = static_cast<size_t>(f0 / 16 + r) * ngroup + G;
-                        bulk_g2s(base + L::OFF_W + s * kWStage + r * kRecBytes, tiles + rec * kRecBytes, kRecBytes,
-                                 bar(B_FULL0 + s));
-                    }
+                    tma_load_4d(base + L::OFF_WC + s * kWcStage, &map_wc, 0, 0, G, f0 / 16, bar(B_FULL0 + s));
+                    tma_load_3d(base + L::OFF_WS + s * kWsStage, &map_ws, 0, G, f0 / 16, bar(B_FULL0 + s));
                 }
             }
             if (!ok) {
@@ -248,18 +254,19 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                     uint32_t wv[16];
                     uint32_t zp = 0x43004300u, sp = 0u;
                     if (have) {
-                        const uint8_t* rec = gb + L::OFF_W + s * kWStage + (rrow >> 4) * kRecBytes;
-                        const uint4* row = reinterpret_cast<const uint4*>(rec + (rrow & 15) * 64);
+                        const uint8_t* row = gb + L::OFF_WC + s * kWcStage + rrow * 64;
+                        const uint8_t* rec = gb + L::OFF_WS + s * kWsStage + (rrow >> 4) * 48;
+                        const int sw = (rrow >> 1) & 3;  // the 64-byte swizzle of this row
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
-                            const uint4 u = row[i];
+                            const uint4 u = *reinterpret_cast<const uint4*>(row + 16 * (i ^ sw));
                             wv[4 * i] = u.x;
                             wv[4 * i + 1] = u.y;
                             wv[4 * i + 2] = u.z;
                             wv[4 * i + 3] = u.w;
                         }
-                        const uint32_t sc = *reinterpret_cast<const uint16_t*>(rec + 1024 + (rrow & 15) * 2);
-                        const uint32_t z = rec[1056 + (rrow & 15)];
+                        const uint32_t sc = *reinterpret_cast<const uint16_t*>(rec + (rrow & 15) * 2);
+                        const uint32_t z = rec[32 + (rrow & 15)];
                         zp = (0x4300u + z) * 0x00010001u;  // (128 + z) in both halves
                         sp = sc * 0x00010001u;
                     } else {
@@ -450,15 +457,42 @@ cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N
             g_configured[dev] = true;
         }
     }
-    CUtensorMap map;
-    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
-    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
-    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBT)};
-    const cuuint32_t estr[2] = {1, 1};
-    const CUresult r = g_encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(x), dims, strides, box,
-                                estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    CUtensorMap map, map_wc, map_ws;
+    {
+        const cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(T)};
+        const cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+        const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kBT)};
+        const cuuint32_t estr[2] = {1, 1};
+        const CUresult r = g_encode(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(x), dims, strides,
+                                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
+    // The tile stream as two views: record (row tile t, group g) at (t * K/128 + g) * 1072 bytes.
+    //   codes  [row tile][group][16 rows][64 bytes]  (16-bit elements, box 32 x 16 x 1 x 16)
+    //   scales and zero points [row tile][group][48 bytes] from byte 1024 of each record
+    const cuuint64_t ng = static_cast<cuuint64_t>(K / 128), nt = static_cast<cuuint64_t>(N / 16);
+    {
+        const cuuint64_t dims[4] = {32, 16, ng, nt};
+        const cuuint64_t strides[3] = {64, kRecBytes, kRecBytes * ng};
+        const cuuint32_t box[4] = {32, 16, 1, static_cast<cuuint32_t>(kRecs)};
+        const cuuint32_t estr[4] = {1, 1, 1, 1};
+        const CUresult r = g_encode(&map_wc, CU_TENSOR_MAP_DATA_TYPE_UINT16, 4, const_cast<uint8_t*>(tiles), dims,
+                                    strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
+    {
+        const cuuint64_t dims[3] = {24, ng, nt};
+        const cuuint64_t strides[2] = {kRecBytes, kRecBytes * ng};
+        const cuuint32_t box[3] = {24, 1, static_cast<cuuint32_t>(kRecs)};
+        const cuuint32_t estr[3] = {1, 1, 1};
+        const CUresult r = g_encode(&map_ws, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, const_cast<uint8_t*>(tiles) + 1024,
+                                    dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                                    CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
     int sms = 0;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
@@ -466,7 +500,7 @@ cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N
     const unsigned grid = static_cast<unsigned>(std::min<long long>(n_tiles, sms));
     W4GemmEpi epi = {N, N, nullptr, nullptr, nullptr};
     if (epi_in != nullptr) epi = *epi_in;
-    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, tiles, T, N, K, y, err, epi);
+    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, map_wc, map_ws, T, N, K, y, err, epi);
     return cudaGetLastError();
 }
 
