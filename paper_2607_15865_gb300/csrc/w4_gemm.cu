@@ -37,6 +37,7 @@
 
 #include <algorithm>
 #include <cstdint>
+#include <map>
 #include <mutex>
 
 #include "internal.h"
@@ -104,9 +105,25 @@ __device__ __forceinline__ uint32_t code_pair(uint32_t w, int j, uint32_t mask, 
     return r;
 }
 
+// Work units: units [0, n_full) are whole output tiles (tile = unit); the tiles after them
+// are cut into their two 128-feature halves, one unit each, so that the last round of the
+// persistent CTAs ends more evenly.  Returns the tile and the mask of its halves (a half
+// past N is never on).
+__device__ __forceinline__ int unit_tile(int u, int n_full, int n_tt, int N, int& hmask) {
+    int tile = u;
+    hmask = 3;
+    if (u >= n_full) {
+        tile = n_full + ((u - n_full) >> 1);
+        hmask = 1 << ((u - n_full) & 1);
+    }
+    if ((tile / n_tt) * kBF + 128 >= N) hmask &= 1;
+    return tile;
+}
+
 __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_constant__ CUtensorMap map_x,
                                                               const __grid_constant__ CUtensorMap map_wc,
-                                                              const __grid_constant__ CUtensorMap map_ws, int T, int N, int K,
+                                                              const __grid_constant__ CUtensorMap map_ws, int n_full, int n_units,
+                                                              int T, int N, int K,
                                                               uint16_t* __restrict__ y, int* err, const W4GemmEpi epi) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -116,8 +133,7 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
     auto bar = [&](int i) -> uint32_t { return base + L::OFF_BAR + 8u * static_cast<uint32_t>(i); };
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int ngroup = K / 128;
-    const int n_tt = (T + kBT - 1) / kBT, n_ft = (N + kBF - 1) / kBF;
-    const int n_tiles = n_tt * n_ft;
+    const int n_tt = (T + kBT - 1) / kBT;
 
     if (tid == 0) {
         *abort_flag = 0;
@@ -150,7 +166,9 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
         if (lane == 0) {
             uint32_t gs = 0;  // groups issued
             bool ok = true;
-            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+                int hmask;
+                const int tile = unit_tile(u, n_full, n_tt, N, hmask);
                 const int ft = tile / n_tt, tt = tile - ft * n_tt;
                 const int f0 = ft * kBF, t0 = tt * kBT;
                 for (int G = 0; G < ngroup; ++G, ++gs) {
@@ -185,9 +203,9 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
             uint32_t gs = 0;
             int tiles_done = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tiles_done) {
-                const int ft = tile / n_tt;
-                const bool half1 = ft * kBF + 128 < N;
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++tiles_done) {
+                int hmask;
+                unit_tile(u, n_full, n_tt, N, hmask);
                 for (int G = 0; G < ngroup; ++G, ++gs) {
                     const int s = static_cast<int>(gs % kStages), b = static_cast<int>(gs & 1u);
                     if (!mbar_wait(bar(B_FULL0 + s), (gs / kStages) & 1u, abort_flag, kWaitNs) ||
@@ -199,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
                     const uint32_t xa = x_lo0 + ((s * kXStage) >> 4);
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
-                        if (h == 1 && !half1) break;
+                        if (!((hmask >> h) & 1)) continue;
                         // the accumulator of half h is free once the epilogue read the previous tile's
                         if (G == 0 && tiles_done > 0 &&
                             !mbar_wait(bar(B_ACCEMPTY0 + h), static_cast<uint32_t>(tiles_done - 1) & 1u, abort_flag,
@@ -238,11 +256,13 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
         const uint32_t magic = 0x43004300u, mask = 0x000F000Fu;
         uint32_t gs = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+            int hmask;
+            const int tile = unit_tile(u, n_full, n_tt, N, hmask);
             const int ft = tile / n_tt;
             const int f0 = ft * kBF;
             const bool have = f0 + rrow < N;   // this feature exists (N is a multiple of 16)
-            const bool half_on = f0 + 128 * h < N;
+            const bool half_on = (hmask >> h) & 1;
             for (int G = 0; G < ngroup; ++G, ++gs) {
                 const int s = static_cast<int>(gs % kStages), b = static_cast<int>(gs & 1u);
                 bool w_ok = mbar_wait(bar(B_FULL0 + s), (gs / kStages) & 1u, abort_flag, kWaitNs);
@@ -305,7 +325,9 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
         const int fl = q * 32 + lane;
         int tiles_done = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++tiles_done) {
+        for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++tiles_done) {
+            int hmask;
+            const int tile = unit_tile(u, n_full, n_tt, N, hmask);
             const int ft = tile / n_tt, tt = tile - ft * n_tt;
             const int f0 = ft * kBF, t0 = tt * kBT;
             ok = __all_sync(0xFFFFFFFFu,
@@ -315,7 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1) w4_gemm_kernel(const __grid_const
 #pragma unroll 1
             for (int h = 0; h < 2; ++h) {
                 const int n = f0 + 128 * h + fl;
-                if (f0 + 128 * h < N) {
+                if ((hmask >> h) & 1) {
                     // destination of feature n: y, or a part of the split output
                     uint16_t* dst = y;
                     int stride = epi.n0, cc = n;
@@ -427,6 +449,41 @@ PFN_encodeTiled g_encode = nullptr;
 constexpr int kMaxDevices = 64;
 bool g_configured[kMaxDevices] = {};
 
+// How many of the last tiles to cut into halves: the split that minimises the busiest
+// CTA's work as the kernel deals units (unit u to CTA u mod grid), a half counted as 0.6
+// of a tile (the x tile and the MMA issue do not halve).  Cached per (tiles, SMs).
+int tail_halves(long long n_tiles, int sms) {
+    static std::mutex mu;
+    static std::map<std::pair<long long, int>, int> cache;
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        const auto it = cache.find({n_tiles, sms});
+        if (it != cache.end()) return it->second;
+    }
+    int best_x = 0;
+    double best = 1e300;
+    for (int xs = 0; xs <= std::min<long long>(n_tiles, 3LL * sms); ++xs) {
+        const long long units = n_tiles + xs;
+        const long long g = std::min<long long>(units, sms);
+        const long long n_full = n_tiles - xs;
+        // CTA c gets full units c, c+g, ... below n_full and half units from n_full on
+        double worst = 0.0;
+        for (long long c = 0; c < std::min<long long>(g, 2LL * sms); ++c) {
+            const long long nf = c < n_full ? (n_full - 1 - c) / g + 1 : 0;
+            const long long first_h = c >= n_full ? c : c + nf * g;  // its first unit past n_full
+            const long long nh = first_h < units ? (units - 1 - first_h) / g + 1 : 0;
+            worst = std::max(worst, static_cast<double>(nf) + 0.6 * static_cast<double>(nh));
+        }
+        if (worst < best - 1e-9) {
+            best = worst;
+            best_x = xs;
+        }
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    cache[{n_tiles, sms}] = best_x;
+    return best_x;
+}
+
 }  // namespace
 
 cudaError_t launch_rmsnorm_rows(const uint16_t* x, const uint16_t* gamma, float eps, int T, int K, uint16_t* xn,
@@ -497,10 +554,13 @@ cudaError_t launch_w4_gemm(const uint8_t* tiles, const uint16_t* x, int T, int N
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
     const long long n_tiles = static_cast<long long>((T + kBT - 1) / kBT) * ((N + kBF - 1) / kBF);
-    const unsigned grid = static_cast<unsigned>(std::min<long long>(n_tiles, sms));
+    if (n_tiles > (1LL << 29)) return cudaErrorInvalidValue;
+    const int best_x = tail_halves(n_tiles, sms);
+    const int n_full = static_cast<int>(n_tiles - best_x), n_units = static_cast<int>(n_tiles + best_x);
+    const unsigned grid = static_cast<unsigned>(std::min<long long>(n_units, sms));
     W4GemmEpi epi = {N, N, nullptr, nullptr, nullptr};
     if (epi_in != nullptr) epi = *epi_in;
-    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, map_wc, map_ws, T, N, K, y, err, epi);
+    w4_gemm_kernel<<<grid, kThreads, L::ALLOC, st>>>(map, map_wc, map_ws, n_full, n_units, T, N, K, y, err, epi);
     return cudaGetLastError();
 }
 
