@@ -38,7 +38,7 @@
  * context owns only its own device memory: the RoPE tables (2 x max_len x
  * head_dim/2 floats, held twice: position-major and pair-major), the decode
  * split-KV partials (batch x n_q_heads x 256 x (head_dim + 2) floats) and counters
- * (2 x batch x n_kv_heads x 16 ints: one set per column group of the multi-token
+ * (5 x batch x n_kv_heads x 16 + 1 ints: one set per column group of the multi-token
  * decode), the prefill partials of split work (SM count x 256 x (head_dim + 2)
  * floats), the q, k, v and attention output of one decode block (attn_decode_layer)
  * and a device error word; all allocated by attn_create
@@ -268,8 +268,8 @@ int attn_timing_read(attn_ctx* ctx, double* ms, long long* launches);
  *     back (it receives the ATTN_DEVERR_* bits, as attn_device_error reports);
  *   - the split-KV partials live in a static device array of
  *     ATTN_NOALLOC_SCRATCH_FLOATS floats (4 MiB) that every GPU which loads this
- *     library holds until the process exits, beside 32768 int counters
- *     (128 KiB).  Shapes whose partials do not fit even with one split
+ *     library holds until the process exits, beside 40961 int counters
+ *     (160 KiB).  Shapes whose partials do not fit even with one split
  *     (batch * n_q_heads * (head_dim + 2) > that size) are rejected with
  *     ATTN_EINVAL; larger ones use fewer splits.
  * All calls share those arrays.  Nothing in the partials has to start at zero

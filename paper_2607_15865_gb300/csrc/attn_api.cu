@@ -260,7 +260,8 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
     oom |= cudaMalloc(&c->d_lv, kd * sizeof(uint16_t)) != cudaSuccess;
     oom |= cudaMalloc(&c->d_lo, qd * sizeof(uint16_t)) != cudaSuccess;
     // merge counts and tile claims per (sequence, kv head, column group of the multi-token decode)
-    const size_t n_counters = 2 * static_cast<size_t>(cfg->batch) * cfg->n_kv_heads * kMaxColumnGroups;
+    const size_t n_counters = static_cast<size_t>(
+        attn::decode_tc_counter_ints(static_cast<long long>(cfg->batch) * cfg->n_kv_heads * kMaxColumnGroups));
     oom |= cudaMalloc(&c->d_counters, n_counters * sizeof(int)) != cudaSuccess;
     if (oom) {
         cudaGetLastError();
@@ -360,7 +361,7 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
         if (tc)
             return attn::launch_decode_tc(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                           c->d_sin, c->d_part_o, c->d_part_ml, c->d_counters, nsplit, out,
-                                          c->d_err, after_decode, ntok, st, producer_early, c->wait_ns);
+                                          c->d_err, after_decode, ntok, st, producer_early, c->wait_ns, c->num_sms);
         return attn::launch_decode_split(c->shape, c->dec_maps, q, k, v, d_hist_len, hist_add, k_cache, v_cache, c->d_cos,
                                          c->d_sin, c->d_part_o, c->d_part_ml, nsplit, c->d_err, st, c->wait_ns);
     });

@@ -32,11 +32,11 @@ namespace {
 // Split-KV partials of attn_decode_noalloc: [B*Hq*nsplit*D] accumulators followed by
 // [B*Hq*nsplit*2] (max, sum) pairs.  Shared by every call on the device.
 static __device__ __align__(256) float g_noalloc_scratch[ATTN_NOALLOC_SCRATCH_FLOATS];
-// Counters of the tensor-core decode, two per (sequence, kv head) (merge count, tile
-// claims); zero at load and left zero by every launch.  B*Hkv <= B*Hq <=
-// scratch / (D + 2) < 16384.
-constexpr int kNoallocCounters = 16384;
-static __device__ int g_noalloc_counters[2 * kNoallocCounters] = {0};
+// Counters of the tensor-core decode for up to kNoallocCounters (sequence, kv head) items
+// (decode_tc_counter_ints of them); zero at load and left zero by every launch.
+// B*Hkv <= B*Hq <= scratch / (D + 2) < 8192.
+constexpr int kNoallocCounters = 8192;
+static __device__ __align__(16) int g_noalloc_counters[5 * kNoallocCounters + 1] = {0};
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
@@ -144,7 +144,8 @@ extern "C" int attn_decode_noalloc(const attn_cfg* cfg, const float* d_cos, cons
     const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (tc && static_cast<long long>(cfg->batch) * cfg->n_kv_heads > kNoallocCounters) return ATTN_EINVAL;
     cudaError_t e = tc ? attn::launch_decode_tc(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin, part_o,
-                                                part_ml, counters, nsplit, out, d_err, false, 1, st)
+                                                part_ml, counters, nsplit, out, d_err, false, 1, st, false,
+                                                attn::kWaitLimitNs, num_sms)
                        : attn::launch_decode_split(s, maps, q, k, v, d_hist_len, 0, k_cache, v_cache, d_cos, d_sin,
                                                    part_o, part_ml, nsplit, d_err, st);
     if (e == cudaSuccess && !tc) e = attn::launch_decode_combine(s, d_hist_len, 0, part_o, part_ml, nsplit, out, st);

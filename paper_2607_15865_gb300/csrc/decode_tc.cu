@@ -14,9 +14,11 @@
 //   S^T [128 keys x 16] = K_tile [128 x D] . Q^T       (Q: C columns, zero-padded to 16)
 //   O^T [D x 16]      += V_tile^T [D x 128] . P^T [128 x 16]
 // Both accumulate in TMEM.  The T = ceil((p+ntok)/128) key tiles of a sequence are
-// claimed by the nsplit CTAs of (b, kv head): split s starts with tile s, then takes
-// tickets from a per-(b, kv head) counter, so CTAs that stream faster take more tiles
-// and no CTA loads keys that another one owns.
+// claimed by the nsplit CTAs of its item (b, kv head, column group): in a one-wave grid
+// split s starts with tile s, in a larger one only split 0 has a fixed first tile; every
+// other tile is a ticket from the item's counter, so CTAs that stream faster take more
+// tiles, splits dispatched late help the items that still have tiles, and no CTA loads
+// keys that another one owns.
 // 192 threads:
 //   warps 0-3  one thread per key of the tile: scores from TMEM, masking, P^T (bf16)
 //              into shared memory, per-thread partial row sums.  The running max m
@@ -33,10 +35,10 @@
 //              copies of the tiles that hold those slots (zeroing the V rows past the
 //              last new slot: slots past it may hold anything, and 0 * NaN would poison
 //              O), so the MMA itself produces the new keys' scores.
-// Merge: with one working split (splits past the sequence's T tiles get none) the CTA
-// writes the normalised output.  Otherwise each working CTA writes its partial
-// (m, l, acc[D]) per column; the last of them to finish (a device counter, reset by
-// that CTA) merges them:
+// Merge: a split that took all T tiles writes the normalised output.  Otherwise each
+// split that took tiles writes its partial (m, l, acc[D]) per column to a slot it took
+// from a counter, then adds (1 contributor, its tile count) to the item's done word; the
+// split whose addition completes T tiles merges the slots:
 //   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its copies
 // and MMAs finish, releases TMEM and still takes part in the merge count.
@@ -84,7 +86,9 @@ struct L {
     static constexpr int OFF_TMEM = OFF_BAR + NBAR * 8;
     static constexpr int OFF_ABORT = OFF_TMEM + 4;
     static constexpr int OFF_LAST = OFF_ABORT + 4;
-    static constexpr int OFF_CROW = OFF_LAST + 8;  // size_t [16]: partial row (split 0) of column c
+    // int [8] at OFF_LAST: merge flag, merged slots, this CTA's partial slot, tiles it
+    // claimed, a helper split's first ticket
+    static constexpr int OFF_CROW = OFF_LAST + 32;  // size_t [16]: partial row (slot 0) of column c
     static constexpr int OFF_OROW = OFF_CROW + NH * 8;  // size_t [16]: q / out row of column c
     static constexpr int BYTES = OFF_OROW + NH * 8;
     static constexpr int ALLOC = BYTES + 1024;
@@ -198,7 +202,9 @@ __device__ __forceinline__ bool halving_leader(int lane) {
 // columns (G * ntok > 16) the grid's z dimension is (sequence, column group): every column
 // group streams the same key tiles, which its sibling CTAs read at about the same time, so
 // the repeats come from L2.
-template <int NHP, int MAXTOK>
+// WAVES: the grid is several waves (s0 < nsplit); its own instantiation, so that a one-wave
+// launch runs code without the helper splits, slot and visit counters and staging.
+template <int NHP, int MAXTOK, bool WAVES>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
@@ -206,7 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     uint16_t* __restrict__ v_cache, const float* __restrict__ cos_tab, const float* __restrict__ sin_tab, int Hq, int Hkv,
     int max_len, int nsplit,
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
-    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg, int spec) {
+    uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg, int spec,
+    int s0) {
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -220,10 +227,16 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const int G = Hq / Hkv;
     // Columns: global column c = token c / G, head h0 + c % G, of G * ntok; this CTA takes the
     // 16-column group cg, columns c0 .. c0 + C - 1 (its local column h is global column c0 + h).
-    const int s = blockIdx.x;
-    const int g = blockIdx.y;
-    const int b = static_cast<int>(blockIdx.z) / ncg;
-    const int cg = static_cast<int>(blockIdx.z) - b * ncg;
+    // Grid (split, kv head, sequence x column group) for one wave; for several waves (s0 <
+    // nsplit) (kv head, sequence x column group, split), so that every item's split 0 is
+    // dispatched before any split 1, and so on: the later splits start as SMs free up and
+    // help the items that still have tiles.
+    constexpr bool wave_grid = WAVES;
+    const int s = wave_grid ? blockIdx.z : blockIdx.x;
+    const int g = wave_grid ? blockIdx.x : blockIdx.y;
+    const int bz = static_cast<int>(wave_grid ? blockIdx.y : blockIdx.z);
+    const int b = bz / ncg;
+    const int cg = bz - b * ncg;
     const int c0 = cg * NH;
     const int C = min(NH, G * ntok - c0);
     const int h0 = g * G;
@@ -235,12 +248,54 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     // dependents start only once its own predecessors are complete).
     const int hist = decode_hist(d_hist, b, hist_add);  // in flight while the barriers and TMEM are set up
     const int kv_row = b * Hkv + g;
+    const bool multi = nsplit > 1;
+    // Several waves (s0 < nsplit): helper splits may claim after their item is merged, so
+    // slots are taken from a counter and every split records its visit; in one wave the
+    // splits with tiles are exactly s < min(nsplit, T), each using slot s.
+    const bool waves = WAVES && multi;
+    int* lastv = reinterpret_cast<int*>(gb + L::OFF_LAST);  // [0] merge flag [1] slots [2] slot [3] claimed
+    const int n_items = static_cast<int>(wave_grid ? gridDim.x * gridDim.y : gridDim.y * gridDim.z);
+    // Counters of this item (sequence, kv head, column group): tile claims, partial slots and
+    // visits (ints, then 64-bit (contributors << 32 | tiles done) words from an even offset);
+    // all zero between launches: the last split to visit resets the first three, the merging
+    // split the fourth.
+    const int ctr_row = kv_row * ncg + cg;
+    int* claim_ctr = counters + ctr_row;
+    int* slot_ctr = counters + n_items + ctr_row;
+    int* visit_ctr = counters + 2 * n_items + ctr_row;
+    unsigned long long* done_ctr = reinterpret_cast<unsigned long long*>(counters + ((3 * n_items + 1) & ~1)) + ctr_row;
+    // A helper split (s >= s0: a grid of several waves) first asks its item's counter for a
+    // tile.  If none is left -- the item is done, or its tiles are all taken -- the CTA
+    // records its visit and leaves before any set-up.  (After the previous decode step it
+    // touches the counters only once that step is complete.)
+    int first_ticket = 0;
+    if (WAVES && multi && s >= s0) {
+        if (tid == 0) {
+            if (producer_early == 0) griddep_wait();
+            int t = -1;
+            if (hist >= 0 && hist <= max_len - ntok) {
+                t = s0 + atomicAdd(claim_ctr, 1);
+                if (t >= (hist + ntok + KT - 1) / KT) {
+                    t = -1;
+                    if (atomicAdd(visit_ctr, 1) == nsplit - 1) {
+                        *claim_ctr = 0;
+                        *slot_ctr = 0;
+                        *visit_ctr = 0;
+                    }
+                }
+            }
+            lastv[4] = t;
+        }
+        __syncthreads();
+        first_ticket = lastv[4];
+        if (first_ticket < 0) return;  // (a skipped sequence also leaves here, touching nothing)
+    }
     // The producer sets up the barriers and, unless the previous kernel may have written the
     // cache (a decode step right after another, spec = 0), issues the copies of its first
     // tile, tile s, before the length is known: the K slot's arrival is held back until the
     // producer knows whether tile s holds keys of the sequence (the copies read in-range
     // slots or the map's zero fill either way; a tile past the sequence is not used).
-    const bool spec_first = spec != 0 && s * KT < max_len;
+    const bool spec_first = spec != 0 && s < s0 && s * KT < max_len;
     if (warp == kWarpTma && lane == 0) {
         *abort_flag = 0;
         mbar_init(bar(B_QREADY), 128);
@@ -306,14 +361,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     if (!hist_ok && s == 0 && g == 0 && cg == 0 && tid == 0) atomicOr(err, kDevErrHistRange);
     const int nkeys = hist + ntok;        // slots [0, hist) and the new tokens' [hist, hist + ntok)
     const int T = (nkeys + KT - 1) / KT;  // key tiles of the sequence; tile T-1 holds the last new slot
-    // Splits s < T each take at least tile s; splits past T get no tile, write nothing and
-    // stay out of the merge, which combines the n_work = min(nsplit, T) working splits.
-    const bool working = s < T;
-    const int n_work = min(nsplit, T);
-    const int ctr_row = kv_row * ncg + cg;  // counters of this (sequence, kv head, column group)
+    // Splits s < s0 start with tile s; every other tile is claimed from the item's counter
+    // (tickets s0, s0 + 1, ...).  A split that gets no tile writes nothing.
     // Rows of column c (token c / G, head h0 + c % G), tabulated once in the prologue:
-    // q / out row (b * ntok + c / G) * Hq + h0 + c % G, and partial row of split 0 that
-    // times nsplit (split sp adds sp).  Columns past C repeat column C - 1.
+    // q / out row (b * ntok + c / G) * Hq + h0 + c % G, and partial row of slot 0 that
+    // times nsplit (slot sp adds sp).  Columns past C repeat column C - 1.
     const size_t* crow = reinterpret_cast<const size_t*>(gb + L::OFF_CROW);
     const size_t* orow = reinterpret_cast<const size_t*>(gb + L::OFF_OROW);
     int* meta = reinterpret_cast<int*>(gb + L::OFF_META);  // tile index of local tile j at [j % 8]; -1 ends
@@ -327,17 +379,30 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
         }
     } else if (warp == kWarpTma) {
         // ------------------------------------------------------------ TMA producer (lane 0)
-        // Tiles are claimed, not fixed: split s starts with tile s, then takes tickets
-        // nsplit, nsplit+1, ... from the (sequence, kv head)'s tile counter until they run
-        // past T, so CTAs that stream faster take more tiles.  The next ticket is claimed
-        // while the current tile's copies are issued.  One thread feeds both rings: the
-        // V slot of tile j frees (PV(j-4) done) before the K slot does (S(j-2) done).
+        // Tiles are claimed, not fixed: split s < s0 starts with tile s, then takes tickets
+        // s0, s0+1, ... from the item's tile counter until they run past T, so CTAs that
+        // stream faster take more tiles and splits that start late find the tiles taken.  The
+        // next ticket is claimed while the current tile's copies are issued.  A split that
+        // gets a tile takes a partial slot; every split records its visit once its claims are
+        // over.  One thread feeds both rings: the V slot of tile j frees (PV(j-4) done)
+        // before the K slot does (S(j-2) done).
         if (lane == 0) {
-            int* tile_ctr = counters + gridDim.y * gridDim.z + ctr_row;
-            int cur = s < T ? s : T;
-            int nxt = (n_work > 1 && cur < T) ? nsplit + atomicAdd(tile_ctr, 1) : cur + 1;
+            // (one wave with a single split that has tiles: it walks them in order, touching
+            // no counter, as does the only split of an item)
+            const bool claims = waves || (multi && min(nsplit, T) > 1);
+            auto take = [&]() { return s0 + atomicAdd(claim_ctr, 1); };
+            int cur = !multi ? 0 : (s < s0 ? min(s, T) : first_ticket);
+            int claimed = cur < T ? 1 : 0;
+            int nxt = !claims ? cur + 1 : (cur < T ? take() : T);
             int issued_k = 0, issued_v = 0;
             bool ok = true;
+            auto advance = [&]() {
+                cur = nxt;
+                if (cur < T) {
+                    ++claimed;
+                    nxt = claims ? take() : cur + 1;
+                }
+            };
             for (int j = 0;; ++j) {
                 const int tile = cur < T ? cur : -1;
                 const int ks = j % KST, vs = j % VST;
@@ -354,12 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                         mbar_wait(bar(B_VFULL0), 0u, nullptr);
                         break;
                     }
-                    cur = nxt;
-                    if (n_work > 1) {
-                        if (cur < T) nxt = nsplit + atomicAdd(tile_ctr, 1);
-                    } else {
-                        nxt = cur + 1;
-                    }
+                    advance();
                     continue;
                 }
                 if (tile < 0) {  // no more tiles: complete the K slot's phase without data
@@ -382,12 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     tma_load_3d(base + L::OFF_V + vs * L::TILE + c * L::BOX, &map_v, c * 64, tile * KT, kv_row,
                                 bar(B_VFULL0 + vs));
                 issued_v = j + 1;
-                cur = nxt;
-                if (n_work > 1) {
-                    if (cur < T) nxt = nsplit + atomicAdd(tile_ctr, 1);
-                } else {
-                    nxt = cur + 1;
-                }
+                advance();
             }
             if (!ok) {
                 *abort_flag = 1;
@@ -396,6 +451,22 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     mbar_wait(bar(B_KFULL0 + t % KST), static_cast<uint32_t>(t / KST) & 1u, nullptr);
                 for (int t = max(0, issued_v - VST); t < issued_v; ++t)
                     mbar_wait(bar(B_VFULL0 + t % VST), static_cast<uint32_t>(t / VST) & 1u, nullptr);
+                if (claims) {
+                    // take every ticket still unclaimed (and count it, unprocessed), so that the
+                    // item's tiles are all accounted for and its merge and reset still happen
+                    const int first = s0 + atomicAdd(claim_ctr, T);
+                    if (first < T) claimed += T - first;
+                }
+            }
+            // a partial slot for a split with tiles, taken before its visit (read after the CTA
+            // barrier of the merge, as is the claim count)
+            lastv[2] = waves && claimed > 0 ? atomicAdd(slot_ctr, 1) : s;
+            lastv[3] = claimed;
+            if (waves && atomicAdd(visit_ctr, 1) == nsplit - 1) {
+                // every split of the item has made its last claim: reset for the next launch
+                *claim_ctr = 0;
+                *slot_ctr = 0;
+                *visit_ctr = 0;
             }
         }
         if (early) griddep_wait();
@@ -656,12 +727,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             tc_fence_before();
             mbar_arrive(bar(B_PFULL0 + (j & 1)));
         }
-        if (ok && n == 0) {
-            if (working && n_work > 1 && t < C) {  // (not reached: a working split has tile s)
-                part_ml[(crow[t] + s) * 2 + 0] = -INFINITY;
-                part_ml[(crow[t] + s) * 2 + 1] = 0.f;
-            }
-        } else if (ok) {
+        if (ok && n > 0) {
             // (PVDONE could be two phases behind here -- PV(n-2) may still run -- so the
             // epilogue waits on its own barrier, committed once after the last PV.)
             ok = !named_or_128(!mbar_wait(bar(B_OFULL), 0u, abort_flag, wait_ns));
@@ -675,20 +741,26 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             tmem_ld_cols<NHP>(tmem + lane_base + TM_O, o);  // thread t = output dimension d
             tmem_wait_ld();
             named_sync_128();
+            // the output (one split with tiles), the partial (m, l, acc) at slot s (one wave),
+            // or, for several waves, (m, l, acc) staged in the idle V ring and written out
+            // below once the producer has taken this CTA's partial slot
+            float* st_o = reinterpret_cast<float*>(gb + L::OFF_V);
+            float2* st_ml = reinterpret_cast<float2*>(gb + L::OFF_V + NH * D * 4);
+            const bool alone = !multi || (!waves && T == 1);
 #pragma unroll
             for (int h = 0; h < NHP; ++h) {
                 if (h < C) {
                     const float4 l4 = reinterpret_cast<const float4*>(ls)[h];
                     const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
-                    if (n_work == 1) {
+                    if (alone) {
                         out[orow[h] * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
-                    } else {
+                    } else if (!waves) {
                         const size_t row = crow[h] + s;
                         part_o[row * D + t] = __uint_as_float(o[h]);
-                        if (t == 0) {
-                            part_ml[row * 2 + 0] = m_run[h];
-                            part_ml[row * 2 + 1] = l_tot;
-                        }
+                        if (t == 0) reinterpret_cast<float2*>(part_ml)[row] = make_float2(m_run[h], l_tot);
+                    } else {
+                        st_o[h * D + t] = __uint_as_float(o[h]);
+                        if (t == 0) st_ml[h] = make_float2(m_run[h], l_tot);
                     }
                 }
             }
@@ -699,23 +771,69 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     }
 
     // ---------------------------------------------------------------- merge of the splits
-    if (hist_ok && n_work > 1 && working) {
-        int* last_flag = reinterpret_cast<int*>(gb + L::OFF_LAST);
-        __threadfence();  // this CTA's partials are visible before it is counted
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0) {
-            int* cnt = counters + ctr_row;
-            const int last = atomicAdd(cnt, 1) == n_work - 1;
-            if (last) {  // every split of this launch has been counted and has claimed its last tile
-                *cnt = 0;
-                counters[gridDim.y * gridDim.z + ctr_row] = 0;
+    if (hist_ok && multi) {
+        bool contrib;  // (uniform over the CTA) this split wrote a partial and takes part
+        if (waves) {
+            tc_fence_before();
+            __syncthreads();  // the staged result, and the producer's slot and claim count
+            const int claimed = lastv[3];
+            const float4* st_o4 = reinterpret_cast<const float4*>(gb + L::OFF_V);
+            const float2* st_ml = reinterpret_cast<const float2*>(gb + L::OFF_V + NH * D * 4);
+            contrib = claimed > 0 && claimed < T;
+            if (claimed == T) {
+                // this split took every tile: normalise straight from the staging
+                for (int p = tid; p < C * (D / 4); p += kThreads) {
+                    const int h = p / (D / 4), c = p % (D / 4);
+                    const float4 v4 = st_o4[h * (D / 4) + c];
+                    const float inv = 1.f / st_ml[h].y;
+                    *reinterpret_cast<uint2*>(out + orow[h] * D + 4 * c) =
+                        make_uint2(to_bf16(v4.x * inv) | (static_cast<uint32_t>(to_bf16(v4.y * inv)) << 16),
+                                   to_bf16(v4.z * inv) | (static_cast<uint32_t>(to_bf16(v4.w * inv)) << 16));
+                }
+            } else if (contrib) {
+                const int slot = lastv[2];
+                for (int p = tid; p < C * (D / 4); p += kThreads) {
+                    const int h = p / (D / 4), c = p % (D / 4);
+                    reinterpret_cast<float4*>(part_o + (crow[h] + slot) * D)[c] = st_o4[h * (D / 4) + c];
+                }
+                if (tid < C) reinterpret_cast<float2*>(part_ml)[crow[tid] + slot] = st_ml[tid];
             }
-            *last_flag = last;
+        } else {
+            contrib = s < T && T > 1;  // one wave: the softmax wrote the partial at slot s
         }
-        __syncthreads();
-        tc_fence_after();
-        if (*last_flag) {
+        if (contrib) {
+            __threadfence();  // this CTA's partials are visible before it is counted
+            tc_fence_before();
+            __syncthreads();
+            if (tid == 0) {
+                // (contributors << 32 | tiles done): the split that completes the item's T tiles
+                // merges, every contributor having counted itself after writing its partial
+                if constexpr (WAVES) {
+                    const int claimed = lastv[3];
+                    const unsigned long long old =
+                        atomicAdd(done_ctr, (1ull << 32) | static_cast<unsigned>(claimed));
+                    const int last = static_cast<int>(old & 0xFFFFFFFFull) + claimed == T;
+                    if (last) *done_ctr = 0ull;
+                    lastv[0] = last;
+                    lastv[1] = static_cast<int>(old >> 32) + 1;
+                } else {
+                    // one wave: the min(nsplit, T) splits with tiles count themselves (in the slot
+                    // counter's place); the last of them merges and resets both counters, every
+                    // claimer having counted itself
+                    const int last = atomicAdd(slot_ctr, 1) == min(nsplit, T) - 1;
+                    if (last) {
+                        *slot_ctr = 0;
+                        *claim_ctr = 0;
+                    }
+                    lastv[0] = last;
+                    lastv[1] = min(nsplit, T);
+                }
+            }
+            __syncthreads();
+            tc_fence_after();
+        }
+        const int n_slots = lastv[1];
+        if (contrib && lastv[0]) {
             // All six warps merge in one pass over the partials: warp w takes splits w, w+6, ...,
             // lane l dimensions 4l .. 4l+3 of every column, and keeps a running (M, L, acc) per
             // column, rescaled as a larger split maximum comes in; then the six warps' results
@@ -737,7 +855,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             // (Every load is issued unconditionally -- padded columns re-read column C-1 --
             // so that the loads of a split for all columns are in flight together.)
 #pragma unroll 2
-            for (int sp = warp; sp < n_work; sp += kThreads / 32) {
+            for (int sp = warp; sp < n_slots; sp += kThreads / 32) {
                 float4 o4[NHP];
                 float2 ml[NHP];
 #pragma unroll
@@ -807,20 +925,27 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
 
 cudaError_t configure_decode_tc() {
     cudaError_t e = cudaSuccess;
-    for (auto fn : {decode_tc_kernel<8, 1>, decode_tc_kernel<16, 1>, decode_tc_kernel<8, kMaxTok>,
-                    decode_tc_kernel<16, kMaxTok>})
+    for (auto fn : {decode_tc_kernel<8, 1, false>, decode_tc_kernel<16, 1, false>, decode_tc_kernel<8, kMaxTok, false>,
+                    decode_tc_kernel<16, kMaxTok, false>, decode_tc_kernel<8, 1, true>, decode_tc_kernel<16, 1, true>,
+                    decode_tc_kernel<8, kMaxTok, true>, decode_tc_kernel<16, kMaxTok, true>})
         if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
     return e;
 }
 
-// One wave of CTAs, one per SM: with fewer (sequence, kv head) items than SMs, each
-// item gets floor(SMs / items) splits; otherwise one split per item.
+// Split counts.  With at most half as many (sequence, kv head, column group) items as SMs,
+// one wave of CTAs, floor(SMs / items) splits per item, each starting with its own tile.
+// With more items, kWaveSplits splits per item over several waves: split 0 of every item
+// comes first and the later splits, dispatched as SMs free up, claim what their items
+// still have (nothing, for an item that is done), so long sequences in a batch of mixed
+// lengths get help once the short ones finish.
+constexpr int kWaveSplits = 3;
+
 int decode_tc_column_groups(int G, int ntok) { return (G * ntok + NH - 1) / NH; }
 
 int decode_tc_num_splits(const Shape& s, int num_sms, int ncg) {
     const long items = static_cast<long>(s.batch) * s.n_kv_heads * ncg;
     const long max_tiles = std::max(1L, static_cast<long>((s.max_len + KT - 1) / KT));
-    long ns = items >= num_sms ? 1 : num_sms / items;
+    long ns = 2 * items > num_sms ? kWaveSplits : num_sms / items;
     ns = std::min(ns, std::min(max_tiles, 256L));
     return static_cast<int>(std::max(1L, ns));
 }
@@ -846,12 +971,17 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              const uint16_t* v_new, const int32_t* d_hist, int hist_add, uint16_t* k_cache,
                              uint16_t* v_cache, const float* cos_tab, const float* sin_tab, float* part_o,
                              float* part_ml, int* counters, int nsplit, uint16_t* out, int* err, bool after_decode,
-                             int ntok, cudaStream_t st, bool producer_early, uint64_t wait_ns) {
+                             int ntok, cudaStream_t st, bool producer_early, uint64_t wait_ns, int num_sms) {
     const float scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(D)));
     const int G = s.n_q_heads / s.n_kv_heads;
     const int ncg = decode_tc_column_groups(G, ntok);
-    const dim3 grid(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads),
-                    static_cast<unsigned>(s.batch * ncg));
+    // every split starts with its own tile when the grid is one wave, else only split 0
+    const long long ctas = static_cast<long long>(s.n_kv_heads) * s.batch * ncg * nsplit;
+    const int s0 = ctas <= num_sms ? nsplit : 1;
+    const dim3 grid = s0 == nsplit ? dim3(static_cast<unsigned>(nsplit), static_cast<unsigned>(s.n_kv_heads),
+                                          static_cast<unsigned>(s.batch * ncg))
+                                   : dim3(static_cast<unsigned>(s.n_kv_heads), static_cast<unsigned>(s.batch * ncg),
+                                          static_cast<unsigned>(nsplit));
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = dim3(kThreads);
@@ -864,12 +994,16 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     // dependent launch only right after another decode step, or with producer_early
     cfg.numAttrs = (after_decode || producer_early) ? 1 : 0;
     if (ntok < 1 || ntok > kMaxTok || G > NH) return cudaErrorInvalidValue;
-    const auto kernel = ntok == 1 ? (G <= 8 ? decode_tc_kernel<8, 1> : decode_tc_kernel<16, 1>)
-                                  : (G * ntok <= 8 ? decode_tc_kernel<8, kMaxTok> : decode_tc_kernel<16, kMaxTok>);
+    const bool w = s0 < nsplit;
+    const auto kernel =
+        ntok == 1 ? (G <= 8 ? (w ? decode_tc_kernel<8, 1, true> : decode_tc_kernel<8, 1, false>)
+                            : (w ? decode_tc_kernel<16, 1, true> : decode_tc_kernel<16, 1, false>))
+                  : (G * ntok <= 8 ? (w ? decode_tc_kernel<8, kMaxTok, true> : decode_tc_kernel<8, kMaxTok, false>)
+                                   : (w ? decode_tc_kernel<16, kMaxTok, true> : decode_tc_kernel<16, kMaxTok, false>));
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
-                              producer_early ? 1 : 0, wait_ns, ncg, after_decode ? 0 : 1);
+                              producer_early ? 1 : 0, wait_ns, ncg, after_decode ? 0 : 1, s0);
 }
 
 }  // namespace attn

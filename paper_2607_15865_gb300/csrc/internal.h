@@ -96,12 +96,13 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
                                 uint16_t* v_cache,
                                 const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                                 int nsplit, int* err, cudaStream_t st, uint64_t wait_ns = kWaitLimitNs);
-// K3 for head_dim 128 on the tensor cores (decode_tc.cu): one CTA per SM, maps with
-// 128-key boxes; same partial layout as launch_decode_split, but the merge is fused
-// in (the last CTA of each (b, kv head) merges and writes `out`), so no K4 follows.
-// Splits claim key tiles from a per-(b, kv head) counter.  `counters`: 2*B*Hkv ints
-// (merge counts, then tile claims) per column group, zero before the first launch; every
-// launch leaves them zero.  1 <= ntok <= 16 new tokens per sequence (q/k/v/out
+// K3 for head_dim 128 on the tensor cores (decode_tc.cu): maps with 128-key boxes; same
+// partial layout as launch_decode_split, but the merge is fused in (the split that
+// completes an item's tiles merges and writes `out`), so no K4 follows.  Splits claim key
+// tiles from a per-item counter (item: sequence, kv head, column group).  `counters`:
+// decode_tc_counter_ints(items) ints, zero before the first launch; every launch leaves
+// them zero.  num_sms: whether the grid fits one wave.  1 <= ntok <= 16 new tokens per
+// sequence (q/k/v/out
 // [B, ntok, H, D]) at positions d_hist[b] + hist_add + i, token i attending causally to
 // slots [0, that position]; the partials need B * ntok * Hq * nsplit rows.
 // after_decode: the stream's previous kernel is a decode_tc launch (the
@@ -112,8 +113,11 @@ cudaError_t launch_decode_split(const Shape& s, const DecodeMaps& maps, const ui
 // neither the caches, the lengths nor the counters); the K/V stream starts before the wait.
 cudaError_t configure_decode_tc();
 // Column groups of 16 (query head, new token) columns one launch runs for ntok new tokens
-// per sequence: ceil(G * ntok / 16); the counters need 2 * B * Hkv * that many ints.
+// per sequence: ceil(G * ntok / 16); items = B * Hkv * that many.
 int decode_tc_column_groups(int G, int ntok);
+// Ints of the counter array for `items` items: claims, slots and visits, then 64-bit
+// (contributors, tiles done) words from an even offset.
+inline long long decode_tc_counter_ints(long long items) { return 3 * items + 1 + 2 * items; }
 int decode_tc_num_splits(const Shape& s, int num_sms, int ncg = 1);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                                 const uint16_t* v_cache, DecodeMaps* maps);
@@ -122,7 +126,7 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
                              uint16_t* v_cache,
                              const float* cos_tab, const float* sin_tab, float* part_o, float* part_ml,
                              int* counters, int nsplit, uint16_t* out, int* err, bool after_decode, int ntok,
-                             cudaStream_t st, bool producer_early = false, uint64_t wait_ns = kWaitLimitNs);
+                             cudaStream_t st, bool producer_early, uint64_t wait_ns, int num_sms);
 cudaError_t launch_decode_combine(const Shape& s, const int32_t* d_hist, int hist_add, const float* part_o,
                                   const float* part_ml, int nsplit, uint16_t* out, cudaStream_t st);
 

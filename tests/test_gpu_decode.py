@@ -111,6 +111,61 @@ def test_decode_out_of_range_length_sets_error_and_skips(torch):
     assert_out_close(out[:1], ref, "valid sequence next to invalid ones")
 
 
+# More (sequence, kv head) items than half the SMs: the grid runs several waves of splits
+# that claim what their items still have (split 0 of every item first).
+MULTIWAVE = [
+    ("b24_g4_lengths_0_to_4095", Shape("mw1", 24, 16, 4, 128, 4096, 1.0e4)),
+    ("b16_g4_lengths_64_to_8191", Shape("mw2", 16, 32, 8, 128, 8192, 5.0e5)),
+]
+
+
+@pytest.mark.parametrize("name,shape", MULTIWAVE, ids=[m[0] for m in MULTIWAVE])
+def test_decode_multiwave_mixed_lengths(torch, name, shape):
+    rng = np.random.default_rng(len(name))
+    lo = 0 if shape.max_len == 4096 else 64
+    hist = rng.integers(lo, shape.max_len, size=shape.batch).astype(np.int32)
+    hist[0], hist[-1] = lo, shape.max_len - 1
+    pick = [(b, 0, h) for b in range(shape.batch) for h in (0, shape.n_q_heads - 1)]
+    pick += [(int(rng.integers(shape.batch)), 0, int(rng.integers(shape.n_q_heads))) for _ in range(48)]
+    check_decode(torch, shape, name, hist, np.array(pick, np.int32))
+
+
+REPEATED = [
+    # several waves of splits (160 items)
+    ("multiwave", Shape("mwrep", 20, 16, 8, 128, 2048, 1.0e4)),
+    # one wave (16 items x 9 splits): single-tile sequences next to ones with more tiles
+    # than splits, so that a call whose item needs no counter precedes one that does
+    ("onewave", Shape("owrep", 2, 16, 8, 128, 4096, 1.0e4)),
+]
+
+
+@pytest.mark.parametrize("name,shape", REPEATED, ids=[r[0] for r in REPEATED])
+def test_decode_repeated_calls_leave_counters_clean(torch, name, shape):
+    """Four calls on one context with different length mixes: the per-item counters
+    (claims, slots, visits, done words) must be back at zero after every launch."""
+    from paper_2607_15865_gb300.attention import Attention
+    attn = Attention.for_shape(shape)
+    rng = np.random.default_rng(5)
+    for i in range(4):
+        hist = rng.integers(0, shape.max_len, size=shape.batch).astype(np.int32)
+        if i == 2:
+            hist[:] = shape.max_len - 1
+        if i % 2 == 0:
+            hist[0] = 17  # one key tile
+        else:
+            hist[0] = shape.max_len - 1 - i
+        q, k, v = w.tokens(shape, f"mwrep_{i}", 1)
+        kc, vc = w.cache(shape, f"mwrep_{i}", int(hist.max()), fill="random")
+        hl = torch.from_numpy(hist).cuda()
+        out = to_host(attn.decode(to_dev(q), to_dev(k), to_dev(v), hl, to_dev(kc), to_dev(vc)))
+        rk, rv = kc.copy(), vc.copy()
+        ref = O.decode(shape, q, k, v, hist, rk, rv)
+        assert_out_close(out, ref, f"{name}: call {i}")
+    torch.cuda.synchronize()
+    assert attn.device_error() == 0
+    attn.close()
+
+
 def test_decode_chain_reuses_merge_state(torch):
     """Consecutive decode steps on one context and one cache: each step appends its
     token and attends to the previous steps' tokens; tile boundaries (128, 256) and
