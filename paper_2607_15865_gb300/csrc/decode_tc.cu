@@ -266,25 +266,44 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     unsigned long long* done_ctr = reinterpret_cast<unsigned long long*>(counters + ((3 * n_items + 1) & ~1)) + ctr_row;
     // A helper split (s >= s0: a grid of several waves) first asks its item's counter for a
     // tile.  If none is left -- the item is done, or its tiles are all taken -- the CTA
-    // records its visit and leaves before any set-up.  (After the previous decode step it
-    // touches the counters only once that step is complete.)
+    // records its visit and leaves before any set-up.  When the batch's lengths are within
+    // 10% of each other (read by one warp, batches of up to 1024) there is nothing to even
+    // out, and helpers leave without asking: the splits 0 then finish their items alone and
+    // write the outputs without a merge.  (After the previous decode step the counters are
+    // touched only once that step is complete.)
     int first_ticket = 0;
     if (WAVES && multi && s >= s0) {
-        if (tid == 0) {
+        if (warp == 0) {
             if (producer_early == 0) griddep_wait();
-            int t = -1;
-            if (hist >= 0 && hist <= max_len - ntok) {
-                t = s0 + atomicAdd(claim_ctr, 1);
-                if (t >= (hist + ntok + KT - 1) / KT) {
-                    t = -1;
-                    if (atomicAdd(visit_ctr, 1) == nsplit - 1) {
+            const int batch = static_cast<int>(gridDim.y) / ncg;
+            int tmax = 0, tsum = 0;
+            if (batch <= 1024) {
+                for (int bb = lane; bb < batch; bb += 32) {
+                    const int hb = decode_hist(d_hist, bb, hist_add);
+                    const int tb = hb >= 0 && hb <= max_len - ntok ? (hb + ntok + KT - 1) / KT : 0;
+                    tmax = max(tmax, tb);
+                    tsum += tb;
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) {
+                    tmax = max(tmax, __shfl_xor_sync(0xFFFFFFFFu, tmax, off));
+                    tsum += __shfl_xor_sync(0xFFFFFFFFu, tsum, off);
+                }
+            }
+            const bool even = batch <= 1024 && 10LL * tmax * batch <= 11LL * tsum;
+            if (lane == 0) {
+                int t = -1;
+                if (hist >= 0 && hist <= max_len - ntok) {
+                    if (!even) t = s0 + atomicAdd(claim_ctr, 1);
+                    if (t >= (hist + ntok + KT - 1) / KT) t = -1;
+                    if (t < 0 && atomicAdd(visit_ctr, 1) == nsplit - 1) {
                         *claim_ctr = 0;
                         *slot_ctr = 0;
                         *visit_ctr = 0;
                     }
                 }
+                lastv[4] = t;
             }
-            lastv[4] = t;
         }
         __syncthreads();
         first_ticket = lastv[4];
