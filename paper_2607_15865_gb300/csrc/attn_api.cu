@@ -174,7 +174,8 @@ int run_prefill(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_
         if (rc != ATTN_OK) return rc;
     }
     cudaError_t e = timed(c, ATTN_KERNEL_ROPE_APPEND, st, [&](int*) {
-        return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, seq_stride, c->d_cos, c->d_sin, kc, vc, c->d_err,
+        return attn::launch_rope_append(s, k, v, hist, nullptr, chunk, seq_stride, c->d_cos, c->d_sin, c->d_cos_t,
+                                        c->d_sin_t, kc, vc, c->d_err,
                                         st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "rope_append launch");

@@ -54,9 +54,12 @@ __device__ __forceinline__ int fdiv(int n, const FastDiv& f) {
 // k and v into cache slots hist+i (Listing 2 "Concat"; Section 4.6.3).
 // hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.  k and v
 // hold `chunk` tokens of each sequence, sequence b starting at token b * seq_stride.
+// cos_t / sin_t (the pair-major table copies, or null): their lines for the chunk's
+// positions are prefetched into L2 for K2's rotation of q.
 cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
                                const int32_t* d_hist, int chunk, int seq_stride, const float* cos_tab,
-                               const float* sin_tab, uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st);
+                               const float* sin_tab, const float* cos_t, const float* sin_t, uint16_t* k_cache,
+                               uint16_t* v_cache, int* err, cudaStream_t st);
 
 // K2: causal flash attention of `chunk` new queries at positions hist.. over cache
 // slots [0, hist+chunk) (prefill: hist=0).  RoPE of q is applied in the kernel.

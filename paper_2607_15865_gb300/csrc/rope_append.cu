@@ -34,6 +34,7 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
                                                           int seq_stride, int Hkv,
                                                           int max_len, const float* __restrict__ cos_tab,
                                                           const float* __restrict__ sin_tab,
+                                                          const float* __restrict__ cos_t, const float* __restrict__ sin_t,
                                                           uint16_t* __restrict__ k_cache,
                                                           uint16_t* __restrict__ v_cache, int* __restrict__ err) {
     constexpr int HALF = D / 2;
@@ -53,6 +54,14 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
         }
     }
     const int p = h0 + i;
+    // Warm L2 with the lines of the pair-major tables (cos_t, sin_t: [D/2][max_len]) that the
+    // attention kernel's softmax threads read to rotate the q rows of this chunk: the CTA of
+    // every 32nd position (and the first) touches one line per pair and table.
+    if (cos_t != nullptr && b == 0 && threadIdx.x < 2 * HALF && (i == 0 || (p & 31) == 0)) {
+        const float* tab = threadIdx.x < HALF ? cos_t : sin_t;
+        const int j = static_cast<int>(threadIdx.x) % HALF;
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + static_cast<size_t>(j) * max_len + (p & ~31)));
+    }
     const int n_rope = Hkv * ROPE_UNITS;
     const int n_units = n_rope + Hkv * COPY_UNITS;
     for (int u = threadIdx.x; u < n_units; u += blockDim.x) {
@@ -102,14 +111,15 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
 
 cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
                                const int32_t* d_hist, int chunk, int seq_stride, const float* cos_tab,
-                               const float* sin_tab, uint16_t* k_cache, uint16_t* v_cache, int* err, cudaStream_t st) {
+                               const float* sin_tab, const float* cos_t, const float* sin_t, uint16_t* k_cache,
+                               uint16_t* v_cache, int* err, cudaStream_t st) {
     const dim3 grid(static_cast<unsigned>(chunk), static_cast<unsigned>(s.batch));
     if (s.head_dim == 128)
         rope_append_kernel<128><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, seq_stride, s.n_kv_heads, s.max_len, cos_tab,
-                                                      sin_tab, k_cache, v_cache, err);
+                                                      sin_tab, cos_t, sin_t, k_cache, v_cache, err);
     else
         rope_append_kernel<64><<<grid, 128, 0, st>>>(k, v, hist, d_hist, chunk, seq_stride, s.n_kv_heads, s.max_len, cos_tab,
-                                                     sin_tab, k_cache, v_cache, err);
+                                                     sin_tab, cos_t, sin_t, k_cache, v_cache, err);
     return cudaGetLastError();
 }
 
