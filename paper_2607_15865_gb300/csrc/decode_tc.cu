@@ -952,19 +952,24 @@ cudaError_t configure_decode_tc() {
 }
 
 // Split counts.  With at most half as many (sequence, kv head, column group) items as SMs,
-// one wave of CTAs, floor(SMs / items) splits per item, each starting with its own tile.
+// one wave of CTAs, min(16, floor(SMs / items)) splits per item, each starting with its own
+// tile.
 // With more items, kWaveSplits splits per item over several waves: split 0 of every item
 // comes first and the later splits, dispatched as SMs free up, claim what their items
 // still have (nothing, for an item that is done), so long sequences in a batch of mixed
 // lengths get help once the short ones finish.
 constexpr int kWaveSplits = 3;
+// One wave: at most 16 splits per item.  The long decode (8 items) measured 29.5 us with 16
+// splits, 30.4-30.8 us with 19 (one per SM), 32.5 with 12 and 42 with 8: past 16 the extra
+// partials and the later last CTA cost more than the SMs add.
+constexpr long kMaxWaveSplits1 = 16;
 
 int decode_tc_column_groups(int G, int ntok) { return (G * ntok + NH - 1) / NH; }
 
 int decode_tc_num_splits(const Shape& s, int num_sms, int ncg) {
     const long items = static_cast<long>(s.batch) * s.n_kv_heads * ncg;
     const long max_tiles = std::max(1L, static_cast<long>((s.max_len + KT - 1) / KT));
-    long ns = 2 * items > num_sms ? kWaveSplits : num_sms / items;
+    long ns = 2 * items > num_sms ? kWaveSplits : std::min<long>(kMaxWaveSplits1, num_sms / items);
     ns = std::min(ns, std::min(max_tiles, 256L));
     return static_cast<int>(std::max(1L, ns));
 }
