@@ -202,9 +202,14 @@ __device__ __forceinline__ bool halving_leader(int lane) {
 // columns (G * ntok > 16) the grid's z dimension is (sequence, column group): every column
 // group streams the same key tiles, which its sibling CTAs read at about the same time, so
 // the repeats come from L2.
-// WAVES: the grid is several waves (s0 < nsplit); its own instantiation, so that a one-wave
-// launch runs code without the helper splits, slot and visit counters and staging.
-template <int NHP, int MAXTOK, bool WAVES>
+// MODE: how the splits of an item meet.  kModeGlobal (one wave): each split with tiles
+// writes its partial (m, l, acc) at slot s in global memory and the last of them merges;
+// kModeCluster (one wave): the item's splits are one thread-block cluster and merge through
+// distributed shared memory; kModeWaves: the grid is several waves (s0 < nsplit), with
+// helper splits and slot and visit counters.  Each is its own instantiation, so that a
+// launch runs only the code of its mode.
+constexpr int kModeGlobal = 0, kModeCluster = 1, kModeWaves = 2;
+template <int NHP, int MAXTOK, int MODE>
 __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
     const uint16_t* __restrict__ q, const uint16_t* __restrict__ k_new, const uint16_t* __restrict__ v_new,
@@ -214,6 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     float scale_log2, float* __restrict__ part_o, float* __restrict__ part_ml, int* __restrict__ counters,
     uint16_t* __restrict__ out, int* __restrict__ err, int producer_early, uint64_t wait_ns, int ncg, int spec,
     int s0) {
+    constexpr bool WAVES = MODE == kModeWaves;
     constexpr int HALF = D / 2;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
@@ -760,9 +766,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
             tmem_ld_cols<NHP>(tmem + lane_base + TM_O, o);  // thread t = output dimension d
             tmem_wait_ld();
             named_sync_128();
-            // the output (one split with tiles), the partial (m, l, acc) at slot s (one wave),
-            // or, for several waves, (m, l, acc) staged in the idle V ring and written out
-            // below once the producer has taken this CTA's partial slot
+            // the output (one split with tiles), the partial (m, l, acc) at slot s (global
+            // merge), or (m, l, acc) staged in the idle V ring: read by the cluster's merge, or
+            // written out below once the producer has taken this CTA's partial slot (waves)
             float* st_o = reinterpret_cast<float*>(gb + L::OFF_V);
             float2* st_ml = reinterpret_cast<float2*>(gb + L::OFF_V + NH * D * 4);
             const bool alone = !multi || (!waves && T == 1);
@@ -773,7 +779,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
                     const float l_tot = (l4.x + l4.y) + (l4.z + l4.w);
                     if (alone) {
                         out[orow[h] * D + t] = to_bf16(__uint_as_float(o[h]) / l_tot);
-                    } else if (!waves) {
+                    } else if constexpr (MODE == kModeGlobal) {
                         const size_t row = crow[h] + s;
                         part_o[row * D + t] = __uint_as_float(o[h]);
                         if (t == 0) reinterpret_cast<float2*>(part_ml)[row] = make_float2(m_run[h], l_tot);
@@ -790,9 +796,53 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
     }
 
     // ---------------------------------------------------------------- merge of the splits
-    if (hist_ok && multi) {
+    if constexpr (MODE == kModeCluster) {
+        // The nsplit CTAs of an item form a thread-block cluster (rank = split s).
+        // The splits with tiles (s < min(nsplit, T)) have staged (m, l, acc) in shared
+        // memory; after a cluster barrier every CTA merges its share of the dimensions,
+        // reading its peers' staging directly, then waits at a second barrier until its own
+        // staging has been read.  (T is the same in every CTA of the cluster, so all or none
+        // of them take part.)
+        if (hist_ok && multi && T > 1) {
+            tc_fence_before();
+            cluster_sync();
+            if (s == 0 && tid == 0) *claim_ctr = 0;  // every split has made its last claim
+            const int nw = min(nsplit, T);
+            const int ds = (D + nsplit - 1) / nsplit;  // dimensions merged by this CTA
+            const int d0 = s * ds, nd = max(0, min(D, d0 + ds) - d0);
+            const uint32_t st_base = base + L::OFF_V;
+            for (int p = tid; p < C * nd; p += kThreads) {
+                const int h = p / nd, d = d0 + (p - h * nd);
+                float mr[16], lr[16], orr[16];
+#pragma unroll
+                for (int r = 0; r < 16; ++r) {
+                    if (r < nw) {
+                        const uint32_t rb = mapa_shared(st_base, static_cast<uint32_t>(r));
+                        const float2 ml = ld_dsmem_f32x2(rb + NH * D * 4 + h * 8);
+                        mr[r] = ml.x;
+                        lr[r] = ml.y;
+                        orr[r] = ld_dsmem_f32(rb + (h * D + d) * 4);
+                    }
+                }
+                float mm = -INFINITY;
+#pragma unroll
+                for (int r = 0; r < 16; ++r)
+                    if (r < nw && lr[r] > 0.f) mm = fmaxf(mm, mr[r]);
+                float l_tot = 0.f, acc = 0.f;
+#pragma unroll
+                for (int r = 0; r < 16; ++r)
+                    if (r < nw && lr[r] > 0.f) {
+                        const float wgt = fast_exp2(mr[r] - mm);
+                        l_tot = fmaf(wgt, lr[r], l_tot);
+                        acc = fmaf(wgt, orr[r], acc);
+                    }
+                out[orow[h] * D + d] = to_bf16(acc / l_tot);
+            }
+            cluster_sync();
+        }
+    } else if (hist_ok && multi) {
         bool contrib;  // (uniform over the CTA) this split wrote a partial and takes part
-        if (waves) {
+        if constexpr (WAVES) {
             tc_fence_before();
             __syncthreads();  // the staged result, and the producer's slot and claim count
             const int claimed = lastv[3];
@@ -942,14 +992,60 @@ __global__ void __launch_bounds__(kThreads, 1) decode_tc_kernel(
 
 }  // namespace
 
+// How many clusters of each size (2 .. 16 CTAs) of the one-wave decode fit on the device at
+// once, per device, set by configure_decode_tc; 0 where the size is refused.
+constexpr int kMaxDevices = 64;
+constexpr int kMaxCluster = 16;
+int g_cluster_fit[kMaxDevices][kMaxCluster + 1] = {};
+
+#define DECODE_TC_MODES(NHP, MAXTOK)                                                          \
+    decode_tc_kernel<NHP, MAXTOK, kModeGlobal>, decode_tc_kernel<NHP, MAXTOK, kModeCluster>, \
+        decode_tc_kernel<NHP, MAXTOK, kModeWaves>
+
 cudaError_t configure_decode_tc() {
     cudaError_t e = cudaSuccess;
-    for (auto fn : {decode_tc_kernel<8, 1, false>, decode_tc_kernel<16, 1, false>, decode_tc_kernel<8, kMaxTok, false>,
-                    decode_tc_kernel<16, kMaxTok, false>, decode_tc_kernel<8, 1, true>, decode_tc_kernel<16, 1, true>,
-                    decode_tc_kernel<8, kMaxTok, true>, decode_tc_kernel<16, kMaxTok, true>})
+    for (auto fn : {DECODE_TC_MODES(8, 1), DECODE_TC_MODES(16, 1), DECODE_TC_MODES(8, kMaxTok),
+                    DECODE_TC_MODES(16, kMaxTok)})
         if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, L::ALLOC);
-    return e;
+    for (auto fn : {decode_tc_kernel<8, 1, kModeCluster>, decode_tc_kernel<16, 1, kModeCluster>,
+                    decode_tc_kernel<8, kMaxTok, kModeCluster>, decode_tc_kernel<16, kMaxTok, kModeCluster>})
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    int dev = 0;
+    if (e == cudaSuccess) e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    // (the four cluster instantiations share the block size, shared memory and one block per SM)
+    for (int c = 2; c <= kMaxCluster; ++c) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(c), 1, 1);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = L::ALLOC;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = static_cast<unsigned>(c);
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, decode_tc_kernel<8, 1, kModeCluster>, &cfg) != cudaSuccess) {
+            n = 0;
+            cudaGetLastError();  // a refused size is never used
+        }
+        g_cluster_fit[dev][c] = n;
+    }
+    return cudaSuccess;
 }
+
+namespace {
+// Whether `items` clusters of nsplit CTAs all fit on the current device at once.
+bool decode_tc_clusters_fit(int nsplit, long long items) {
+    int dev = 0;
+    if (nsplit < 2 || nsplit > kMaxCluster || cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return false;
+    return items <= g_cluster_fit[dev][nsplit];
+}
+}  // namespace
 
 // Split counts.  With at most half as many (sequence, kv head, column group) items as SMs,
 // one wave of CTAs, min(16, floor(SMs / items)) splits per item, each starting with its own
@@ -1011,19 +1107,37 @@ cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint1
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = L::ALLOC;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
+    cudaLaunchAttribute attr[2];
+    unsigned n_attr = 0;
     // dependent launch only right after another decode step, or with producer_early
-    cfg.numAttrs = (after_decode || producer_early) ? 1 : 0;
-    if (ntok < 1 || ntok > kMaxTok || G > NH) return cudaErrorInvalidValue;
+    if (after_decode || producer_early) {
+        attr[n_attr].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[n_attr].val.programmaticStreamSerializationAllowed = 1;
+        ++n_attr;
+    }
     const bool w = s0 < nsplit;
-    const auto kernel =
-        ntok == 1 ? (G <= 8 ? (w ? decode_tc_kernel<8, 1, true> : decode_tc_kernel<8, 1, false>)
-                            : (w ? decode_tc_kernel<16, 1, true> : decode_tc_kernel<16, 1, false>))
-                  : (G * ntok <= 8 ? (w ? decode_tc_kernel<8, kMaxTok, true> : decode_tc_kernel<8, kMaxTok, false>)
-                                   : (w ? decode_tc_kernel<16, kMaxTok, true> : decode_tc_kernel<16, kMaxTok, false>));
+    // one wave: the splits of an item are one cluster (their merge) when a cluster per item
+    // fits on the device at once, else they merge through global memory
+    const int mode = w ? kModeWaves
+                       : (decode_tc_clusters_fit(nsplit, static_cast<long long>(s.n_kv_heads) * s.batch * ncg)
+                              ? kModeCluster
+                              : kModeGlobal);
+    if (mode == kModeCluster) {
+        attr[n_attr].id = cudaLaunchAttributeClusterDimension;
+        attr[n_attr].val.clusterDim.x = static_cast<unsigned>(nsplit);
+        attr[n_attr].val.clusterDim.y = 1;
+        attr[n_attr].val.clusterDim.z = 1;
+        ++n_attr;
+    }
+    cfg.attrs = attr;
+    cfg.numAttrs = n_attr;
+    if (ntok < 1 || ntok > kMaxTok || G > NH) return cudaErrorInvalidValue;
+    using Kernel = decltype(&decode_tc_kernel<8, 1, kModeGlobal>);
+    static const Kernel kernels[4][3] = {{DECODE_TC_MODES(8, 1)},
+                                         {DECODE_TC_MODES(16, 1)},
+                                         {DECODE_TC_MODES(8, kMaxTok)},
+                                         {DECODE_TC_MODES(16, kMaxTok)}};
+    const Kernel kernel = kernels[ntok == 1 ? (G <= 8 ? 0 : 1) : (G * ntok <= 8 ? 2 : 3)][mode];
     return cudaLaunchKernelEx(&cfg, kernel, maps.k, maps.v, q,
                               k_new, v_new, d_hist, hist_add, ntok, k_cache, v_cache, cos_tab, sin_tab, s.n_q_heads,
                               s.n_kv_heads, s.max_len, nsplit, scale_log2, part_o, part_ml, counters, out, err,
