@@ -500,7 +500,11 @@ def config_rows(dev, reps: int, graphs: bool):
     long-context stages one by one).  Each row is the median of `reps` calls timed with CUDA
     events around the stage call, inputs resident, L2 flushed (256 MB write + 256 MB read)
     before every call and a short GPU sleep in front of it, so the host's launch cost stays
-    outside the events.  graphs: also time each decode step replayed from a CUDA graph."""
+    outside the events.  CUDA events on a GB300 tick in steps of 2.048 us and read about
+    4.5 us around an empty kernel, which dominates the small rows; so every row also has
+    `loop_ms`: the same call replayed 10 times from one CUDA graph, each time after the L2
+    flush, less the same graph with the flushes alone, per call (the rates in `loop_*`).
+    graphs: also time each decode step replayed from a CUDA graph."""
     import torch
     from paper_2607_15865_gb300.attention import Attention
     from synthetic.workloads import Shape
@@ -528,6 +532,34 @@ def config_rows(dev, reps: int, graphs: bool):
         torch.cuda.synchronize()
         return sorted(a.elapsed_time(b) for a, b in evs)[reps // 2]  # median, ms
 
+    def loop_ms(fn, n=10):
+        # per call, in a CUDA graph of n (L2 flush, call) pairs, less the flushes alone (ms)
+        t = []
+        for with_call in (False, True):
+            side = torch.cuda.Stream()
+            side.wait_stream(torch.cuda.current_stream())
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.stream(side), torch.cuda.graph(gr, stream=side):
+                for _ in range(n):
+                    flush_w.zero_()
+                    flush_r.sum()
+                    if with_call:
+                        fn()
+            torch.cuda.current_stream().wait_stream(side)
+            gr.replay()
+            torch.cuda.synchronize()
+            ts = []
+            for _ in range(5):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                gr.replay()
+                b.record()
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(b))
+            t.append(sorted(ts)[2])
+            del gr
+        return max(t[1] - t[0], 0.0) / n
+
     rows = []
     gen = torch.Generator(device=dev).manual_seed(1)
     cases = [("7B prefill 512", w.PREFILL_7B, 0, 512),
@@ -543,8 +575,11 @@ def config_rows(dev, reps: int, graphs: bool):
         vc = rnd((sh.batch, sh.n_kv_heads, sh.max_len, sh.head_dim), gen)
         out = torch.empty_like(q)
         ms = time_calls(lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out), reps)
-        tf = attn_flops(sh, prefill_pairs(hist, chunk)) / (ms * 1e-3) / 1e12
-        rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak})
+        lms = loop_ms(lambda: attn.prefill_kv(q, k, v, hist, kc, vc, out))
+        fl = attn_flops(sh, prefill_pairs(hist, chunk))
+        tf, ltf = fl / (ms * 1e-3) / 1e12, fl / (lms * 1e-3) / 1e12
+        rows.append({"config": name, "ms": ms, "TFLOP/s": tf, "frac_tensor": tf / tc_peak,
+                     "loop_ms": lms, "loop_TFLOP/s": ltf, "loop_frac_tensor": ltf / tc_peak})
         attn.close()
     for bsz in w.DECODE_BATCHES:
         sh = w.decode_shape(bsz)
@@ -565,8 +600,10 @@ def config_rows(dev, reps: int, graphs: bool):
                 it[0] += 1
                 attn.decode(q, k, v, hl, kc, vc, out)
             ms = time_calls(call, reps)
-            gbs = decode_bytes(sh, hist) / (ms * 1e-3) / 1e9
-            row = {"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm}
+            lms = loop_ms(call)
+            gbs, lgbs = decode_bytes(sh, hist) / (ms * 1e-3) / 1e9, decode_bytes(sh, hist) / (lms * 1e-3) / 1e9
+            row = {"config": f"decode B{bsz} hist {hist}", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm,
+                   "loop_ms": lms, "loop_GB/s": lgbs, "loop_frac_hbm": lgbs / hbm}
             rows.append(row)
             if not graphs:
                 continue
@@ -605,11 +642,13 @@ def config_rows(dev, reps: int, graphs: bool):
     lens = np.random.default_rng(16).integers(64, 8192, sh.batch).astype(np.int32)
     hl = torch.from_numpy(lens).to(dev)
     ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), reps)
+    lms = loop_ms(lambda: attn.decode(q, k, v, hl, kc, vc, out))
     one = Shape("one", 1, sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.max_len, sh.rope_theta)
     byts = sum(decode_bytes(one, int(h)) for h in lens)
-    gbs = byts / (ms * 1e-3) / 1e9
+    gbs, lgbs = byts / (ms * 1e-3) / 1e9, byts / (lms * 1e-3) / 1e9
     rows.append({"config": f"decode B16 lengths spread over 64..8191 (mean {int(lens.mean())})", "ms": ms,
-                 "GB/s": gbs, "frac_hbm": gbs / hbm})
+                 "GB/s": gbs, "frac_hbm": gbs / hbm, "loop_ms": lms, "loop_GB/s": lgbs,
+                 "loop_frac_hbm": lgbs / hbm})
     attn.close()
     del kc, vc
     attn = Attention.for_shape(S)
@@ -619,8 +658,10 @@ def config_rows(dev, reps: int, graphs: bool):
     out = torch.empty_like(q)
     hl = torch.full((1,), w.LONG_DECODE_HIST, dtype=torch.int32, device=dev)
     ms = time_calls(lambda: attn.decode(q, k, v, hl, kc, vc, out), reps)
-    gbs = DECODE_BYTES / (ms * 1e-3) / 1e9
-    rows.append({"config": "long decode hist 32767", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm})
+    lms = loop_ms(lambda: attn.decode(q, k, v, hl, kc, vc, out))
+    gbs, lgbs = DECODE_BYTES / (ms * 1e-3) / 1e9, DECODE_BYTES / (lms * 1e-3) / 1e9
+    rows.append({"config": "long decode hist 32767", "ms": ms, "GB/s": gbs, "frac_hbm": gbs / hbm,
+                 "loop_ms": lms, "loop_GB/s": lgbs, "loop_frac_hbm": lgbs / hbm})
     attn.close()
     del kc, vc
     return rows, time_calls, rnd, gen
@@ -846,6 +887,8 @@ def run_sweep(args):
     for r in rows:
         extra = f"{r['TFLOP/s']:8.1f} TFLOP/s {100*r['frac_tensor']:5.1f}%" if "TFLOP/s" in r else \
             f"{r['GB/s']:8.1f} GB/s    {100*r['frac_hbm']:5.1f}%"
+        if "loop_ms" in r:
+            extra += f"   (flushed graph loop: {r['loop_ms']*1e3:6.1f} us)"
         if "graph_ms" in r:
             extra += f"   (CUDA graph: {r['graph_ms']*1e3:6.1f} us {r['graph_GB/s']:7.1f} GB/s)"
         print(f"{r['config']:36s} {r['ms']*1e3:9.1f} us {extra}", file=sys.stderr)
