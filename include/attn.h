@@ -36,7 +36,7 @@
  *
  * Ownership.  The caller owns every device buffer passed to a call.  The
  * context owns only its own device memory: the RoPE tables (2 x max_len x
- * head_dim/2 floats, held twice: position-major and pair-major), the decode
+ * head_dim/2 floats, held twice: position-major and in groups of four pairs), the decode
  * split-KV partials (batch x n_q_heads x 256 x (head_dim + 2) floats) and counters
  * (5 x batch x n_kv_heads x 16 + 1 ints: one set per column group of the multi-token
  * decode), the prefill partials of split work (SM count x 256 x (head_dim + 2)

@@ -32,7 +32,7 @@ struct attn_ctx {
     int nsplit_max;
     float* d_cos;       // RoPE tables [max_len][D/2]
     float* d_sin;
-    float* d_cos_t;     // the same, pair-major [D/2][max_len] (flash_fwd's q rows)
+    float* d_cos_t;     // the same in groups of four pairs, [D/8][max_len][4] (flash_fwd's q rows)
     float* d_sin_t;
     float* d_part_o;
     float* d_part_ml;
@@ -238,8 +238,9 @@ int attn_create(const attn_cfg* cfg, attn_ctx** out) {
             const double ang = static_cast<double>(p) * inv_freq;
             hc[static_cast<size_t>(p) * half + j] = static_cast<float>(std::cos(ang));
             hs[static_cast<size_t>(p) * half + j] = static_cast<float>(std::sin(ang));
-            hct[static_cast<size_t>(j) * cfg->max_len + p] = hc[static_cast<size_t>(p) * half + j];
-            hst[static_cast<size_t>(j) * cfg->max_len + p] = hs[static_cast<size_t>(p) * half + j];
+            const size_t q4 = (static_cast<size_t>(j / 4) * cfg->max_len + p) * 4 + j % 4;
+            hct[q4] = hc[static_cast<size_t>(p) * half + j];
+            hst[q4] = hs[static_cast<size_t>(p) * half + j];
         }
     }
     const size_t part_rows = static_cast<size_t>(cfg->batch) * cfg->n_q_heads * c->nsplit_max;

@@ -29,8 +29,8 @@
 // the softmax warpgroup may rescale O_T before it hands P over.  O is rescaled lazily
 // (only when the running max grows by more than 2^8, exact in value).
 // Per row: RoPE of the q row in shared memory before the first MMA (cos/sin
-// gathered by position from pair-major copies of the tables, Section 4.6.2, float
-// arithmetic and bf16 rounding as K1),
+// gathered by position from copies of the tables laid out in groups of four pairs,
+// Section 4.6.2, float arithmetic and bf16 rounding as K1),
 // scores from TMEM, causal mask by index compare on diagonal tiles (no mask
 // tensor), online softmax in the log2 domain, O / l -> bf16 -> out.
 // Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its
@@ -212,9 +212,12 @@ __device__ __forceinline__ int unit_of(int lin, const Sched& sc) {
 }
 
 // RoPE tables of one position in registers: cos/sin of pairs j = 0 .. D/2-1.  They are
-// read from pair-major copies of the tables ([D/2][max_len]: entry (j, p) at
-// j * stride + p), so that the 32 threads of a warp -- 32 consecutive positions --
-// read one coalesced line per pair, and are loaded before the q tile lands.
+// read from copies of the tables in groups of four pairs ([D/8][max_len][4]: entry (j, p)
+// at ((j / 4) * stride + p) * 4 + j % 4), so that a thread loads four pairs at once and
+// the 32 threads of a warp -- 32 consecutive positions -- read 512 contiguous bytes per
+// load: D/4 loads per thread instead of D with one float per pair, which took about 2 us
+// per work unit (the loads in flight, not the bytes, were the limit).  They are loaded
+// before the q tile lands.
 template <int D>
 struct RopeRow {
     float c[D / 2], s[D / 2];
@@ -223,10 +226,20 @@ struct RopeRow {
 template <int D>
 __device__ __forceinline__ void rope_load(RopeRow<D>& t, int pos, const float* __restrict__ cos_t,
                                           const float* __restrict__ sin_t, int stride) {
+    const float4* c4 = reinterpret_cast<const float4*>(cos_t) + pos;
+    const float4* s4 = reinterpret_cast<const float4*>(sin_t) + pos;
 #pragma unroll
-    for (int j = 0; j < D / 2; ++j) {
-        t.c[j] = __ldg(cos_t + static_cast<size_t>(j) * stride + pos);
-        t.s[j] = __ldg(sin_t + static_cast<size_t>(j) * stride + pos);
+    for (int g = 0; g < D / 8; ++g) {
+        const float4 c = __ldg(c4 + static_cast<size_t>(g) * stride);
+        const float4 s = __ldg(s4 + static_cast<size_t>(g) * stride);
+        t.c[4 * g] = c.x;
+        t.c[4 * g + 1] = c.y;
+        t.c[4 * g + 2] = c.z;
+        t.c[4 * g + 3] = c.w;
+        t.s[4 * g] = s.x;
+        t.s[4 * g + 1] = s.y;
+        t.s[4 * g + 2] = s.z;
+        t.s[4 * g + 3] = s.w;
     }
 }
 

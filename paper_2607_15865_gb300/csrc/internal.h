@@ -54,8 +54,8 @@ __device__ __forceinline__ int fdiv(int n, const FastDiv& f) {
 // k and v into cache slots hist+i (Listing 2 "Concat"; Section 4.6.3).
 // hist comes from `d_hist[b]` when non-null (decode), else `hist` for every b.  k and v
 // hold `chunk` tokens of each sequence, sequence b starting at token b * seq_stride.
-// cos_t / sin_t (the pair-major table copies, or null): their lines for the chunk's
-// positions are prefetched into L2 for K2's rotation of q.
+// cos_t / sin_t (the table copies in groups of four pairs, [D/8][max_len][4], or null):
+// their lines for the chunk's positions are prefetched into L2 for K2's rotation of q.
 cudaError_t launch_rope_append(const Shape& s, const uint16_t* k, const uint16_t* v, int hist,
                                const int32_t* d_hist, int chunk, int seq_stride, const float* cos_tab,
                                const float* sin_tab, const float* cos_t, const float* sin_t, uint16_t* k_cache,
@@ -73,7 +73,8 @@ cudaError_t configure_flash_fwd();
 // Work is split across num_sms persistent CTAs; items of the last, partial round are
 // cut into KV pieces whose partials go to ws_o [num_sms*256, D] / ws_ml [num_sms*256, 2]
 // and are merged by a second kernel (then *n_launched = 2).
-// cos_t / sin_t: the RoPE tables pair-major, [D/2][max_len] (entry (j, p) at j * max_len + p).
+// cos_t / sin_t: the RoPE tables in groups of four pairs, [D/8][max_len][4] (entry (j, p) at
+// ((j / 4) * max_len + p) * 4 + j % 4).
 // out holds `chunk` tokens of each sequence, sequence b starting at token b * s_stride (the
 // q map carries the same stride).
 cudaError_t launch_flash_fwd(const Shape& s, const FlashMaps& maps, int hist, int chunk, int s_stride,

@@ -54,13 +54,16 @@ __global__ void __launch_bounds__(128) rope_append_kernel(const uint16_t* __rest
         }
     }
     const int p = h0 + i;
-    // Warm L2 with the lines of the pair-major tables (cos_t, sin_t: [D/2][max_len]) that the
-    // attention kernel's softmax threads read to rotate the q rows of this chunk: the CTA of
-    // every 32nd position (and the first) touches one line per pair and table.
-    if (cos_t != nullptr && b == 0 && threadIdx.x < 2 * HALF && (i == 0 || (p & 31) == 0)) {
+    // Warm L2 with the lines of the table copies in groups of four pairs (cos_t, sin_t:
+    // [D/8][max_len][4]) that the attention kernel's softmax threads read to rotate the q
+    // rows of this chunk: the CTA of every 32nd position (and the first) touches the four
+    // 128-byte lines of the 32 positions from p & ~31 in every group and table (a line
+    // that starts past the table's end is skipped).
+    const int p32 = p & ~31, line = static_cast<int>(threadIdx.x) & 3;
+    if (cos_t != nullptr && b == 0 && threadIdx.x < D && (i == 0 || (p & 31) == 0) && p32 + 8 * line < max_len) {
         const float* tab = threadIdx.x < HALF ? cos_t : sin_t;
-        const int j = static_cast<int>(threadIdx.x) % HALF;
-        asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + static_cast<size_t>(j) * max_len + (p & ~31)));
+        const int g = (static_cast<int>(threadIdx.x) % HALF) / 4;
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + (static_cast<size_t>(g) * max_len + p32) * 4 + 32 * line));
     }
     const int n_rope = Hkv * ROPE_UNITS;
     const int n_units = n_rope + Hkv * COPY_UNITS;
