@@ -357,7 +357,7 @@ int run_decode(attn_ctx* c, const uint16_t* q, const uint16_t* k, const uint16_t
     const int G = c->cfg.n_q_heads / c->cfg.n_kv_heads;
     if (tc ? static_cast<long>(c->cfg.batch) * ncg > 65535 : static_cast<long>(c->cfg.n_kv_heads) * ((G + 7) / 8) > 65535)
         return ATTN_EINVAL;
-    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms, ncg), c->nsplit_max / ntok)
+    const int nsplit = tc ? std::min(attn::decode_tc_num_splits(c->shape, c->num_sms, ncg, ntok), c->nsplit_max / ntok)
                           : attn::decode_num_splits(c->shape, c->num_sms, c->nsplit_max);
     cudaError_t e = timed(c, ATTN_KERNEL_DECODE_SPLIT, st, [&](int*) {
         if (tc)

@@ -122,7 +122,9 @@ int decode_tc_column_groups(int G, int ntok);
 // Ints of the counter array for `items` items: claims, slots and visits, then 64-bit
 // (contributors, tiles done) words from an even offset.
 inline long long decode_tc_counter_ints(long long items) { return 3 * items + 1 + 2 * items; }
-int decode_tc_num_splits(const Shape& s, int num_sms, int ncg = 1);
+// Splits per item for a decode of ntok new tokens with ncg column groups (after the
+// configuration, which measures the cluster sizes that fit).
+int decode_tc_num_splits(const Shape& s, int num_sms, int ncg = 1, int ntok = 1);
 cudaError_t make_decode_tc_maps(PFN_encodeTiled encode, const Shape& s, const uint16_t* k_cache,
                                 const uint16_t* v_cache, DecodeMaps* maps);
 cudaError_t launch_decode_tc(const Shape& s, const DecodeMaps& maps, const uint16_t* q, const uint16_t* k_new,
