@@ -1067,14 +1067,16 @@ int decode_tc_num_splits(const Shape& s, int num_sms, int ncg, int ntok) {
     const long max_tiles = std::max(1L, static_cast<long>((s.max_len + KT - 1) / KT));
     long ns = 2 * items > num_sms ? kWaveSplits : std::min<long>(kMaxWaveSplits1, num_sms / items);
     ns = std::min(ns, std::min(max_tiles, 256L));
-    // Several new tokens: the last split of an item merges ns partials of up to 16 columns in
-    // the global merge, but a cluster spreads the merge over its CTAs; from 128 partial rows
-    // (splits x columns) on, fewer splits whose clusters fit on the device pay for their
-    // longer streams (B1 Hq32, 8188 history tokens: 4 tokens 31.5 -> 25.3 us, 8 tokens
-    // 34.2 -> 31.9 us; Hq40 over 32765, 3 tokens 44.1 -> 41.6 us; but 8 tokens there, 6
-    // splits x 16 columns, went from 68.3 to 75.8 us with 5).
+    // The last split of an item merges ns partials of up to 16 columns in the global merge,
+    // while a cluster spreads the merge over its CTAs.  Fewer splits whose clusters fit on the
+    // device pay for their longer streams with several new tokens from 128 partial rows
+    // (splits x columns) on (B1 Hq32, 8188 history tokens: 4 tokens 31.5 -> 25.3 us, 8 tokens
+    // 34.2 -> 31.9 us; Hq40 over 32765, 3 tokens 44.1 -> 41.6 us; but 8 tokens there, 6 splits x
+    // 16 columns, went from 68.3 to 75.8 us with 5), and with one token when the cache holds
+    // at most 64 tiles (B1 Hq32 over 1024 and 4096 tokens: 11.8 -> 10.3 us and 14.1 -> 12.9 us;
+    // at 32767 tokens 12 splits took 32.5 us against 29.5 us with 16).
     const long cols = std::min<long>(NH, static_cast<long>(s.n_q_heads / s.n_kv_heads) * ntok);
-    if (ntok > 1 && 2 * items <= num_sms && ns * cols >= 128)
+    if (2 * items <= num_sms && ((ntok > 1 && ns * cols >= 128) || (ntok == 1 && max_tiles <= 64)))
         while (ns > 2 && !decode_tc_clusters_fit(static_cast<int>(ns), items)) --ns;
     return static_cast<int>(std::max(1L, ns));
 }
