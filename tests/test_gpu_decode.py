@@ -132,19 +132,22 @@ def test_decode_multiwave_mixed_lengths(torch, name, shape):
 
 # One wave of splits whose items (sequence, kv head) fit as one thread-block cluster each
 # merge through distributed shared memory, the others through global memory.  On a GB300
-# (152 SMs, one 211 KB CTA per SM: 7 clusters of 16 CTAs fit at once, 15 of 8, 23 of 6,
-# 28 of 5, 36 of 4, 76 of 2) these batches (G = 8 or 16, one kv head, so items = batch) take
-# splits = min(16, 152 / items, tiles): clusters of 16, 16 (exactly 7), 8, 6, 5, 2, and the
-# global merge at 16 splits (8 items) and 4 splits (38 items).  Lengths are mixed, so some
-# items have fewer tiles than splits and short ones a single tile.
+# (152 SMs, one 211 KB CTA per SM: 7 clusters of 16 CTAs fit at once, 8 of 12, 15 of 8, 23 of
+# 6, 28 of 5, 36 of 4, 46 of 3, 76 of 2) these batches (G = 8 or 16, one kv head, so items =
+# batch) take splits = min(16, 152 / items, tiles), lowered to a cluster size that fits when
+# the cache holds at most 64 tiles: clusters of 16, 16 (exactly 7), 12, 8, 6, 5, 3 and 2, and
+# the global merge at 16 and 4 splits over 65 tiles.  Lengths are mixed, so some items have
+# fewer tiles than splits and short ones a single tile.
 ONEWAVE_MERGES = [
     ("b1_g8_cluster16", Shape("ow1", 1, 8, 1, 128, 2048, 1.0e4)),
     ("b7_g8_cluster16", Shape("ow7", 7, 8, 1, 128, 2048, 1.0e4)),
-    ("b8_g8_global16", Shape("ow8", 8, 8, 1, 128, 2048, 1.0e4)),
+    ("b8_g8_cluster12", Shape("ow8", 8, 8, 1, 128, 2048, 1.0e4)),
+    ("b8_g8_global16", Shape("ow8g", 8, 8, 1, 128, 8320, 1.0e4)),
     ("b10_g8_cluster8", Shape("ow10", 10, 8, 1, 128, 1024, 1.0e4)),
     ("b22_g8_cluster6", Shape("ow22", 22, 8, 1, 128, 2048, 1.0e4)),
     ("b28_g8_cluster5", Shape("ow28", 28, 8, 1, 128, 2048, 1.0e4)),
-    ("b38_g8_global4", Shape("ow38", 38, 8, 1, 128, 2048, 1.0e4)),
+    ("b38_g8_cluster3", Shape("ow38", 38, 8, 1, 128, 2048, 1.0e4)),
+    ("b38_g8_global4", Shape("ow38g", 38, 8, 1, 128, 8320, 1.0e4)),
     ("b76_g8_cluster2", Shape("ow76", 76, 8, 1, 128, 512, 1.0e4)),
     ("b5_g16_cluster16", Shape("ow5g16", 5, 16, 1, 128, 2048, 1.0e4)),
 ]
