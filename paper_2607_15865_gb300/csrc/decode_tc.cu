@@ -35,13 +35,20 @@
 //              copies of the tiles that hold those slots (zeroing the V rows past the
 //              last new slot: slots past it may hold anything, and 0 * NaN would poison
 //              O), so the MMA itself produces the new keys' scores.
-// Merge: a split that took all T tiles writes the normalised output.  Otherwise each
-// split that took tiles writes its partial (m, l, acc[D]) per column to a slot it took
-// from a counter, then adds (1 contributor, its tile count) to the item's done word; the
-// split whose addition completes T tiles merges the slots:
-//   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
-// Every wait is bounded; on expiry the CTA records kDevErrTimeout, lets its copies
-// and MMAs finish, releases TMEM and still takes part in the merge count.
+// Merge of the splits that took tiles, each holding a partial (m, l, acc[D]) per column:
+//   out = sum_s 2^(m_s - M) acc_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
+// in one of three ways, each its own instantiation (MODE):
+//   one wave, global: split s writes its partial at slot s and counts itself; the last
+//     of the min(nsplit, T) splits with tiles merges;
+//   one wave, cluster (when a cluster per item fits on the device at once): the item's
+//     splits are one thread-block cluster; each stages its partial in shared memory and,
+//     after a cluster barrier, merges a share of the dimensions from its peers' staging;
+//   several waves: a split writes its partial to a slot it takes from a counter and adds
+//     (1 contributor, its tile count) to the item's done word; the split whose addition
+//     completes T tiles merges the slots.
+// A split that took all T tiles writes the normalised output itself.  Every wait is
+// bounded; on expiry the CTA records kDevErrTimeout, lets its copies and MMAs finish,
+// releases TMEM and still takes part in the merge (its count, or the cluster barriers).
 #include <cuda_bf16.h>
 
 #include <algorithm>
