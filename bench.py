@@ -924,7 +924,9 @@ def run_sweep(args):
 def run_stage(args):
     """Runs one stage of the long-context workload --warmup + --reps times on random
     device inputs (no timing, no JSON line): the launch pattern that profiler captures
-    of a single kernel use.  --hist / --chunk override the stage's sizes."""
+    of a single kernel use.  --hist / --chunk override the stage's sizes; --shape 7b or
+    pkv512 takes the 7B-class prefill (Hq28 Hkv4, 512 tokens) or the prefill_kv of 512
+    tokens over 1536 (Hq32 Hkv8) instead."""
     import torch
 
     import __graft_entry__
@@ -935,19 +937,24 @@ def run_stage(args):
     st = STAGES[args.stage]
     hist = st["hist"] if args.hist is None else args.hist
     chunk = st["chunk"] if args.chunk is None else args.chunk
+    shape = S
+    if args.shape == "7b":
+        shape, hist, chunk = w.PREFILL_7B, 0, 512
+    elif args.shape == "pkv512":
+        shape, hist, chunk = w.PREFILL_KV, 1536, 512
     g = torch.Generator(device=dev).manual_seed(3)
 
     def rnd(*shape):
         return (torch.randn(*shape, device=dev, generator=g) * 0.0884).to(torch.bfloat16)
 
-    attn = Attention.for_shape(S)
-    kc = rnd(S.batch, S.n_kv_heads, S.max_len, S.head_dim)
-    vc = rnd(S.batch, S.n_kv_heads, S.max_len, S.head_dim)
-    q = rnd(S.batch, chunk, S.n_q_heads, S.head_dim)
-    k = rnd(S.batch, chunk, S.n_kv_heads, S.head_dim)
-    v = rnd(S.batch, chunk, S.n_kv_heads, S.head_dim)
+    attn = Attention.for_shape(shape)
+    kc = rnd(shape.batch, shape.n_kv_heads, shape.max_len, shape.head_dim)
+    vc = rnd(shape.batch, shape.n_kv_heads, shape.max_len, shape.head_dim)
+    q = rnd(shape.batch, chunk, shape.n_q_heads, shape.head_dim)
+    k = rnd(shape.batch, chunk, shape.n_kv_heads, shape.head_dim)
+    v = rnd(shape.batch, chunk, shape.n_kv_heads, shape.head_dim)
     out = torch.empty_like(q)
-    hl = torch.full((S.batch,), hist, dtype=torch.int32, device=dev)
+    hl = torch.full((shape.batch,), hist, dtype=torch.int32, device=dev)
     for _ in range(args.warmup + args.reps):
         if args.stage == "decode":
             attn.decode(q, k, v, hl, kc, vc, out)
@@ -1076,6 +1083,8 @@ def main():
     ap.add_argument("--reps", type=int, default=2)
     ap.add_argument("--hist", type=int)
     ap.add_argument("--chunk", type=int)
+    ap.add_argument("--shape", choices=("long", "7b", "pkv512"), default="long",
+                    help="with --stage: the long-context shape, the 7B-class prefill 512 or prefill_kv 512 over 1536")
     ap.add_argument("--w4", help="M,N,K: run only the W4BF16 GEMV of that shape (for profiler captures)")
     ap.add_argument("--layer", help="B,HIST: run only the W4BF16 decode block (for profiler captures)")
     ap.add_argument("--gemm", help="T,N,K: run only the W4BF16 GEMM of that shape (for profiler captures)")
